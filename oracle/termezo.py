@@ -1,0 +1,231 @@
+"""TerMeZO mask selection and masked two-sided SPSA step -- oracle.
+
+TEST INFRASTRUCTURE ONLY (see the package header).
+
+Dense restatement of Algorithm 1 (App. C) with K = 1 perturbation, acting on
+the latent weights w only (theta held fixed):
+
+* ``registry``      -- the global order of the ternary linear projections:
+  layer 0..L-1, within a layer q, k, v, o, gate, up, down, each a row-major
+  [N_out, K_in] matrix.  w is their concatenation.
+* ``initial_mask``  -- Eq. 4 and the first two lines of Algorithm 1: tau_0
+  per projection, distances of all weights of all projections, xi_0 the
+  lower rho_0-quantile of these distances (global, across layers), S_0 the
+  weights with d <= xi_0.  Reading: k0 = floor(rho_0 * d) weights are kept
+  exactly, ties at xi_0 broken towards the lower global index, so that
+  |S_0| = k0.
+* ``shrink``        -- Eq. 5: tau_t recomputed on w_t, S_t keeps the members of
+  S_{t-1} with d <= xi_0 (xi_0 fixed).
+* ``masked_spsa``   -- the inner loop of Algorithm 1 for any objective F:
+  w <- w + eps m.z; F+; w <- w - 2 eps m.z; F-; w <- w + eps m.z (restore);
+  g = (F+ - F-) / (2 eps) (Eq. 1 projected onto z); z re-drawn from the seed;
+  w <- w - lr g (m.z).  All latent arithmetic is float32 (the stored
+  precision of the latents), with e = fl32(eps z) and c = fl32(lr g).
+* ``step``          -- one TerMeZO iteration on a BitNet objective: shrink
+  (t >= 1), masked SPSA with the dense requantisation of every projection
+  (tau recomputed from the perturbed latents, Eq. 2) before each forward,
+  and the counters of Eq. 11 (k_t, codes that change between the two
+  evaluations) plus the invariant that frozen weights keep their code.
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, field
+
+import numpy as np
+
+from . import bitnet, philox, ternary
+
+
+@dataclass(frozen=True)
+class Proj:
+    layer: int
+    name: str
+    N: int
+    K: int
+    base: int
+
+    @property
+    def n(self) -> int:
+        return self.N * self.K
+
+
+def registry(cfg):
+    D, F = cfg.hidden, cfg.ffn
+    hd = D // cfg.heads
+    Hq, Hkv = cfg.heads * hd, cfg.kv_heads * hd
+    shapes = [("q", Hq, D), ("k", Hkv, D), ("v", Hkv, D), ("o", D, Hq),
+              ("gate", F, D), ("up", F, D), ("down", D, F)]
+    out, base = [], 0
+    for l in range(cfg.layers):
+        for name, N, K in shapes:
+            out.append(Proj(l, name, N, K, base))
+            base += N * K
+    return out
+
+
+def single_registry(N: int, K: int):
+    """Registry of one projection (the BitLinear-op workload)."""
+    return [Proj(0, "w", N, K, 0)]
+
+
+def views(w: np.ndarray, reg):
+    return [w[p.base:p.base + p.n] for p in reg]
+
+
+def thresholds(w: np.ndarray, reg):
+    """Per projection (gamma, tau, s_w) on the dense latents w."""
+    gam = [ternary.absmean(v) for v in views(w, reg)]
+    return (np.array(gam, dtype=np.float32),
+            np.array([ternary.threshold(g) for g in gam], dtype=np.float32),
+            np.array([ternary.weight_scale(g) for g in gam], dtype=np.float32))
+
+
+def all_distances(w: np.ndarray, reg, tau) -> np.ndarray:
+    return np.concatenate([ternary.distance(v, tau[j]) for j, v in enumerate(views(w, reg))])
+
+
+def requantize(w: np.ndarray, reg):
+    """Dense codes of every projection at its own tau (Eq. 2)."""
+    _, tau, sw = thresholds(w, reg)
+    codes = np.concatenate([ternary.quantize(v, tau[j]) for j, v in enumerate(views(w, reg))])
+    return codes, tau, sw
+
+
+def keep_count(rho0: float, d: int) -> int:
+    if not (0.0 < rho0 <= 1.0):
+        raise ValueError("rho_0 must lie in (0, 1]")
+    return int(math.floor(float(rho0) * float(d)))
+
+
+def initial_mask(w: np.ndarray, reg, rho0: float):
+    """Returns (S_0 as sorted int64 global indices, xi_0 float32, k0, tau_0)."""
+    _, tau, _ = thresholds(w, reg)
+    d = all_distances(w, reg, tau)
+    k0 = keep_count(rho0, d.size)
+    if k0 == 0:
+        return np.zeros(0, dtype=np.int64), np.float32(0.0), 0, tau
+    order = np.argsort(d, kind="stable")  # equal distances: lower index first
+    sel = np.sort(order[:k0]).astype(np.int64)
+    xi0 = np.float32(d[order[k0 - 1]])
+    return sel, xi0, k0, tau
+
+
+def shrink(w: np.ndarray, reg, active: np.ndarray, xi0):
+    """Eq. 5: members of S_{t-1} whose distance at tau_t is <= xi_0."""
+    _, tau, _ = thresholds(w, reg)
+    d = all_distances(w, reg, tau)
+    keep = d[active] <= np.float32(xi0)
+    return active[keep], tau
+
+
+def masked_spsa(w: np.ndarray, active: np.ndarray, z: np.ndarray, eps, lr, objective):
+    """One K = 1 pass of Algorithm 1's inner loops for objective(w) -> float.
+
+    Returns (w_next, F+, F-, g, w_plus, w_minus, w_restored)."""
+    eps = np.float32(eps)
+    e = (eps * z.astype(np.float32)).astype(np.float32)
+    w_plus = w.copy()
+    w_plus[active] = (w[active] + e).astype(np.float32)
+    f_plus = float(objective(w_plus))
+    w_minus = w_plus.copy()
+    w_minus[active] = (w_plus[active] - (np.float32(2.0) * e)).astype(np.float32)
+    f_minus = float(objective(w_minus))
+    w_rest = w_minus.copy()
+    w_rest[active] = (w_minus[active] + e).astype(np.float32)
+    g = (f_plus - f_minus) / (2.0 * float(eps))
+    c = np.float32(float(np.float32(lr)) * g)
+    w_next = w_rest.copy()
+    w_next[active] = (w_rest[active] - (c * z.astype(np.float32)).astype(np.float32)).astype(np.float32)
+    return w_next, f_plus, f_minus, g, w_plus, w_minus, w_rest
+
+
+@dataclass
+class State:
+    """Dense oracle state of a TerMeZO run."""
+    w: np.ndarray                 # dense fp32 latents w_t
+    reg: list
+    active: np.ndarray            # S_t, sorted global indices
+    xi0: np.float32
+    k0: int
+    frozen_code: np.ndarray       # code each weight had when it froze (int8)
+    t: int = 0
+    log: list = field(default_factory=list)
+
+
+def build(w0: np.ndarray, reg, rho0: float) -> State:
+    active, xi0, k0, tau0 = initial_mask(w0, reg, rho0)
+    codes0 = np.concatenate([ternary.quantize(v, tau0[j]) for j, v in enumerate(views(w0, reg))])
+    return State(w=w0.astype(np.float32).copy(), reg=reg, active=active, xi0=xi0,
+                 k0=k0, frozen_code=codes0)
+
+
+def near_threshold(w_act: np.ndarray, tau_act: np.ndarray, sw_act: np.ndarray) -> np.ndarray:
+    """Active latents within 1e-5 * s_w of +-tau (codes excluded from
+    bit-exact comparison)."""
+    dist = np.abs(np.abs(w_act.astype(np.float64)) - tau_act.astype(np.float64))
+    return dist < 1e-5 * sw_act.astype(np.float64)
+
+
+def _tensor_of(reg, idx):
+    bases = np.array([p.base for p in reg], dtype=np.int64)
+    return np.searchsorted(bases, idx, side="right") - 1
+
+
+def step(state: State, loss_fn, seed: int, eps, lr):
+    """One TerMeZO iteration (Algorithm 1, K = 1) on loss_fn(codes, s_w) ->
+    float, where codes are the dense per-projection int8 arrays."""
+    reg = state.reg
+    if state.t >= 1:
+        kept, tau_t = shrink(state.w, reg, state.active, state.xi0)
+        dropped = np.setdiff1d(state.active, kept)
+        if dropped.size:
+            tj = _tensor_of(reg, dropped)
+            state.frozen_code[dropped] = ternary.quantize(state.w[dropped], tau_t[tj])
+        state.active = kept
+    active = state.active
+    z = philox.normal(seed, active) if active.size else np.zeros(0, np.float32)
+    passes = {}
+
+    def objective(wp):
+        codes, tau, sw = requantize(wp, reg)
+        frozen = np.ones(wp.size, dtype=bool)
+        frozen[active] = False
+        mism = int(np.count_nonzero(codes[frozen] != state.frozen_code[frozen]))
+        split = [codes[p.base:p.base + p.n].reshape(p.N, p.K) for p in reg]
+        key = "plus" if "plus" not in passes else "minus"
+        tj = _tensor_of(reg, active)
+        passes[key] = dict(codes=codes, tau=tau, sw=sw, frozen_mismatch=mism,
+                           near=near_threshold(wp[active], tau[tj], sw[tj]))
+        return loss_fn(split, sw)
+
+    w_next, fp, fm, g, w_plus, w_minus, w_rest = masked_spsa(state.w, active, z, eps, lr, objective)
+    cp = passes["plus"]["codes"][active].astype(np.int64)
+    cm = passes["minus"]["codes"][active].astype(np.int64)
+    rec = dict(t=state.t, seed=seed, loss_plus=fp, loss_minus=fm, g=g, k=int(active.size),
+               n_flipped=int(np.count_nonzero(cp != cm)),
+               n_jumps=int(np.count_nonzero(np.abs(cp - cm) == 2)),
+               frozen_mismatch=passes["plus"]["frozen_mismatch"] + passes["minus"]["frozen_mismatch"],
+               tau_plus=passes["plus"]["tau"], tau_minus=passes["minus"]["tau"],
+               codes_minus=passes["minus"]["codes"],
+               near_plus=passes["plus"]["near"], near_minus=passes["minus"]["near"],
+               w_restored=w_rest[active].copy())
+    state.w = w_next
+    state.t += 1
+    state.log.append(rec)
+    return rec
+
+
+def bitnet_loss_fn(cfg, embed, gains, head, tokens, targets, rows=None):
+    """loss_fn for ``step``: minibatch loss of Eq. 7 of the BitNet forward."""
+    embed = np.asarray(embed, dtype=np.float32)
+    gains = np.asarray(gains, dtype=np.float32)
+    head = np.asarray(head, dtype=np.float32)
+
+    def fn(codes, sw):
+        per, mean = bitnet.batch_loss(cfg, codes, sw, embed, gains, head, tokens, targets, rows)
+        fn.per_sequence.append(per)
+        return mean
+
+    fn.per_sequence = []
+    return fn

@@ -1,0 +1,108 @@
+"""Pins of the oracle's masked two-sided SPSA step (Eq. 1, Algorithm 1,
+App. E) against closed forms: the exact two-point quotient of a quadratic,
+the expectation identity of the Gaussian-smoothed objective, and the
+restore/update arithmetic.  CPU only."""
+import math
+
+import numpy as np
+
+from oracle import philox, ternary, termezo
+
+
+def _quadratic(n, seed=0):
+    rng = np.random.default_rng(seed)
+    M = rng.standard_normal((n, n))
+    A = M @ M.T / n + np.eye(n)
+    b = rng.standard_normal(n)
+    return A, b, lambda w: 0.5 * w.astype(np.float64) @ A @ w.astype(np.float64) + b @ w.astype(np.float64)
+
+
+def test_quadratic_two_point_quotient_is_exact():
+    n = 64
+    A, b, F = _quadratic(n)
+    rng = np.random.default_rng(1)
+    w = (rng.standard_normal(n) * 0.1).astype(np.float32)
+    active = np.sort(rng.choice(n, 20, replace=False)).astype(np.int64)
+    z = philox.normal(123, active)
+    eps, lr = 1e-3, 1e-2
+    w_next, fp, fm, g, w_plus, w_minus, _ = termezo.masked_spsa(w, active, z, eps, lr, F)
+    # for a quadratic F(w+) - F(w-) = (w+ - w-)^T (A (w+ + w-)/2 + b) exactly
+    dp = w_plus.astype(np.float64) - w_minus.astype(np.float64)
+    mid = (w_plus.astype(np.float64) + w_minus.astype(np.float64)) / 2
+    g_closed = dp @ (A @ mid + b) / (2 * float(np.float32(eps)))
+    assert abs(g - g_closed) <= 1e-9 * max(1.0, abs(g_closed))
+    # and it approximates z_S^T grad F(w) (perturbation only on S)
+    grad = A @ w.astype(np.float64) + b
+    assert abs(g - z.astype(np.float64) @ grad[active]) < 1e-2 * max(1.0, abs(g))
+    # untouched coordinates never move
+    frozen = np.setdiff1d(np.arange(n), active)
+    assert np.array_equal(w_next[frozen], w[frozen])
+    assert np.array_equal(w_plus[frozen], w[frozen]) and np.array_equal(w_minus[frozen], w[frozen])
+
+
+def test_spsa_is_unbiased_for_masked_gradient():
+    """E[g z_S] = m . grad F for a quadratic (App. E): mean over many seeds."""
+    n = 8
+    A, b, F = _quadratic(n, seed=4)
+    w = np.linspace(-0.5, 0.5, n).astype(np.float32)
+    active = np.array([1, 2, 5, 6], dtype=np.int64)
+    N = 6000
+    acc = np.zeros(n)
+    samples = []
+    for s in range(N):
+        z = philox.normal(10_000 + s, active)
+        _, _, _, g, _, _, _ = termezo.masked_spsa(w, active, z, 1e-2, 0.0, F)
+        v = np.zeros(n)
+        v[active] = g * z
+        samples.append(v)
+    samples = np.array(samples)
+    mean = samples.mean(axis=0)
+    se = samples.std(axis=0) / math.sqrt(N) + 1e-12
+    grad = A @ w.astype(np.float64) + b
+    expect = np.zeros(n)
+    expect[active] = grad[active]
+    assert np.all(np.abs(mean - expect) < 5 * se + 1e-9)
+    assert np.all(mean[np.setdiff1d(np.arange(n), active)] == 0)
+
+
+def test_ternary_smoothed_gradient_closed_form():
+    """One ternary weight, fixed tau: F(w) = Q(w).  The Gaussian-smoothed
+    objective is Phi((w - tau)/eps) - Phi((-tau - w)/eps); its derivative is
+    (phi((w - tau)/eps) + phi((w + tau)/eps)) / eps (App. E, Eq. smoothed_grad)."""
+    tau = np.float32(0.1)
+    eps = 0.05
+    w = np.array([0.08], np.float32)
+    active = np.array([0], dtype=np.int64)
+    F = lambda v: float(ternary.quantize(v, tau)[0])
+    N = 20000
+    vals = np.empty(N)
+    for s in range(N):
+        z = philox.normal(s, np.array([s], dtype=np.uint64))   # fresh z per draw
+        _, _, _, g, _, _, _ = termezo.masked_spsa(w, active, z, eps, 0.0, F)
+        vals[s] = g * float(z[0])
+    phi = lambda x: math.exp(-0.5 * x * x) / math.sqrt(2 * math.pi)
+    expect = (phi((0.08 - 0.1) / eps) + phi((0.08 + 0.1) / eps)) / eps
+    se = vals.std() / math.sqrt(N)
+    assert abs(vals.mean() - expect) < 5 * se
+
+
+def test_restore_and_update_arithmetic():
+    rng = np.random.default_rng(11)
+    n = 100000
+    w = (rng.standard_normal(n) * 0.02).astype(np.float32)
+    active = np.arange(0, n, 3, dtype=np.int64)
+    z = philox.normal(9, active)
+    eps, lr = np.float32(1e-3), np.float32(1e-6)
+    F = lambda v: float(np.sum(v.astype(np.float64) ** 3))
+    w_next, fp, fm, g, w_plus, w_minus, w_rest = termezo.masked_spsa(w, active, z, eps, lr, F)
+    e = (eps * z).astype(np.float32)
+    # +eps z, -2 eps z, +eps z restores within a few ulp of |w| + 2|e|
+    bound = 1.5 * np.spacing(np.abs(w[active]) + 2 * np.abs(e)).astype(np.float64)
+    assert np.all(np.abs(w_rest[active].astype(np.float64) - w[active]) <= bound)
+    # exact restore where w + e and w + e - 2e are exact (e a multiple of ulp(w))
+    exact = (np.float32(w[active] + e) - e == w[active]) & (np.float32(np.float32(w[active] + e) - 2 * e) + e == w[active])
+    assert np.all(w_rest[active][exact] == w[active][exact])
+    # update regenerates the same z and moves by fl32(fl32(lr g) z)
+    c = np.float32(float(lr) * g)
+    assert np.array_equal(w_next[active], (w_rest[active] - (c * z).astype(np.float32)).astype(np.float32))
+    assert g == (fp - fm) / (2 * float(eps))
