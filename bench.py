@@ -1,0 +1,417 @@
+#!/usr/bin/env python
+"""Throughput of the TerMeZO training step (Algorithm 1, K = 1) on GB300.
+
+Prints ONE JSON line.  A step is one whole TerMeZO iteration: shrink (Eq. 5),
+perturb + requantise to 2-bit codes, BitNet forward at +eps z, perturb,
+forward at -eps z, projected gradient, masked update -- over one minibatch
+of synthetic tokens.  Default workload: the BitNet-b1.58-2B-shaped model
+(30 layers, d 2560, 20/5 heads, FFN 6912, vocab 128256, seq 512, batch 16,
+last-token loss over 4 label tokens) at mask density 1%.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl mine|reference]
+
+With N > 1 (torchrun) every rank runs an independent replica (the step has
+no cross-GPU exchange in this build); value = tokens of all ranks / max
+time.  --impl reference times the CPU oracle on a bounded sample of the same
+workload on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+from paper_2609_33548_gb300 import synth  # noqa: E402
+
+METRIC = "TerMeZO steps/s & tokens/s at 2B shape; int8 TC util, HBM GB/s vs peak"
+EPS, LR = 1e-3, 1e-6
+WORKLOADS = {
+    "2b": (synth.BITNET_2B, 0.01),
+    "2b-0.1": (synth.BITNET_2B, 0.001),
+    "0.7b": (synth.BITNET_07B, 0.01),
+    "tiny": (synth.TINY, 0.01),
+}
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return d, "measured"
+    except (OSError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+class Clocks:
+    """Samples SM clocks and throttle reasons with nvidia-smi while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.path = tempfile.mktemp(suffix=".csv")
+        self.proc = None
+        self.gpu = gpu_index
+
+    def __enter__(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) >= 9:
+                rows.append(parts)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        power = [float(r[3]) for r in rows if r[3].replace(".", "").isdigit()]
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows), "power_w_max": max(power) if power else None}
+
+
+def dist_setup(n_gpus):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if torch.cuda.is_available():
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend=backend)
+        return dist, rank, world, local
+    return None, 0, 1, 0
+
+
+def barrier(dist):
+    if dist is not None:
+        dist.barrier()
+
+
+def max_over_ranks(dist, v: float) -> float:
+    if dist is None:
+        return v
+    t = torch.tensor([v], dtype=torch.float64, device="cuda" if torch.cuda.is_available() else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# --------------------------------------------------------------- oracle ----
+
+class OracleSample:
+    """Times the CPU oracle on a bounded sample of one TerMeZO step of the
+    workload: the dense requantisation of one layer's seven projections at
+    w + eps z and w - eps z, and the BitNet forward of one sequence through a
+    one-layer model of the same shape at both perturbations.  The full step
+    is L * (requant + B * forward) of these pieces (the sparse mask, z and
+    update work is O(k) and small next to them).  Inputs are drawn once."""
+
+    def __init__(self, cfg, density):
+        from oracle import bitnet, termezo as otz
+        self.cfg = cfg
+        self.one = synth.ModelConfig(cfg.name + "-1layer", 1, cfg.hidden, cfg.heads, cfg.kv_heads, cfg.ffn,
+                                     cfg.vocab, cfg.seq, 1, cfg.loss_mode, cfg.n_labels)
+        self.reg = otz.registry(self.one)
+        rng = np.random.default_rng(0)
+        n = self.one.d_lat
+        self.w = (rng.standard_normal(n, dtype=np.float32) * np.float32(synth.LATENT_STD)).astype(np.float32)
+        self.act = np.sort(rng.choice(n, max(1, int(density * n)), replace=False)).astype(np.int64)
+        self.tok = rng.integers(0, cfg.vocab, cfg.seq)
+        V, D = cfg.vocab, cfg.hidden
+        # only the rows the forward reads are drawn (token rows, label rows)
+        self.emb = np.zeros((V, D), np.float32)
+        rows = np.unique(self.tok)
+        self.emb[rows] = rng.standard_normal((rows.size, D), dtype=np.float32) * np.float32(0.02)
+        self.head = np.zeros((V, D), np.float32)
+        lab = np.arange(V - max(cfg.n_labels, 1), V) if cfg.loss_mode == 0 else np.arange(V)
+        self.head[lab] = bitnet.bf16_round(rng.standard_normal((lab.size, D), dtype=np.float32) * np.float32(0.02))
+        self.gains = np.ones((3, D), np.float32)
+
+    def run(self, seed=1000):
+        from oracle import bitnet, philox, termezo as otz
+        t0 = time.perf_counter()
+        z = philox.normal(seed, self.act)
+        e = (np.float32(EPS) * z).astype(np.float32)
+        wp = self.w.copy()
+        wp[self.act] += e
+        wm = wp.copy()
+        wm[self.act] -= np.float32(2) * e
+        cp, _, swp = otz.requantize(wp, self.reg)
+        cm, _, swm = otz.requantize(wm, self.reg)
+        t_rq = time.perf_counter() - t0
+        split = lambda c: [c[p.base:p.base + p.n].reshape(p.N, p.K) for p in self.reg]
+        t0 = time.perf_counter()
+        bitnet.sequence_loss(self.one, split(cp), swp, self.emb, self.gains, self.head, self.tok, 0)
+        bitnet.sequence_loss(self.one, split(cm), swm, self.emb, self.gains, self.head, self.tok, 0)
+        t_fw = time.perf_counter() - t0
+        est = self.cfg.layers * (t_rq + self.cfg.batch * t_fw)
+        return est, t_rq, t_fw
+
+
+def cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count()
+
+
+def run_reference(args):
+    dist, rank, world, _ = dist_setup(args.gpus)
+    cfg, density = WORKLOADS[args.workload]
+    if rank != 0:
+        return
+    sample = OracleSample(cfg, density)
+    times = []
+    for i in range(args.warmup + args.steps):
+        t0 = time.perf_counter()
+        est, t_rq, t_fw = sample.run(synth.step_seed(i))
+        wall = time.perf_counter() - t0
+        if i >= args.warmup:
+            times.append((est, wall, t_rq, t_fw))
+    est = statistics.median([t[0] for t in times])
+    value = cfg.tokens / est
+    sample = (f"per step: dense requantisation of 1 of {cfg.layers} layers (2 passes) + forward of 1 of "
+              f"{cfg.batch} sequences through a 1-layer model of the same shape (2 passes); scaled to the full "
+              f"step as layers x (requant + batch x forward)")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": est * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": f"{cfg.name} density {density}", "global_batch": cfg.batch,
+                       "seq_len": cfg.seq, "parallelism": "cpu"},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------ GPU ----
+
+def run_mine(args):
+    from paper_2609_33548_gb300 import termezo as tz
+
+    dist, rank, world, local = dist_setup(args.gpus)
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU for --impl mine")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    cfg, density = WORKLOADS[args.workload]
+    B, S = cfg.batch, cfg.seq
+
+    w = synth.latents(cfg, device=dev)
+    emb, gains, head = synth.theta(cfg, device=dev)
+    nb = args.warmup + args.steps
+    batches = [synth.batch(cfg, device=dev, step=i) for i in range(nb)]
+    ctx = tz.Context(tz.make_cfg(cfg), density, device=dev)
+    ctx.termezo_load_params(w, emb, gains, head)
+    stream = torch.cuda.current_stream()
+
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    k0, xi0 = ctx.termezo_build_mask(density)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    build_ms = e0.elapsed_time(e1)
+    d = cfg.d_lat
+    build_bytes = 6 * 4 * d + d / 4 + 8 * k0          # 6 reads of w_0, packed codes and S_0 written
+
+    for i in range(args.warmup):
+        tok, tgt = batches[i]
+        ctx.termezo_step(synth.step_seed(i), EPS, LR, density, tok, tgt)
+
+    with Clocks(local) as clk:
+        barrier(dist)
+        torch.cuda.synchronize()
+        ctx.termezo_profile(1)
+        e0.record(stream)
+        outs = []
+        for i in range(args.warmup, nb):
+            tok, tgt = batches[i]
+            outs.append(ctx.termezo_step(synth.step_seed(i), EPS, LR, density, tok, tgt))
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier(dist)
+    prof = ctx.termezo_profile(0, read=True)
+    ms = e0.elapsed_time(e1)
+    ms_max = max_over_ranks(dist, ms)
+    clocks = clk.summary()
+
+    # end to end through the public API: host-side inputs copied in, results read back
+    tok_h = [b[0].cpu().pin_memory() for b in batches]
+    tgt_h = [b[1].cpu().pin_memory() for b in batches]
+    tok_d = torch.empty_like(batches[0][0])
+    tgt_d = torch.empty_like(batches[0][1])
+    barrier(dist)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for i in range(args.warmup, nb):
+        tok_d.copy_(tok_h[i], non_blocking=True)
+        tgt_d.copy_(tgt_h[i], non_blocking=True)
+        ctx.termezo_step(synth.step_seed(nb + i), EPS, LR, density, tok_d, tgt_d)
+    torch.cuda.synchronize()
+    e2e_s = max_over_ranks(dist, time.perf_counter() - t0)
+
+    pk, how = peaks()
+    tokens = world * args.steps * B * S
+    value = tokens / (ms_max / 1e3)
+    gemm_s = prof["gemm_ms"] / 1e3
+    achieved = prof["gemm_flops"] / gemm_s / 1e12 if gemm_s > 0 else None
+    peak = float(pk.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+    h2d = tok_h[0].numel() * 4 + tgt_h[0].numel() * 4
+    d2h = 2 * 8 + 8 + 4 * 8 + 4 + 2 * B * 8
+    sparse_gbs = prof["sparse_bytes"] / (prof["sparse_ms"] / 1e3) / 1e9 if prof["sparse_ms"] > 0 else None
+    attn_tf = prof["attn_flops"] / (prof["attn_ms"] / 1e3) / 1e12 if prof["attn_ms"] > 0 else None
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_max / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": f"{cfg.name} density {density}", "global_batch": B * world, "seq_len": S,
+                   "parallelism": f"replicas{world}", "layers": cfg.layers, "hidden": cfg.hidden,
+                   "density": density, "k_active": int(outs[-1]["k_active"]), "eps": EPS, "lr": LR,
+                   "l2": "no flush: per-step working set (521 MB packed codes, >1 GB activations) exceeds L2"},
+        "steps_per_s": world * args.steps / (ms_max / 1e3),
+        "roofline": {"bound": "tensor", "kernel": "k_bitlinear_gemm (tcgen05 kind::f16, exact int8 x ternary)",
+                     "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak if achieved else None, "traffic": None,
+                     "peak_source": f"{how} bf16_tflops_sustained",
+                     "launches": prof["gemm_launches"], "avg_launch_ms": prof["gemm_ms"] / max(1, prof["gemm_launches"]),
+                     "share_of_step": prof["gemm_ms"] / ms},
+        "kernels": {"attention_tflops": attn_tf, "attention_share": prof["attn_ms"] / ms,
+                    "sparse_passes_gbs": sparse_gbs,
+                    "sparse_passes_frac_hbm": sparse_gbs / float(pk.get("hbm_gbs", 6800.0)) if sparse_gbs else None,
+                    "sparse_share": prof["sparse_ms"] / ms,
+                    "mask_build_ms": build_ms, "mask_build_gbs": build_bytes / (build_ms / 1e3) / 1e9},
+        "e2e": {"value": tokens / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": int(prof["launches"]),
+        "clocks": clocks,
+        "last_step": {k: outs[-1][k] for k in ("loss_plus", "loss_minus", "g", "n_flipped", "n_jumps")},
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        est, t_rq, t_fw = OracleSample(cfg, density).run()
+        line["cpu_baseline"] = {"value": cfg.tokens / est, "unit": "tokens/s", "cores": cores(), "kind": "oracle",
+                                "sample": f"dense requant of 1/{cfg.layers} layers x2 ({t_rq:.1f} s) + forward of "
+                                          f"1/{cfg.batch} sequences x2 through a 1-layer model ({t_fw:.1f} s), "
+                                          f"scaled to the full step"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+def run_op(args):
+    """BitLinear-op workload (one [6912, 2560] projection, 2048 activation
+    rows, density from --op-density): per step requantise at +eps z,
+    BitLinear, requantise at -eps z, BitLinear, update, shrink."""
+    from paper_2609_33548_gb300 import termezo as tz
+
+    N, K, M = synth.BITLINEAR_OP["N"], synth.BITLINEAR_OP["K"], synth.BITLINEAR_OP["M"]
+    density = args.op_density
+    dev = torch.device("cuda", 0)
+    w = synth.op_latents(N, K, device=dev).reshape(-1)
+    x = synth.op_activations(M, K, device=dev)
+    y = torch.empty(M, N, dtype=torch.float32, device=dev)
+    ctx = tz.Context(tz.op_cfg(N, K, M), density, device=dev)
+    ctx.termezo_load_params(w)
+    k0, _ = ctx.termezo_build_mask(density)
+
+    def step(i):
+        seed = synth.step_seed(i)
+        ctx.termezo_shrink()
+        ctx.termezo_requantize(seed, EPS, +1)
+        ctx.termezo_bitlinear(0, x, None, y)
+        ctx.termezo_requantize(seed, EPS, -1)
+        ctx.termezo_bitlinear(0, x, None, y)
+        ctx.termezo_update(seed, EPS, LR, 1.0)
+
+    for i in range(args.warmup):
+        step(i)
+    stream = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for i in range(args.warmup, args.warmup + args.steps):
+        step(i)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    # the GEMM alone, timed with events around each launch
+    ts = []
+    for _ in range(5):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        ctx.termezo_bitlinear(0, x, None, y)
+        b.record(stream)
+        torch.cuda.synchronize()
+        ts.append(a.elapsed_time(b))
+    gemm_ms = statistics.median(ts)
+    pk, how = peaks()
+    flops = 2.0 * M * N * K
+    line = {"metric": "BitLinear op step (requant +, GEMM, requant -, GEMM, update, shrink)",
+            "value": args.steps * M / (ms / 1e3), "unit": "rows/s", "n_gpus": 1, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": f"bitlinear-op M{M} K{K} N{N} density {density}", "k0": k0},
+            "bitlinear_call_ms": gemm_ms,
+            "bitlinear_call_tflops": flops / (gemm_ms / 1e3) / 1e12,
+            "peak_bf16_tflops": float(pk.get("bf16_tflops", 1900.0)), "peak_source": how}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=("mine", "reference"), default="mine")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS) + ["op"], default="2b")
+    ap.add_argument("--op-density", type=float, default=0.01)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    elif args.workload == "op":
+        run_op(args)
+    else:
+        run_mine(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,189 @@
+/*
+ * termezo.h -- C ABI of libtermezo.so, a GB300 (sm_103a) implementation of
+ * the TerMeZO training step: sparse zeroth-order fine-tuning of a ternary
+ * BitNet model (Sifaou, Katti, Rajendran, Simeone, arXiv 2609.33548).
+ *
+ * Conventions shared by every call
+ *  - Pointers named d_* are device pointers owned by the caller; h_* are
+ *    host pointers owned by the caller.  The library never allocates device
+ *    memory: every internal buffer is carved from the one workspace the
+ *    caller passes to termezo_create.
+ *  - All device work is ordered on the stream given to termezo_create (a
+ *    cudaStream_t passed as void*; NULL = legacy default stream).  Calls
+ *    that return host values synchronise that stream before returning.
+ *  - Return value: TERMEZO_OK (0), a positive warning, or a negative error
+ *    code; termezo_strerror gives a message.  After TERMEZO_ECUDA or
+ *    TERMEZO_ETIMEOUT the context must be destroyed.
+ *  - Latent layout ("global order"): layer 0..L-1; within a layer the
+ *    projections q, k, v, o, gate, up, down; each a row-major [N_out, K_in]
+ *    fp32 matrix, concatenated.  q: [H*hd, D]; k, v: [KV*hd, D];
+ *    o: [D, H*hd]; gate, up: [F, D]; down: [D, F]; hd = D / H.
+ *  - Packed ternary store: code q + 1 of global weight i (q in {-1,0,1},
+ *    Eq. 2) in bits 2*(i mod 16) of uint32 word i / 16.
+ */
+#ifndef TERMEZO_H
+#define TERMEZO_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define TERMEZO_OK 0
+#define TERMEZO_WMASKFIXED 1   /* density differs from the built mask; ignored */
+#define TERMEZO_EINVAL (-1)    /* bad shape, null pointer, density outside (0,1] */
+#define TERMEZO_ESTATE (-2)    /* call out of order (e.g. step before build_mask) */
+#define TERMEZO_ENOMEM (-3)    /* workspace smaller than termezo_workspace_bytes */
+#define TERMEZO_ECUDA (-4)     /* a CUDA call failed */
+#define TERMEZO_ETIMEOUT (-5)  /* a bounded device-side wait gave up */
+
+typedef struct termezo_ctx termezo_ctx;
+
+/* Shape of the BitNet decoder and of one minibatch.
+ * layers == 0 selects the single-projection ("BitLinear op") context: one
+ * ternary projection of shape [ffn, hidden] and seq*batch activation rows;
+ * termezo_step and termezo_forward_loss are then unavailable.
+ * loss_mode 0: cross-entropy of the last position over the n_labels label
+ * tokens vocab-n_labels .. vocab-1 (targets = class ids [batch]).
+ * loss_mode 1: token-level cross-entropy over the full vocabulary at every
+ * position (targets = token ids [batch, seq]). */
+typedef struct {
+  int32_t layers, hidden, heads, kv_heads, ffn, vocab, seq, batch;
+  int32_t loss_mode;
+  int32_t n_labels;
+} termezo_model_cfg;
+
+/* Per-step report (Algorithm 1 with K = 1; counters of Eq. 11). */
+typedef struct {
+  double loss_plus;   /* F+ = minibatch loss at w + eps m.z            */
+  double loss_minus;  /* F- = minibatch loss at w - eps m.z            */
+  double g;           /* projected gradient (F+ - F-) / (2 eps)        */
+  uint64_t k_active;  /* k_t = |S_t| after this step's shrink (Eq. 5)  */
+  uint64_t n_flipped; /* active codes that differ between the two passes */
+  uint64_t n_jumps;   /* active codes that moved -1 <-> +1 between them  */
+  uint64_t n_dropped; /* weights frozen by this step's shrink           */
+} termezo_step_out;
+
+/* Bytes of device workspace a context needs for cfg and mask density
+ * rho_0 (the sparse store holds floor(rho_0 * d) weights).  Host only. */
+int termezo_workspace_bytes(const termezo_model_cfg* cfg, double density, size_t* bytes);
+
+/* Creates a context over a caller-owned device workspace of `bytes` bytes
+ * (>= termezo_workspace_bytes(cfg, density)); 256-byte aligned.  `stream`
+ * is a cudaStream_t.  The workspace must outlive the context. */
+int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspace,
+                   size_t bytes, void* stream, termezo_ctx** out);
+
+/* Registers the parameters (device pointers, read by later calls; they
+ * must stay valid until termezo_build_mask returns, and d_embed, d_gains,
+ * d_head for the life of the context):
+ *   d_latents fp32 [d]       dense latent weights w_0, global order;
+ *   d_embed   fp32 [V, D]    token embeddings (theta);
+ *   d_gains   fp32 [2L+1, D] RMSNorm gains: 2l = attention input of layer l,
+ *                            2l+1 = MLP input, 2L = final norm;
+ *   d_head    bf16 [V, D]    LM head, raw bfloat16 bits.
+ * For a single-projection context d_embed, d_gains, d_head may be NULL. */
+int termezo_load_params(termezo_ctx* ctx, const float* d_latents, const float* d_embed,
+                        const float* d_gains, const uint16_t* d_head);
+
+/* Algorithm 1, lines 1-2 (Eqs. 2-4): per projection gamma = mean |w|
+ * (exact sum), tau_0 = (gamma + 1e-5) / 2, distances d_i = min(|w_i - tau|,
+ * |w_i + tau|) of all weights of all projections, xi_0 the lower
+ * rho_0-quantile: exactly k0 = floor(rho_0 d) weights with the smallest
+ * (d_i, i) pairs form S_0 (ties at xi_0 go to the lower global index).
+ * Writes the sparse store (sorted active indices + fp32 latents) and the
+ * packed codes of every weight at tau_0.  Host outputs k0, xi0 (nullable).
+ * density must not exceed the one given to termezo_create.  Synchronises. */
+int termezo_build_mask(termezo_ctx* ctx, double density, uint64_t* k0, float* xi0);
+
+/* Minibatch loss F(Q(w_t), theta; B) (Eqs. 6-7) at the current latents:
+ * requantises the active weights, runs the BitNet forward.  d_tokens int32
+ * [batch, seq]; d_targets int32 (see loss_mode).  Host outputs: loss, and
+ * per_seq[batch] (nullable) the loss of each sequence.  Synchronises. */
+int termezo_forward_loss(termezo_ctx* ctx, const int32_t* d_tokens, const int32_t* d_targets,
+                         double* loss, double* per_seq);
+
+/* One TerMeZO iteration (Algorithm 1 loop body, K = 1):
+ *   t >= 1: tau_t recomputed, S_t = {i in S_{t-1}: d_i(w_t) <= xi_0} (Eq. 5);
+ *   z_i ~ N(0,1) regenerated from (seed, i) by Philox-4x32-10 + Box-Muller;
+ *   w += eps m.z -> requantise (Eq. 2) -> F+;  w -= 2 eps m.z -> F-;
+ *   w += eps m.z (restore); g = (F+ - F-) / (2 eps) (Eq. 1);
+ *   w -= lr g m.z with the same z.
+ * density: the mask's rho_0 is fixed after build (xi_0 is fixed, Eq. 5); a
+ * different value returns TERMEZO_WMASKFIXED and is otherwise ignored.
+ * out: host report (required); per_seq_plus / per_seq_minus: host [batch]
+ * per-sequence losses of the two passes (nullable).  Synchronises once. */
+int termezo_step(termezo_ctx* ctx, uint64_t seed, float eps, float lr, double density,
+                 const int32_t* d_tokens, const int32_t* d_targets, termezo_step_out* out,
+                 double* per_seq_plus, double* per_seq_minus);
+
+/* Pieces of the step, for the single-projection context and for tests.
+ * termezo_shrink: Eq. 5 at the current latents (no-op before the first
+ *   update); host output n_dropped (nullable).
+ * termezo_requantize: sign = +1 writes the codes of w + eps z, sign = -1
+ *   the codes of (w + eps z) - 2 eps z, sign = 0 the codes of w, each at
+ *   the tau of the perturbed projection (Eq. 2); active weights only.
+ * termezo_update: restore (+eps z) and w -= (float)(lr * g) z (Algorithm 1).
+ * None of these synchronises. */
+int termezo_shrink(termezo_ctx* ctx, uint64_t* n_dropped);
+int termezo_requantize(termezo_ctx* ctx, uint64_t seed, float eps, int sign);
+int termezo_update(termezo_ctx* ctx, uint64_t seed, float eps, float lr, double g);
+
+/* BitLinear of projection `proj` (global order index) on activations
+ * d_x bf16 [M, K_in] (raw bits, row-major): per row a = max(max|x|, 1e-5),
+ * int8 codes q = clamp(rint(x * (127/a)), -128, 127) decided in fp32,
+ * acc = q . codes^T (exact int32), y = acc * (a/127) * s_w with
+ * s_w = gamma + 1e-5 of the current codes.  Outputs (device, nullable):
+ * d_acc int32 [M, N_out], d_y fp32 [M, N_out].  M <= seq * batch. */
+int termezo_bitlinear(termezo_ctx* ctx, int32_t proj, const uint16_t* d_x, int32_t M,
+                      int32_t* d_acc, float* d_y);
+
+/* Sizes of the state: d (latent count), k_active (current |S_t|),
+ * n_proj (projection count).  Host outputs, each nullable.  Synchronises. */
+int termezo_state_sizes(termezo_ctx* ctx, uint64_t* d, uint64_t* k_active, int32_t* n_proj);
+
+/* Copies the state to host buffers (each nullable): h_idx uint32 [k_active]
+ * sorted active global indices; h_latents fp32 [k_active] their latents;
+ * h_packed uint32 [d/16] the packed codes; h_tau fp32 [3 * n_proj] the
+ * thresholds tau of the current latents, of the + pass and of the - pass.
+ * Synchronises. */
+int termezo_export_state(termezo_ctx* ctx, uint32_t* h_idx, float* h_latents, uint32_t* h_packed,
+                         float* h_tau);
+
+/* z_i for n global indices d_idx (uint32, device) with key `seed`, written
+ * to d_z fp32 [n].  Stateless; ordered on `stream`. */
+int termezo_normal(uint64_t seed, const uint32_t* d_idx, uint64_t n, float* d_z, void* stream);
+
+/* Kernel timing of a context.  enable = 1 resets the totals and starts
+ * recording CUDA events (on the context's stream) around every BitLinear
+ * GEMM, attention and sparse-pass launch; enable = 0 stops recording;
+ * enable = -1 leaves the state unchanged.  When out is non-NULL the stream
+ * is synchronised and the totals since the last reset are written.
+ * Algorithmic work: GEMM 2*M*N*K flops; attention 4*B*H*hd*S(S+1)/2 flops
+ * (QK^T and PV over the causal half); sparse passes 8 B per active weight
+ * (index + latent) read per pass, plus 4 B written per updated latent and
+ * 8 B per packed word rewritten. */
+typedef struct {
+  uint64_t launches;        /* kernels launched by this thread since the reset */
+  uint64_t gemm_launches;
+  double gemm_ms, gemm_flops;
+  uint64_t attn_launches;
+  double attn_ms, attn_flops;
+  uint64_t sparse_launches; /* timed sparse passes (each 1-3 kernels) */
+  double sparse_ms, sparse_bytes;
+} termezo_profile_out;
+
+int termezo_profile(termezo_ctx* ctx, int enable, termezo_profile_out* out);
+
+/* Releases the host-side context (the workspace stays the caller's). */
+void termezo_destroy(termezo_ctx* ctx);
+
+const char* termezo_strerror(int status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TERMEZO_H */

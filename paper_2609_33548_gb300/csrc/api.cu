@@ -1,0 +1,767 @@
+// C ABI of libtermezo.so: context, workspace layout and the host-side
+// orchestration of Algorithm 1 (declarations and contracts in termezo.h).
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "kernels.cuh"
+#include "sparse.cuh"
+#include "termezo.h"
+
+using tmz::ExactSum;
+using tmz::GemmArgs;
+using tmz::GemmPlan;
+using tmz::MaskArgs;
+
+namespace {
+
+constexpr uint32_t DENSE_CHUNK = 4096;
+constexpr uint32_t SPARSE_CHUNK = 4096;
+
+struct Shape {
+  bool op;
+  int L, D, H, KV, hd, F, V, S, B, T, C, mode;
+  int P;
+  std::vector<uint64_t> base;  // [P+1]
+  std::vector<int> N, K;       // [P]
+  uint64_t d;
+};
+
+int make_shape(const termezo_model_cfg* c, Shape* s) {
+  if (!c) return TERMEZO_EINVAL;
+  s->op = c->layers == 0;
+  s->L = c->layers;
+  s->D = c->hidden;
+  s->F = c->ffn;
+  s->S = c->seq;
+  s->B = c->batch;
+  s->T = c->seq * c->batch;
+  s->mode = c->loss_mode;
+  s->C = c->n_labels;
+  s->V = c->vocab;
+  s->H = c->heads;
+  s->KV = c->kv_heads;
+  if (c->layers < 0 || c->hidden <= 0 || c->ffn <= 0 || c->seq <= 0 || c->batch <= 0) return TERMEZO_EINVAL;
+  if (c->hidden % 16 || c->ffn % 16) return TERMEZO_EINVAL;
+  s->base.assign(1, 0);
+  s->N.clear();
+  s->K.clear();
+  if (s->op) {
+    s->P = 1;
+    s->N.push_back(c->ffn);
+    s->K.push_back(c->hidden);
+    s->hd = 0;
+  } else {
+    if (c->heads <= 0 || c->kv_heads <= 0 || c->hidden % c->heads || c->heads % c->kv_heads) return TERMEZO_EINVAL;
+    s->hd = c->hidden / c->heads;
+    if (s->hd != 64 && s->hd != 96 && s->hd != 128) return TERMEZO_EINVAL;
+    if (c->seq % 64) return TERMEZO_EINVAL;
+    if (c->vocab <= 0) return TERMEZO_EINVAL;
+    if (c->loss_mode != 0) return TERMEZO_EINVAL;  // token-level loss: not provided by this build
+    if (c->n_labels < 1 || c->n_labels > 64 || c->n_labels > c->vocab) return TERMEZO_EINVAL;
+    const int Hq = s->H * s->hd, Hkv = s->KV * s->hd;
+    const int n[7] = {Hq, Hkv, Hkv, s->D, s->F, s->F, s->D};
+    const int k[7] = {s->D, s->D, s->D, Hq, s->D, s->D, s->F};
+    s->P = 7 * s->L;
+    for (int l = 0; l < s->L; ++l)
+      for (int j = 0; j < 7; ++j) {
+        s->N.push_back(n[j]);
+        s->K.push_back(k[j]);
+      }
+  }
+  for (int p = 0; p < s->P; ++p) s->base.push_back(s->base.back() + (uint64_t)s->N[p] * (uint64_t)s->K[p]);
+  s->d = s->base.back();
+  if (s->d >= (1ull << 32)) return TERMEZO_EINVAL;
+  return TERMEZO_OK;
+}
+
+uint64_t keep_count(double density, uint64_t d) { return (uint64_t)std::floor(density * (double)d); }
+
+// Bump allocator over the workspace; with base == nullptr it only measures.
+struct Carver {
+  uint8_t* base;
+  size_t off = 0;
+  template <typename T>
+  T* take(size_t count) {
+    off = (off + 255) & ~(size_t)255;
+    T* p = base ? reinterpret_cast<T*>(base + off) : nullptr;
+    off += count * sizeof(T);
+    return p;
+  }
+};
+
+}  // namespace
+
+struct termezo_ctx {
+  Shape sh;
+  double density = 0;
+  uint64_t k_cap = 0;
+  cudaStream_t stream = nullptr;
+  MaskArgs ma{};
+  uint32_t NBS_max = 0;
+  uint32_t* d_total = nullptr;
+  std::vector<uint32_t> dpre;
+  int cur = 0;
+  bool built = false;
+  int t = 0;
+  bool updated = false;
+  float xi0 = 0.f;
+  uint64_t k0 = 0, k_active = 0;
+  const float* latents = nullptr;
+  const float* embed = nullptr;
+  const float* gains = nullptr;
+  const uint16_t* head = nullptr;
+  // forward buffers
+  float* x = nullptr;
+  uint16_t* xq = nullptr;
+  float* deq = nullptr;
+  float* qkv = nullptr;
+  uint16_t *qb = nullptr, *kb = nullptr, *vt = nullptr;
+  float* attn = nullptr;
+  float* gu = nullptr;
+  uint16_t* wexp = nullptr;
+  float *cosb = nullptr, *sinb = nullptr;
+  double* per_seq = nullptr;  // [2B]
+  double* loss = nullptr;     // [2]
+  double* g = nullptr;        // [1]
+  GemmPlan plan_qkv{}, plan_o{}, plan_gu{}, plan_down{};
+  const float* code_sw = nullptr;  // s_w array matching the codes now in the packed store
+  uint64_t pm_seed = 0;
+  float pm_eps = 0.f;
+  bool pm_valid = false;
+  // kernel timing (termezo_profile)
+  struct ProfRec {
+    int cat;  // 0 GEMM, 1 attention, 2 sparse pass
+    cudaEvent_t a, b;
+    double work;
+  };
+  bool prof_on = false;
+  std::vector<ProfRec> prof;
+  std::vector<cudaEvent_t> ev_pool;
+  size_t ev_used = 0;
+  uint64_t launch_base = 0;
+  ~termezo_ctx() {
+    for (cudaEvent_t e : ev_pool) cudaEventDestroy(e);
+  }
+};
+
+namespace {
+
+size_t xq_cols(const Shape& s) {
+  if (s.op) return (size_t)s.D;
+  size_t m = s.D;
+  if ((size_t)s.H * s.hd > m) m = (size_t)s.H * s.hd;
+  if ((size_t)s.F > m) m = s.F;
+  return m;
+}
+
+size_t wexp_elems(const Shape& s) {
+  size_t m = 0;
+  if (s.op) return (size_t)s.N[0] * s.K[0];
+  const size_t qkv = (size_t)(s.H + 2 * s.KV) * s.hd * s.D, o = (size_t)s.D * s.H * s.hd, gu = (size_t)2 * s.F * s.D,
+               dn = (size_t)s.D * s.F;
+  m = qkv;
+  if (o > m) m = o;
+  if (gu > m) m = gu;
+  if (dn > m) m = dn;
+  return m;
+}
+
+void carve(termezo_ctx* c, Carver& cv) {
+  const Shape& s = c->sh;
+  const int P = s.P;
+  MaskArgs& a = c->ma;
+  a.P = P;
+  a.base = cv.take<uint64_t>(P + 1);
+  a.dpre = cv.take<uint32_t>(P + 1);
+  a.spre = cv.take<uint32_t>(P + 1);
+  a.packed = cv.take<uint32_t>(s.d / 16);
+  for (int i = 0; i < 2; ++i) {
+    a.idx[i] = cv.take<uint32_t>(c->k_cap);
+    a.lat[i] = cv.take<float>(c->k_cap);
+    a.off[i] = cv.take<uint32_t>(P + 1);
+  }
+  a.S_total = cv.take<ExactSum>(P);
+  a.A_frozen = cv.take<ExactSum>(P);
+  const size_t nbd = c->dpre.empty() ? 0 : c->dpre.back();
+  const size_t nblk = nbd > c->NBS_max ? nbd : c->NBS_max;
+  a.partials = cv.take<ExactSum>(nbd > 2 * (size_t)c->NBS_max ? nbd : 2 * (size_t)c->NBS_max);
+  float** fl[9] = {&a.gamma_cur, &a.tau_cur, &a.sw_cur, &a.gamma_plus, &a.tau_plus,
+                   &a.sw_plus,   &a.gamma_minus, &a.tau_minus, &a.sw_minus};
+  for (auto f : fl) *f = cv.take<float>(P + 2);
+  a.hist = cv.take<unsigned long long>(2048);
+  a.sel = cv.take<tmz::SelectState>(1);
+  a.blk_a = cv.take<uint32_t>(nblk);
+  a.blk_b = cv.take<uint32_t>(nblk);
+  a.blk_c = cv.take<uint32_t>(nblk);
+  a.blk_d = cv.take<uint32_t>(nblk);
+  a.counters = cv.take<unsigned long long>(4);
+  a.err = cv.take<unsigned>(1);
+  c->d_total = cv.take<uint32_t>(1);
+  const size_t T = s.T;
+  c->xq = cv.take<uint16_t>(T * xq_cols(s));
+  c->deq = cv.take<float>(T);
+  c->wexp = cv.take<uint16_t>(wexp_elems(s));
+  if (!s.op) {
+    const size_t hq = (size_t)s.H * s.hd, hkv = (size_t)s.KV * s.hd;
+    c->x = cv.take<float>(T * s.D);
+    c->qkv = cv.take<float>(T * (hq + 2 * hkv));
+    c->qb = cv.take<uint16_t>(T * hq);
+    c->kb = cv.take<uint16_t>(T * hkv);
+    c->vt = cv.take<uint16_t>(T * hkv);
+    c->attn = cv.take<float>(T * hq);
+    c->gu = cv.take<float>(T * 2 * (size_t)s.F);
+    c->cosb = cv.take<float>((size_t)s.S * s.hd / 2);
+    c->sinb = cv.take<float>((size_t)s.S * s.hd / 2);
+  }
+  c->per_seq = cv.take<double>(2 * (size_t)s.B);
+  c->loss = cv.take<double>(2);
+  c->g = cv.take<double>(1);
+}
+
+void plan_sizes(termezo_ctx* c, double density) {
+  const Shape& s = c->sh;
+  c->density = density;
+  c->k_cap = keep_count(density, s.d);
+  if (c->k_cap == 0) c->k_cap = 1;
+  c->dpre.assign(1, 0);
+  for (int p = 0; p < s.P; ++p) {
+    const uint64_t n = s.base[p + 1] - s.base[p];
+    c->dpre.push_back(c->dpre.back() + (uint32_t)((n + DENSE_CHUNK - 1) / DENSE_CHUNK));
+  }
+  c->NBS_max = (uint32_t)(2 * s.P + c->k_cap / SPARSE_CHUNK + 1);
+}
+
+int cuda_status(termezo_ctx* c) {
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    fprintf(stderr, "termezo: CUDA error %s\n", cudaGetErrorString(e));
+    return TERMEZO_ECUDA;
+  }
+  (void)c;
+  return TERMEZO_OK;
+}
+
+int sync_status(termezo_ctx* c) {
+  cudaError_t e = cudaStreamSynchronize(c->stream);
+  if (e == cudaSuccess) e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    fprintf(stderr, "termezo: CUDA error %s\n", cudaGetErrorString(e));
+    return TERMEZO_ECUDA;
+  }
+  unsigned err = 0;
+  if (cudaMemcpy(&err, c->ma.err, sizeof(unsigned), cudaMemcpyDeviceToHost) != cudaSuccess) return TERMEZO_ECUDA;
+  if (err & tmz::ERR_TIMEOUT) return TERMEZO_ETIMEOUT;
+  if (err & tmz::ERR_BOUNDS) {
+    cudaMemsetAsync(c->ma.err, 0, sizeof(unsigned), c->stream);
+    return TERMEZO_EINVAL;
+  }
+  return TERMEZO_OK;
+}
+
+int proj_of(const Shape& s, int layer, int j) { return 7 * layer + j; }
+
+cudaEvent_t ev_get(termezo_ctx* c) {
+  if (c->ev_used == c->ev_pool.size()) {
+    cudaEvent_t e;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    c->ev_pool.push_back(e);
+  }
+  return c->ev_pool[c->ev_used++];
+}
+
+// Records CUDA events around the launches made during its lifetime when
+// profiling is on.
+struct ProfScope {
+  termezo_ctx* c;
+  int cat;
+  double work;
+  cudaEvent_t a = nullptr;
+  ProfScope(termezo_ctx* ctx, int category, double w) : c(ctx), cat(category), work(w) {
+    if (c->prof_on && (a = ev_get(c))) cudaEventRecord(a, c->stream);
+  }
+  ~ProfScope() {
+    if (!a) return;
+    cudaEvent_t b = ev_get(c);
+    if (!b) return;
+    cudaEventRecord(b, c->stream);
+    c->prof.push_back({cat, a, b, work});
+  }
+};
+
+double gemm_flops(const GemmPlan& p) { return 2.0 * p.M * (double)p.N * p.K; }
+
+// BitNet forward at the codes now in the packed store, with weight scales
+// sw[] (one per projection); writes per_seq[slot*B ..] and loss[slot].
+int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, const float* sw, int slot) {
+  const Shape& s = c->sh;
+  cudaStream_t st = c->stream;
+  const int T = s.T, D = s.D, F = s.F, hq = s.H * s.hd, hkv = s.KV * s.hd;
+  tmz::launch_embed(tokens, c->embed, T, D, s.V, c->x, c->ma.err, st);
+  for (int l = 0; l < s.L; ++l) {
+    const int pq = proj_of(s, l, 0), po = proj_of(s, l, 3), pg = proj_of(s, l, 4), pd = proj_of(s, l, 6);
+    // attention block
+    tmz::launch_norm_quant(c->x, c->gains + (size_t)(2 * l) * D, T, D, c->xq, c->deq, st);
+    tmz::launch_expand_codes(c->ma.packed + s.base[pq] / 16, (uint64_t)(hq + 2 * hkv), D, c->wexp, st);
+    GemmArgs a{};
+    a.out = c->qkv;
+    a.ldo = hq + 2 * hkv;
+    a.mode = 0;
+    a.deq = c->deq;
+    a.sw = sw + pq;
+    a.n1 = hq;
+    a.n2 = hq + hkv;
+    a.err = c->ma.err;
+    {
+      ProfScope ps(c, 0, gemm_flops(c->plan_qkv));
+      if (tmz::gemm_launch(c->plan_qkv, a, st) != cudaSuccess) return TERMEZO_ECUDA;
+    }
+    tmz::launch_rope_pack(c->qkv, c->cosb, c->sinb, s.B, s.S, s.H, s.KV, s.hd, c->qb, c->kb, c->vt, st);
+    {
+      ProfScope ps(c, 1, 4.0 * s.B * s.H * (double)s.hd * (0.5 * s.S * (s.S + 1.0)));
+      tmz::launch_attention(c->qb, c->kb, c->vt, s.B, s.S, s.H, s.KV, s.hd, c->attn, st);
+    }
+    tmz::launch_norm_quant(c->attn, nullptr, T, hq, c->xq, c->deq, st);
+    tmz::launch_expand_codes(c->ma.packed + s.base[po] / 16, (uint64_t)D, hq, c->wexp, st);
+    a.out = c->x;
+    a.ldo = D;
+    a.mode = 1;
+    a.sw = sw + po;
+    a.n1 = a.n2 = D;
+    {
+      ProfScope ps(c, 0, gemm_flops(c->plan_o));
+      if (tmz::gemm_launch(c->plan_o, a, st) != cudaSuccess) return TERMEZO_ECUDA;
+    }
+    // MLP block
+    tmz::launch_norm_quant(c->x, c->gains + (size_t)(2 * l + 1) * D, T, D, c->xq, c->deq, st);
+    tmz::launch_expand_codes(c->ma.packed + s.base[pg] / 16, (uint64_t)(2 * F), D, c->wexp, st);
+    a.out = c->gu;
+    a.ldo = 2 * F;
+    a.mode = 0;
+    a.sw = sw + pg;
+    a.n1 = F;
+    a.n2 = 2 * F;
+    {
+      ProfScope ps(c, 0, gemm_flops(c->plan_gu));
+      if (tmz::gemm_launch(c->plan_gu, a, st) != cudaSuccess) return TERMEZO_ECUDA;
+    }
+    tmz::launch_relu2_quant(c->gu, T, F, c->xq, c->deq, st);
+    tmz::launch_expand_codes(c->ma.packed + s.base[pd] / 16, (uint64_t)D, F, c->wexp, st);
+    a.out = c->x;
+    a.ldo = D;
+    a.mode = 1;
+    a.sw = sw + pd;
+    a.n1 = a.n2 = D;
+    {
+      ProfScope ps(c, 0, gemm_flops(c->plan_down));
+      if (tmz::gemm_launch(c->plan_down, a, st) != cudaSuccess) return TERMEZO_ECUDA;
+    }
+  }
+  tmz::launch_head_ce_last(c->x, c->gains + (size_t)(2 * s.L) * D, c->head, targets, s.B, s.S, D, s.V, s.C,
+                           c->per_seq + (size_t)slot * s.B, c->loss + slot, st);
+  return cuda_status(c);
+}
+
+void ensure_pm(termezo_ctx* c, uint64_t seed, float eps) {
+  if (c->pm_valid && c->pm_seed == seed && c->pm_eps == eps) return;
+  tmz::sparse_pm_taus(c->ma, c->cur, seed, eps, c->stream);
+  c->pm_seed = seed;
+  c->pm_eps = eps;
+  c->pm_valid = true;
+}
+
+int do_shrink(termezo_ctx* c) {
+  ProfScope ps(c, 2, 3.0 * 8.0 * (double)c->k_active);
+  tmz::sparse_shrink(c->ma, c->cur, c->xi0, c->d_total, c->stream);
+  c->cur ^= 1;
+  c->pm_valid = false;
+  return cuda_status(c);
+}
+
+}  // namespace
+
+extern "C" {
+
+int termezo_workspace_bytes(const termezo_model_cfg* cfg, double density, size_t* bytes) {
+  if (!bytes || !(density > 0.0 && density <= 1.0)) return TERMEZO_EINVAL;
+  termezo_ctx tmp;
+  int rc = make_shape(cfg, &tmp.sh);
+  if (rc) return rc;
+  plan_sizes(&tmp, density);
+  Carver cv{nullptr};
+  carve(&tmp, cv);
+  *bytes = cv.off + 256;
+  return TERMEZO_OK;
+}
+
+int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspace, size_t bytes, void* stream,
+                   termezo_ctx** out) {
+  if (!out || !d_workspace || !(density > 0.0 && density <= 1.0)) return TERMEZO_EINVAL;
+  if ((uintptr_t)d_workspace & 255) return TERMEZO_EINVAL;
+  *out = nullptr;
+  termezo_ctx* c = new (std::nothrow) termezo_ctx();
+  if (!c) return TERMEZO_ENOMEM;
+  int rc = make_shape(cfg, &c->sh);
+  if (rc) {
+    delete c;
+    return rc;
+  }
+  plan_sizes(c, density);
+  Carver cv{reinterpret_cast<uint8_t*>(d_workspace)};
+  carve(c, cv);
+  if (cv.off > bytes) {
+    delete c;
+    return TERMEZO_ENOMEM;
+  }
+  c->stream = reinterpret_cast<cudaStream_t>(stream);
+  const Shape& s = c->sh;
+  c->ma.NBD = c->dpre.back();
+  cudaStream_t st = c->stream;
+  cudaMemcpyAsync((void*)c->ma.base, s.base.data(), (s.P + 1) * sizeof(uint64_t), cudaMemcpyHostToDevice, st);
+  cudaMemcpyAsync((void*)c->ma.dpre, c->dpre.data(), (s.P + 1) * sizeof(uint32_t), cudaMemcpyHostToDevice, st);
+  cudaMemsetAsync(c->ma.err, 0, sizeof(unsigned), st);
+  cudaMemsetAsync(c->ma.counters, 0, 4 * sizeof(unsigned long long), st);
+  for (float* f : {c->ma.gamma_cur, c->ma.tau_cur, c->ma.sw_cur, c->ma.gamma_plus, c->ma.tau_plus, c->ma.sw_plus,
+                   c->ma.gamma_minus, c->ma.tau_minus, c->ma.sw_minus})
+    cudaMemsetAsync(f, 0, (s.P + 2) * sizeof(float), st);
+  if (!s.op) {
+    tmz::launch_rope_tables(s.S, s.hd, c->cosb, c->sinb, st);
+    const int T = s.T, D = s.D, F = s.F, hq = s.H * s.hd, hkv = s.KV * s.hd;
+    bool ok = tmz::gemm_make_plan(&c->plan_qkv, c->xq, T, D, c->wexp, hq + 2 * hkv) &&
+              tmz::gemm_make_plan(&c->plan_o, c->xq, T, hq, c->wexp, D) &&
+              tmz::gemm_make_plan(&c->plan_gu, c->xq, T, D, c->wexp, 2 * F) &&
+              tmz::gemm_make_plan(&c->plan_down, c->xq, T, F, c->wexp, D);
+    if (!ok) {
+      delete c;
+      return TERMEZO_ECUDA;
+    }
+  }
+  c->code_sw = c->ma.sw_cur;
+  rc = sync_status(c);
+  if (rc) {
+    delete c;
+    return rc;
+  }
+  *out = c;
+  return TERMEZO_OK;
+}
+
+int termezo_load_params(termezo_ctx* c, const float* d_latents, const float* d_embed, const float* d_gains,
+                        const uint16_t* d_head) {
+  if (!c || !d_latents) return TERMEZO_EINVAL;
+  if (!c->sh.op && (!d_embed || !d_gains || !d_head)) return TERMEZO_EINVAL;
+  if ((uintptr_t)d_latents & 15) return TERMEZO_EINVAL;
+  c->latents = d_latents;
+  c->embed = d_embed;
+  c->gains = d_gains;
+  c->head = d_head;
+  return TERMEZO_OK;
+}
+
+int termezo_build_mask(termezo_ctx* c, double density, uint64_t* k0_out, float* xi0_out) {
+  if (!c) return TERMEZO_EINVAL;
+  if (!c->latents) return TERMEZO_ESTATE;
+  if (!(density > 0.0 && density <= 1.0)) return TERMEZO_EINVAL;
+  const uint64_t k0 = keep_count(density, c->sh.d);
+  if (k0 > keep_count(c->density, c->sh.d)) return TERMEZO_EINVAL;
+  const Shape& s = c->sh;
+  cudaStream_t st = c->stream;
+  tmz::SelectState sel{k0, 0u, 0u};
+  cudaMemcpyAsync(c->ma.sel, &sel, sizeof(sel), cudaMemcpyHostToDevice, st);
+  cudaMemsetAsync(c->ma.hist, 0, 2048 * sizeof(unsigned long long), st);
+  tmz::mask_build(c->ma, c->latents, k0, st);
+  int rc = cuda_status(c);
+  if (rc) return rc;
+  std::vector<uint32_t> off(s.P + 1);
+  cudaMemcpyAsync(off.data(), c->ma.off[0], (s.P + 1) * sizeof(uint32_t), cudaMemcpyDeviceToHost, st);
+  cudaMemcpyAsync(&sel, c->ma.sel, sizeof(sel), cudaMemcpyDeviceToHost, st);
+  rc = sync_status(c);
+  if (rc) return rc;
+  if (off[s.P] != k0) {
+    fprintf(stderr, "termezo: mask build selected %u weights, expected %llu\n", off[s.P], (unsigned long long)k0);
+    return TERMEZO_ECUDA;
+  }
+  std::vector<uint32_t> spre(s.P + 1, 0);
+  for (int p = 0; p < s.P; ++p) {
+    const uint32_t cnt = off[p + 1] - off[p];
+    uint32_t nb = (cnt + SPARSE_CHUNK - 1) / SPARSE_CHUNK;
+    spre[p + 1] = spre[p] + (nb ? nb : 1);
+  }
+  if (spre[s.P] > c->NBS_max) return TERMEZO_ECUDA;
+  c->ma.NBS = spre[s.P];
+  cudaMemcpyAsync((void*)c->ma.spre, spre.data(), (s.P + 1) * sizeof(uint32_t), cudaMemcpyHostToDevice, st);
+  tmz::mask_finish(c->ma, st);
+  c->cur = 0;
+  c->k0 = k0;
+  c->k_active = k0;
+  uint32_t key = sel.prefix;
+  float xi0 = 0.f;
+  if (k0) memcpy(&xi0, &key, 4);
+  c->xi0 = xi0;
+  c->t = 0;
+  c->updated = false;
+  c->pm_valid = false;
+  c->code_sw = c->ma.sw_cur;
+  rc = sync_status(c);
+  if (rc) return rc;
+  c->built = true;
+  if (k0_out) *k0_out = k0;
+  if (xi0_out) *xi0_out = xi0;
+  return TERMEZO_OK;
+}
+
+int termezo_forward_loss(termezo_ctx* c, const int32_t* d_tokens, const int32_t* d_targets, double* loss,
+                         double* per_seq) {
+  if (!c || !d_tokens || !d_targets) return TERMEZO_EINVAL;
+  if (c->sh.op || !c->built) return TERMEZO_ESTATE;
+  tmz::sparse_requant(c->ma, c->cur, 0, 0.f, 0, c->stream);
+  c->code_sw = c->ma.sw_cur;
+  int rc = run_forward(c, d_tokens, d_targets, c->ma.sw_cur, 0);
+  if (rc) return rc;
+  double l = 0;
+  cudaMemcpyAsync(&l, c->loss, sizeof(double), cudaMemcpyDeviceToHost, c->stream);
+  if (per_seq)
+    cudaMemcpyAsync(per_seq, c->per_seq, c->sh.B * sizeof(double), cudaMemcpyDeviceToHost, c->stream);
+  rc = sync_status(c);
+  if (rc) return rc;
+  if (loss) *loss = l;
+  return TERMEZO_OK;
+}
+
+int termezo_step(termezo_ctx* c, uint64_t seed, float eps, float lr, double density, const int32_t* d_tokens,
+                 const int32_t* d_targets, termezo_step_out* out, double* per_seq_plus, double* per_seq_minus) {
+  if (!c || !d_tokens || !d_targets || !out) return TERMEZO_EINVAL;
+  if (c->sh.op || !c->built) return TERMEZO_ESTATE;
+  if (!(eps > 0.f) || !std::isfinite(lr)) return TERMEZO_EINVAL;
+  const int warn = (density != c->density) ? TERMEZO_WMASKFIXED : TERMEZO_OK;
+  cudaStream_t st = c->stream;
+  cudaMemsetAsync(c->ma.counters, 0, 3 * sizeof(unsigned long long), st);
+  int rc;
+  if (c->updated) {
+    rc = do_shrink(c);
+    if (rc) return rc;
+  }
+  c->pm_valid = false;
+  const double k8 = 8.0 * (double)c->k_active;
+  {
+    ProfScope ps(c, 2, k8);
+    ensure_pm(c, seed, eps);
+  }
+  {
+    ProfScope ps(c, 2, k8);
+    tmz::sparse_requant(c->ma, c->cur, seed, eps, +1, st);
+  }
+  rc = run_forward(c, d_tokens, d_targets, c->ma.sw_plus, 0);
+  if (rc) return rc;
+  {
+    ProfScope ps(c, 2, k8);
+    tmz::sparse_requant(c->ma, c->cur, seed, eps, -1, st);
+  }
+  rc = run_forward(c, d_tokens, d_targets, c->ma.sw_minus, 1);
+  if (rc) return rc;
+  c->code_sw = c->ma.sw_minus;
+  tmz::launch_grad(c->loss, eps, c->g, st);
+  {
+    ProfScope ps(c, 2, 1.5 * k8);
+    tmz::sparse_update(c->ma, c->cur, seed, eps, lr, c->g, 0.0, 0, st);
+  }
+  c->pm_valid = false;
+  struct {
+    double loss[2];
+    double g;
+    unsigned long long cnt[4];
+    uint32_t k;
+  } h{};
+  cudaMemcpyAsync(h.loss, c->loss, 2 * sizeof(double), cudaMemcpyDeviceToHost, st);
+  cudaMemcpyAsync(&h.g, c->g, sizeof(double), cudaMemcpyDeviceToHost, st);
+  cudaMemcpyAsync(h.cnt, c->ma.counters, 4 * sizeof(unsigned long long), cudaMemcpyDeviceToHost, st);
+  cudaMemcpyAsync(&h.k, c->ma.off[c->cur] + c->sh.P, sizeof(uint32_t), cudaMemcpyDeviceToHost, st);
+  if (per_seq_plus)
+    cudaMemcpyAsync(per_seq_plus, c->per_seq, c->sh.B * sizeof(double), cudaMemcpyDeviceToHost, st);
+  if (per_seq_minus)
+    cudaMemcpyAsync(per_seq_minus, c->per_seq + c->sh.B, c->sh.B * sizeof(double), cudaMemcpyDeviceToHost, st);
+  rc = sync_status(c);
+  if (rc) return rc;
+  c->updated = true;
+  c->t += 1;
+  c->k_active = h.k;
+  out->loss_plus = h.loss[0];
+  out->loss_minus = h.loss[1];
+  out->g = h.g;
+  out->k_active = h.k;
+  out->n_flipped = h.cnt[0];
+  out->n_jumps = h.cnt[1];
+  out->n_dropped = h.cnt[2];
+  return warn;
+}
+
+int termezo_shrink(termezo_ctx* c, uint64_t* n_dropped) {
+  if (!c) return TERMEZO_EINVAL;
+  if (!c->built) return TERMEZO_ESTATE;
+  if (!c->updated) {
+    if (n_dropped) *n_dropped = 0;
+    return TERMEZO_OK;
+  }
+  cudaMemsetAsync(c->ma.counters + 2, 0, sizeof(unsigned long long), c->stream);
+  int rc = do_shrink(c);
+  if (rc) return rc;
+  c->updated = false;
+  if (n_dropped) {
+    unsigned long long d = 0;
+    uint32_t k = 0;
+    cudaMemcpyAsync(&d, c->ma.counters + 2, sizeof(d), cudaMemcpyDeviceToHost, c->stream);
+    cudaMemcpyAsync(&k, c->ma.off[c->cur] + c->sh.P, sizeof(k), cudaMemcpyDeviceToHost, c->stream);
+    rc = sync_status(c);
+    if (rc) return rc;
+    *n_dropped = d;
+    c->k_active = k;
+  }
+  return TERMEZO_OK;
+}
+
+int termezo_requantize(termezo_ctx* c, uint64_t seed, float eps, int sign) {
+  if (!c || sign < -1 || sign > 1) return TERMEZO_EINVAL;
+  if (!c->built) return TERMEZO_ESTATE;
+  if (sign != 0) {
+    if (!(eps > 0.f)) return TERMEZO_EINVAL;
+    ensure_pm(c, seed, eps);
+  }
+  tmz::sparse_requant(c->ma, c->cur, seed, eps, sign, c->stream);
+  c->code_sw = sign > 0 ? c->ma.sw_plus : (sign < 0 ? c->ma.sw_minus : c->ma.sw_cur);
+  return cuda_status(c);
+}
+
+int termezo_update(termezo_ctx* c, uint64_t seed, float eps, float lr, double g) {
+  if (!c) return TERMEZO_EINVAL;
+  if (!c->built) return TERMEZO_ESTATE;
+  if (!(eps > 0.f) || !std::isfinite(lr) || !std::isfinite(g)) return TERMEZO_EINVAL;
+  tmz::sparse_update(c->ma, c->cur, seed, eps, lr, nullptr, g, 1, c->stream);
+  c->updated = true;
+  c->pm_valid = false;
+  c->t += 1;
+  return cuda_status(c);
+}
+
+int termezo_bitlinear(termezo_ctx* c, int32_t proj, const uint16_t* d_x, int32_t M, int32_t* d_acc, float* d_y) {
+  if (!c || !d_x || proj < 0 || proj >= c->sh.P || M <= 0 || M > c->sh.T) return TERMEZO_EINVAL;
+  if (!c->built) return TERMEZO_ESTATE;
+  const int N = c->sh.N[proj], K = c->sh.K[proj];
+  if ((size_t)K > xq_cols(c->sh) || (size_t)N * K > wexp_elems(c->sh)) return TERMEZO_EINVAL;
+  cudaStream_t st = c->stream;
+  tmz::launch_norm_quant_bf16(d_x, M, K, c->xq, c->deq, st);
+  tmz::launch_expand_codes(c->ma.packed + c->sh.base[proj] / 16, (uint64_t)N, K, c->wexp, st);
+  GemmPlan plan;
+  if (!tmz::gemm_make_plan(&plan, c->xq, M, K, c->wexp, N)) return TERMEZO_ECUDA;
+  GemmArgs a{};
+  a.out = d_y;
+  a.ldo = N;
+  a.mode = 0;
+  a.acc_out = d_acc;
+  a.deq = c->deq;
+  a.sw = c->code_sw + proj;
+  a.n1 = a.n2 = N;
+  a.err = c->ma.err;
+  if (tmz::gemm_launch(plan, a, st) != cudaSuccess) return TERMEZO_ECUDA;
+  return cuda_status(c);
+}
+
+int termezo_state_sizes(termezo_ctx* c, uint64_t* d, uint64_t* k_active, int32_t* n_proj) {
+  if (!c) return TERMEZO_EINVAL;
+  uint32_t k = 0;
+  if (c->built) {
+    cudaMemcpyAsync(&k, c->ma.off[c->cur] + c->sh.P, sizeof(k), cudaMemcpyDeviceToHost, c->stream);
+    int rc = sync_status(c);
+    if (rc) return rc;
+  }
+  if (d) *d = c->sh.d;
+  if (k_active) *k_active = k;
+  if (n_proj) *n_proj = c->sh.P;
+  return TERMEZO_OK;
+}
+
+int termezo_export_state(termezo_ctx* c, uint32_t* h_idx, float* h_latents, uint32_t* h_packed, float* h_tau) {
+  if (!c) return TERMEZO_EINVAL;
+  if (!c->built) return TERMEZO_ESTATE;
+  cudaStream_t st = c->stream;
+  uint32_t k = 0;
+  cudaMemcpyAsync(&k, c->ma.off[c->cur] + c->sh.P, sizeof(k), cudaMemcpyDeviceToHost, st);
+  int rc = sync_status(c);
+  if (rc) return rc;
+  if (h_idx && k) cudaMemcpyAsync(h_idx, c->ma.idx[c->cur], k * sizeof(uint32_t), cudaMemcpyDeviceToHost, st);
+  if (h_latents && k) cudaMemcpyAsync(h_latents, c->ma.lat[c->cur], k * sizeof(float), cudaMemcpyDeviceToHost, st);
+  if (h_packed) cudaMemcpyAsync(h_packed, c->ma.packed, c->sh.d / 16 * sizeof(uint32_t), cudaMemcpyDeviceToHost, st);
+  if (h_tau) {
+    const int P = c->sh.P;
+    cudaMemcpyAsync(h_tau, c->ma.tau_cur, P * sizeof(float), cudaMemcpyDeviceToHost, st);
+    cudaMemcpyAsync(h_tau + P, c->ma.tau_plus, P * sizeof(float), cudaMemcpyDeviceToHost, st);
+    cudaMemcpyAsync(h_tau + 2 * P, c->ma.tau_minus, P * sizeof(float), cudaMemcpyDeviceToHost, st);
+  }
+  return sync_status(c);
+}
+
+int termezo_normal(uint64_t seed, const uint32_t* d_idx, uint64_t n, float* d_z, void* stream) {
+  if (n && (!d_idx || !d_z)) return TERMEZO_EINVAL;
+  tmz::launch_normal(seed, d_idx, n, d_z, reinterpret_cast<cudaStream_t>(stream));
+  return cudaGetLastError() == cudaSuccess ? TERMEZO_OK : TERMEZO_ECUDA;
+}
+
+int termezo_profile(termezo_ctx* c, int enable, termezo_profile_out* out) {
+  if (!c || enable < -1 || enable > 1) return TERMEZO_EINVAL;
+  if (enable == 1) {
+    int rc = sync_status(c);
+    if (rc) return rc;
+    c->prof.clear();
+    c->ev_used = 0;
+    c->launch_base = tmz::kernel_launches();
+    cudaMemsetAsync(c->ma.counters + 3, 0, sizeof(unsigned long long), c->stream);
+    c->prof_on = true;
+  } else if (enable == 0) {
+    c->prof_on = false;
+  }
+  if (out) {
+    int rc = sync_status(c);
+    if (rc) return rc;
+    memset(out, 0, sizeof(*out));
+    out->launches = tmz::kernel_launches() - c->launch_base;
+    for (const auto& r : c->prof) {
+      float ms = 0.f;
+      if (cudaEventElapsedTime(&ms, r.a, r.b) != cudaSuccess) return TERMEZO_ECUDA;
+      if (r.cat == 0) {
+        out->gemm_launches++;
+        out->gemm_ms += ms;
+        out->gemm_flops += r.work;
+      } else if (r.cat == 1) {
+        out->attn_launches++;
+        out->attn_ms += ms;
+        out->attn_flops += r.work;
+      } else {
+        out->sparse_launches++;
+        out->sparse_ms += ms;
+        out->sparse_bytes += r.work;
+      }
+    }
+    unsigned long long words = 0;
+    cudaMemcpy(&words, c->ma.counters + 3, sizeof(words), cudaMemcpyDeviceToHost);
+    out->sparse_bytes += 8.0 * (double)words;
+  }
+  return TERMEZO_OK;
+}
+
+void termezo_destroy(termezo_ctx* c) { delete c; }
+
+const char* termezo_strerror(int status) {
+  switch (status) {
+    case TERMEZO_OK: return "ok";
+    case TERMEZO_WMASKFIXED: return "mask density is fixed after termezo_build_mask; the new value was ignored";
+    case TERMEZO_EINVAL: return "invalid argument (shape, pointer, density or token id)";
+    case TERMEZO_ESTATE: return "call out of order for this context";
+    case TERMEZO_ENOMEM: return "workspace smaller than termezo_workspace_bytes";
+    case TERMEZO_ECUDA: return "CUDA error";
+    case TERMEZO_ETIMEOUT: return "a bounded device wait timed out";
+    default: return "unknown status";
+  }
+}
+
+}  // extern "C"

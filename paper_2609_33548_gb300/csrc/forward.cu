@@ -1,0 +1,470 @@
+// BitNet forward kernels other than the BitLinear GEMM: RMSNorm and
+// per-token absmax int8 activation quantisation, squared-ReLU gating,
+// 2-bit code expansion, embedding, RoPE, causal GQA attention, and the
+// label-token LM head with cross-entropy.
+#include <cuda_bf16.h>
+
+#include <cfloat>
+
+#include "common.cuh"
+#include "kernels.cuh"
+
+namespace tmz {
+
+namespace {
+
+__device__ __forceinline__ float block_sum(float v, float* red) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, o));
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) red[w] = v;
+  __syncthreads();
+  float t = 0.f;
+  for (int i = 0; i < (int)(blockDim.x >> 5); ++i) t = __fadd_rn(t, red[i]);
+  return t;
+}
+
+__device__ __forceinline__ float block_max(float v, float* red) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) red[w] = v;
+  __syncthreads();
+  float t = 0.f;
+  for (int i = 0; i < (int)(blockDim.x >> 5); ++i) t = fmaxf(t, red[i]);
+  return t;
+}
+
+__device__ __forceinline__ uint16_t int_to_bf16_bits(float v) {
+  return (uint16_t)(__float_as_uint(v) >> 16);  // exact for |v| <= 256 integers
+}
+
+__device__ __forceinline__ float quant_code(float h, float s) {
+  float v = rintf(__fmul_rn(h, s));
+  return fminf(fmaxf(v, -128.f), 127.f);
+}
+
+// One block per row.  h_k = (x_k * r) * g_k with r = 1/sqrt(mean(x^2)+1e-5)
+// (RMSNorm) or h_k = x_k; a = max(max|h|, 1e-5); q_k = rint(h_k * (127/a)).
+template <typename In>
+__global__ void k_norm_quant(const In* __restrict__ x, const float* __restrict__ gain, int D,
+                             uint16_t* __restrict__ q, float* __restrict__ deq) {
+  __shared__ float red[32];
+  const size_t row = blockIdx.x;
+  const In* xr = x + row * (size_t)D;
+  float r = 1.f;
+  if (gain) {
+    float ss = 0.f;
+    for (int k = threadIdx.x; k < D; k += blockDim.x) {
+      const float v = (float)xr[k];
+      ss = __fadd_rn(ss, __fmul_rn(v, v));
+    }
+    ss = block_sum(ss, red);
+    r = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(__fdiv_rn(ss, (float)D), 1e-5f)));
+  }
+  float amax = 0.f;
+  for (int k = threadIdx.x; k < D; k += blockDim.x) {
+    const float v = (float)xr[k];
+    const float h = gain ? __fmul_rn(__fmul_rn(v, r), gain[k]) : v;
+    amax = fmaxf(amax, fabsf(h));
+  }
+  const float a = fmaxf(block_max(amax, red), 1e-5f);
+  const float s = __fdiv_rn(127.f, a);
+  uint16_t* qr = q + row * (size_t)D;
+  for (int k = threadIdx.x; k < D; k += blockDim.x) {
+    const float v = (float)xr[k];
+    const float h = gain ? __fmul_rn(__fmul_rn(v, r), gain[k]) : v;
+    qr[k] = int_to_bf16_bits(quant_code(h, s));
+  }
+  if (threadIdx.x == 0) deq[row] = __fdiv_rn(a, 127.f);
+}
+
+struct Bf16In {
+  uint16_t bits;
+  __device__ __forceinline__ explicit operator float() const { return __uint_as_float((uint32_t)bits << 16); }
+};
+
+// h_k = relu(gate_k)^2 * up_k, then per-row absmax int8.
+__global__ void k_relu2_quant(const float* __restrict__ gu, int F, uint16_t* __restrict__ q,
+                              float* __restrict__ deq) {
+  __shared__ float red[32];
+  const size_t row = blockIdx.x;
+  const float* g = gu + row * (size_t)(2 * F);
+  const float* u = g + F;
+  float amax = 0.f;
+  for (int k = threadIdx.x; k < F; k += blockDim.x) {
+    const float gr = fmaxf(g[k], 0.f);
+    amax = fmaxf(amax, fabsf(__fmul_rn(__fmul_rn(gr, gr), u[k])));
+  }
+  const float a = fmaxf(block_max(amax, red), 1e-5f);
+  const float s = __fdiv_rn(127.f, a);
+  uint16_t* qr = q + row * (size_t)F;
+  for (int k = threadIdx.x; k < F; k += blockDim.x) {
+    const float gr = fmaxf(g[k], 0.f);
+    qr[k] = int_to_bf16_bits(quant_code(__fmul_rn(__fmul_rn(gr, gr), u[k]), s));
+  }
+  if (threadIdx.x == 0) deq[row] = __fdiv_rn(a, 127.f);
+}
+
+// One thread per packed word: 16 codes -> 16 bf16 values (32 bytes).
+__global__ void k_expand_codes(const uint32_t* __restrict__ words, uint64_t n_words, uint16_t* __restrict__ out) {
+  const uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n_words) return;
+  const uint32_t w = words[i];
+  uint32_t v[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const uint32_t c0 = (w >> (4 * j)) & 3u, c1 = (w >> (4 * j + 2)) & 3u;
+    const uint32_t b0 = c0 == 2u ? 0x3F80u : (c0 == 0u ? 0xBF80u : 0u);
+    const uint32_t b1 = c1 == 2u ? 0x3F80u : (c1 == 0u ? 0xBF80u : 0u);
+    v[j] = b0 | (b1 << 16);
+  }
+  uint4* o = reinterpret_cast<uint4*>(out + i * 16);
+  o[0] = make_uint4(v[0], v[1], v[2], v[3]);
+  o[1] = make_uint4(v[4], v[5], v[6], v[7]);
+}
+
+__global__ void k_embed(const int32_t* __restrict__ tok, const float* __restrict__ embed, int D, int V,
+                        float* __restrict__ x, unsigned* err) {
+  const size_t t = blockIdx.x;
+  int id = tok[t];
+  if (id < 0 || id >= V) {
+    if (threadIdx.x == 0) atomicOr(err, ERR_BOUNDS);
+    id = 0;
+  }
+  const float* e = embed + (size_t)id * D;
+  for (int k = threadIdx.x; k < D; k += blockDim.x) x[t * D + k] = e[k];
+}
+
+__global__ void k_rope_tables(int S, int hd, float* cosb, float* sinb) {
+  const int half = hd / 2;
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= S * half) return;
+  const int pos = i / half, j = i % half;
+  const double inv = pow(10000.0, -(2.0 * j) / (double)hd);
+  const double ang = (double)pos * inv;
+  cosb[i] = (float)cos(ang);
+  sinb[i] = (float)sin(ang);
+}
+
+// One block per token; threads over (head, j < hd/2) pairs of Q and K, and
+// over V elements.
+__global__ void k_rope_pack(const float* __restrict__ qkv, const float* __restrict__ cosb,
+                            const float* __restrict__ sinb, int S, int H, int KV, int hd,
+                            uint16_t* __restrict__ q, uint16_t* __restrict__ k) {
+  const int t = blockIdx.x;
+  const int b = t / S, pos = t % S;
+  const int half = hd / 2;
+  const int width = (H + 2 * KV) * hd;
+  const float* row = qkv + (size_t)t * width;
+  const float* cr = cosb + (size_t)pos * half;
+  const float* sr = sinb + (size_t)pos * half;
+  for (int i = threadIdx.x; i < (H + KV) * half; i += blockDim.x) {
+    const int head = i / half, j = i % half;
+    const float* src = row + head * hd;
+    const float x1 = src[j], x2 = src[j + half];
+    const float c = cr[j], s = sr[j];
+    const float o1 = __fsub_rn(__fmul_rn(x1, c), __fmul_rn(x2, s));
+    const float o2 = __fadd_rn(__fmul_rn(x2, c), __fmul_rn(x1, s));
+    __nv_bfloat16 b1 = __float2bfloat16_rn(o1), b2 = __float2bfloat16_rn(o2);
+    uint16_t* dst;
+    if (head < H)
+      dst = q + (((size_t)b * H + head) * S + pos) * hd;
+    else
+      dst = k + (((size_t)b * KV + (head - H)) * S + pos) * hd;
+    dst[j] = *reinterpret_cast<uint16_t*>(&b1);
+    dst[j + half] = *reinterpret_cast<uint16_t*>(&b2);
+  }
+}
+
+// V [B*S, KV*hd] (inside qkv) -> Vt bf16 [B, KV, hd, S] through a 32x32 tile.
+__global__ void k_pack_vt(const float* __restrict__ qkv, int S, int H, int KV, int hd, uint16_t* __restrict__ vt) {
+  __shared__ float tile[32][33];
+  const int b = blockIdx.z / KV, kvh = blockIdx.z % KV;
+  const int s0 = blockIdx.x * 32, d0 = blockIdx.y * 32;
+  const int width = (H + 2 * KV) * hd;
+  const float* v = qkv + (size_t)(H + KV) * hd + (size_t)kvh * hd;
+  for (int r = threadIdx.y; r < 32; r += blockDim.y) {
+    const int s = s0 + r, d = d0 + threadIdx.x;
+    tile[r][threadIdx.x] = (s < S && d < hd) ? v[((size_t)b * S + s) * width + d] : 0.f;
+  }
+  __syncthreads();
+  for (int r = threadIdx.y; r < 32; r += blockDim.y) {
+    const int d = d0 + r, s = s0 + threadIdx.x;
+    if (d < hd && s < S) {
+      __nv_bfloat16 bv = __float2bfloat16_rn(tile[threadIdx.x][r]);
+      vt[(((size_t)b * KV + kvh) * hd + d) * S + s] = *reinterpret_cast<uint16_t*>(&bv);
+    }
+  }
+}
+
+__device__ __forceinline__ void mma_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat16 l = __float2bfloat16_rn(lo), h = __float2bfloat16_rn(hi);
+  return (uint32_t)(*reinterpret_cast<uint16_t*>(&l)) | ((uint32_t)(*reinterpret_cast<uint16_t*>(&h)) << 16);
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
+
+// Causal attention, two passes over the keys: pass 1 finds the exact row
+// maximum of the scores, pass 2 forms P = bf16(exp(s - max)), l = sum P and
+// O = P V / l.  4 warps x 16 query rows per block; bf16 mma.sync tiles.
+template <int HD>
+__global__ void __launch_bounds__(128) k_attention(const uint16_t* __restrict__ Q, const uint16_t* __restrict__ K,
+                                                   const uint16_t* __restrict__ Vt, int S, int H, int KV,
+                                                   float scale, float* __restrict__ out) {
+  constexpr int KP = HD + 8, VP = 64 + 8;
+  __shared__ __align__(16) uint16_t Ks[64 * KP];
+  __shared__ __align__(16) uint16_t Vs[HD * VP];
+  const int qblk = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int kvh = h / (H / KV);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int g = lane >> 2, c = lane & 3;
+  const int q0 = qblk * 64 + warp * 16;
+  const uint16_t* Qp = Q + ((size_t)b * H + h) * S * HD;
+  const uint16_t* Kp = K + ((size_t)b * KV + kvh) * S * HD;
+  const uint16_t* Vp = Vt + ((size_t)b * KV + kvh) * HD * S;
+
+  uint32_t qa[HD / 16][4];
+#pragma unroll
+  for (int kk = 0; kk < HD / 16; ++kk) {
+    const int col = kk * 16 + 2 * c;
+    qa[kk][0] = *reinterpret_cast<const uint32_t*>(Qp + (size_t)(q0 + g) * HD + col);
+    qa[kk][1] = *reinterpret_cast<const uint32_t*>(Qp + (size_t)(q0 + g + 8) * HD + col);
+    qa[kk][2] = *reinterpret_cast<const uint32_t*>(Qp + (size_t)(q0 + g) * HD + col + 8);
+    qa[kk][3] = *reinterpret_cast<const uint32_t*>(Qp + (size_t)(q0 + g + 8) * HD + col + 8);
+  }
+  const int nkb = qblk + 1;
+  const int r0 = q0 + g, r1 = q0 + g + 8;
+  float mx0 = -FLT_MAX, mx1 = -FLT_MAX;
+
+  auto load_k = [&](int kb) {
+    for (int i = threadIdx.x; i < 64 * (HD / 8); i += 128) {
+      const int r = i / (HD / 8), c8 = i % (HD / 8);
+      *reinterpret_cast<uint4*>(&Ks[r * KP + c8 * 8]) =
+          *reinterpret_cast<const uint4*>(Kp + (size_t)(kb * 64 + r) * HD + c8 * 8);
+    }
+  };
+  auto scores = [&](float (&sacc)[8][4]) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      sacc[j][0] = sacc[j][1] = sacc[j][2] = sacc[j][3] = 0.f;
+#pragma unroll
+      for (int kk = 0; kk < HD / 16; ++kk) {
+        const uint16_t* kr = &Ks[(j * 8 + g) * KP + kk * 16 + 2 * c];
+        mma_16816(sacc[j], qa[kk], *reinterpret_cast<const uint32_t*>(kr), *reinterpret_cast<const uint32_t*>(kr + 8));
+      }
+    }
+  };
+
+  for (int kb = 0; kb < nkb; ++kb) {
+    __syncthreads();
+    load_k(kb);
+    __syncthreads();
+    float sacc[8][4];
+    scores(sacc);
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int key = kb * 64 + j * 8 + 2 * c + (e & 1);
+        const int row = e < 2 ? r0 : r1;
+        if (key <= row) {
+          const float s = __fmul_rn(sacc[j][e], scale);
+          if (e < 2) mx0 = fmaxf(mx0, s); else mx1 = fmaxf(mx1, s);
+        }
+      }
+  }
+#pragma unroll
+  for (int o = 1; o <= 2; o <<= 1) {
+    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
+    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+  }
+
+  float oacc[HD / 8][4];
+#pragma unroll
+  for (int n = 0; n < HD / 8; ++n) oacc[n][0] = oacc[n][1] = oacc[n][2] = oacc[n][3] = 0.f;
+  float l0 = 0.f, l1 = 0.f;
+  for (int kb = 0; kb < nkb; ++kb) {
+    __syncthreads();
+    load_k(kb);
+    for (int i = threadIdx.x; i < HD * 8; i += 128) {
+      const int d = i / 8, c8 = i % 8;
+      *reinterpret_cast<uint4*>(&Vs[d * VP + c8 * 8]) =
+          *reinterpret_cast<const uint4*>(Vp + (size_t)d * S + kb * 64 + c8 * 8);
+    }
+    __syncthreads();
+    float sacc[8][4];
+    scores(sacc);
+    uint32_t pf[8][2];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      float pv[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int key = kb * 64 + j * 8 + 2 * c + (e & 1);
+        const int row = e < 2 ? r0 : r1;
+        pv[e] = key <= row ? expf(__fsub_rn(__fmul_rn(sacc[j][e], scale), e < 2 ? mx0 : mx1)) : 0.f;
+      }
+      pf[j][0] = pack_bf16(pv[0], pv[1]);
+      pf[j][1] = pack_bf16(pv[2], pv[3]);
+      l0 = __fadd_rn(__fadd_rn(l0, bf16_lo(pf[j][0])), bf16_hi(pf[j][0]));
+      l1 = __fadd_rn(__fadd_rn(l1, bf16_lo(pf[j][1])), bf16_hi(pf[j][1]));
+    }
+#pragma unroll
+    for (int kc = 0; kc < 4; ++kc) {
+      const uint32_t a[4] = {pf[2 * kc][0], pf[2 * kc][1], pf[2 * kc + 1][0], pf[2 * kc + 1][1]};
+#pragma unroll
+      for (int n = 0; n < HD / 8; ++n) {
+        const uint16_t* vr = &Vs[(n * 8 + g) * VP + kc * 16 + 2 * c];
+        mma_16816(oacc[n], a, *reinterpret_cast<const uint32_t*>(vr), *reinterpret_cast<const uint32_t*>(vr + 8));
+      }
+    }
+  }
+#pragma unroll
+  for (int o = 1; o <= 2; o <<= 1) {
+    l0 = __fadd_rn(l0, __shfl_xor_sync(0xffffffffu, l0, o));
+    l1 = __fadd_rn(l1, __shfl_xor_sync(0xffffffffu, l1, o));
+  }
+  float* o0 = out + ((size_t)b * S + r0) * (size_t)(H * HD) + h * HD;
+  float* o1 = out + ((size_t)b * S + r1) * (size_t)(H * HD) + h * HD;
+#pragma unroll
+  for (int n = 0; n < HD / 8; ++n) {
+    const int col = n * 8 + 2 * c;
+    *reinterpret_cast<float2*>(o0 + col) = make_float2(__fdiv_rn(oacc[n][0], l0), __fdiv_rn(oacc[n][1], l0));
+    *reinterpret_cast<float2*>(o1 + col) = make_float2(__fdiv_rn(oacc[n][2], l1), __fdiv_rn(oacc[n][3], l1));
+  }
+}
+
+// Loss mode 0.  One block per sequence: final RMSNorm of the last position,
+// h -> bf16, logits over the C label tokens accumulated in float64 (every
+// bf16 product is exact in float64), cross-entropy in float64.
+__global__ void k_head_ce_last(const float* __restrict__ x, const float* __restrict__ gain,
+                               const uint16_t* __restrict__ head, const int32_t* __restrict__ targets, int S,
+                               int D, int V, int C, double* __restrict__ per_seq) {
+  __shared__ float red[32];
+  __shared__ double dred[32];
+  __shared__ double logits[64];
+  const int b = blockIdx.x;
+  const float* xr = x + ((size_t)b * S + (S - 1)) * D;
+  float ss = 0.f;
+  for (int k = threadIdx.x; k < D; k += blockDim.x) ss = __fadd_rn(ss, __fmul_rn(xr[k], xr[k]));
+  ss = block_sum(ss, red);
+  const float r = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(__fdiv_rn(ss, (float)D), 1e-5f)));
+  for (int cl = 0; cl < C; ++cl) {
+    const uint16_t* wr = head + (size_t)(V - C + cl) * D;
+    double acc = 0.0;
+    for (int k = threadIdx.x; k < D; k += blockDim.x) {
+      const float hv = __bfloat162float(__float2bfloat16_rn(__fmul_rn(__fmul_rn(xr[k], r), gain[k])));
+      acc += (double)hv * (double)__uint_as_float((uint32_t)wr[k] << 16);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    __syncthreads();
+    if ((threadIdx.x & 31) == 0) dred[threadIdx.x >> 5] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      double t = 0.0;
+      for (int i = 0; i < (int)(blockDim.x >> 5); ++i) t += dred[i];
+      logits[cl] = t;
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double m = -DBL_MAX;
+    for (int cl = 0; cl < C; ++cl) m = fmax(m, logits[cl]);
+    double se = 0.0;
+    for (int cl = 0; cl < C; ++cl) se += exp(logits[cl] - m);
+    int tg = targets[b];
+    tg = tg < 0 ? 0 : (tg >= C ? C - 1 : tg);
+    per_seq[b] = m + log(se) - logits[tg];
+  }
+}
+
+__global__ void k_mean(const double* __restrict__ v, int n, double* __restrict__ out) {
+  if (threadIdx.x == 0 && blockIdx.x == 0) {
+    double t = 0.0;
+    for (int i = 0; i < n; ++i) t += v[i];
+    *out = t / (double)n;
+  }
+}
+
+}  // namespace
+
+uint64_t& kernel_launches() {
+  static thread_local uint64_t n = 0;
+  return n;
+}
+
+void launch_norm_quant(const float* x, const float* gain, int M, int D, uint16_t* q, float* deq, cudaStream_t s) {
+  kernel_launches() += 1;
+  k_norm_quant<float><<<M, 256, 0, s>>>(x, gain, D, q, deq);
+}
+
+void launch_norm_quant_bf16(const uint16_t* x, int M, int D, uint16_t* q, float* deq, cudaStream_t s) {
+  kernel_launches() += 1;
+  k_norm_quant<Bf16In><<<M, 256, 0, s>>>(reinterpret_cast<const Bf16In*>(x), nullptr, D, q, deq);
+}
+
+void launch_relu2_quant(const float* gu, int M, int F, uint16_t* q, float* deq, cudaStream_t s) {
+  kernel_launches() += 1;
+  k_relu2_quant<<<M, 256, 0, s>>>(gu, F, q, deq);
+}
+
+void launch_expand_codes(const uint32_t* words, uint64_t rows, int K, uint16_t* out, cudaStream_t s) {
+  kernel_launches() += 1;
+  const uint64_t n = rows * (uint64_t)(K / 16);
+  k_expand_codes<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(words, n, out);
+}
+
+void launch_embed(const int32_t* tok, const float* embed, int T, int D, int V, float* x, unsigned* err,
+                  cudaStream_t s) {
+  kernel_launches() += 1;
+  k_embed<<<T, 256, 0, s>>>(tok, embed, D, V, x, err);
+}
+
+void launch_rope_tables(int S, int hd, float* cosb, float* sinb, cudaStream_t s) {
+  kernel_launches() += 1;
+  const int n = S * hd / 2;
+  k_rope_tables<<<(n + 255) / 256, 256, 0, s>>>(S, hd, cosb, sinb);
+}
+
+void launch_rope_pack(const float* qkv, const float* cosb, const float* sinb, int B, int S, int H, int KV, int hd,
+                      uint16_t* q, uint16_t* k, uint16_t* vt, cudaStream_t s) {
+  kernel_launches() += 2;
+  k_rope_pack<<<B * S, 256, 0, s>>>(qkv, cosb, sinb, S, H, KV, hd, q, k);
+  dim3 grid((S + 31) / 32, (hd + 31) / 32, B * KV);
+  k_pack_vt<<<grid, dim3(32, 8), 0, s>>>(qkv, S, H, KV, hd, vt);
+}
+
+void launch_attention(const uint16_t* q, const uint16_t* k, const uint16_t* vt, int B, int S, int H, int KV, int hd,
+                      float* out, cudaStream_t s) {
+  kernel_launches() += 1;
+  dim3 grid(S / 64, H, B);
+  const float scale = 1.0f / sqrtf((float)hd);
+  switch (hd) {
+    case 64: k_attention<64><<<grid, 128, 0, s>>>(q, k, vt, S, H, KV, scale, out); break;
+    case 96: k_attention<96><<<grid, 128, 0, s>>>(q, k, vt, S, H, KV, scale, out); break;
+    case 128: k_attention<128><<<grid, 128, 0, s>>>(q, k, vt, S, H, KV, scale, out); break;
+    default: break;
+  }
+}
+
+void launch_head_ce_last(const float* x, const float* gain, const uint16_t* head, const int32_t* targets, int B,
+                         int S, int D, int V, int C, double* per_seq, double* total, cudaStream_t s) {
+  kernel_launches() += 2;
+  k_head_ce_last<<<B, 256, 0, s>>>(x, gain, head, targets, S, D, V, C, per_seq);
+  k_mean<<<1, 32, 0, s>>>(per_seq, B, total);
+}
+
+}  // namespace tmz

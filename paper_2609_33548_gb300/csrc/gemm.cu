@@ -1,0 +1,333 @@
+// BitLinear GEMM on the 5th-generation tensor cores (sm_103a).
+//
+// acc[m, n] = sum_k q[m, k] * c[n, k] with q the int8 activation codes and c
+// the ternary codes, both held as bf16 (every int8 value and every ternary
+// value is exact in bf16, every product is exact, and every partial sum is
+// an integer of magnitude <= 128 * K < 2^24, so the fp32 accumulator holds
+// the int32 accumulator exactly).  The int8 MMA kind does not exist on
+// sm_103a (ptxas: "Feature '.kind::i8' not supported on .target
+// 'sm_103a'"), so this exact-integer bf16 formulation is the tensor-core
+// path.
+//
+// Structure: a persistent grid (one CTA per SM) walks 128 x BN output tiles;
+// warp 0 issues TMA loads of 128 x 64 (A) and BN x 64 (B) bf16 tiles with
+// 128-byte swizzle into a STAGES-deep ring; one thread of warp 1 issues
+// tcgen05.mma (M = 128, N = BN, K = 16) into one of two fp32 accumulators in
+// tensor memory; warps 2-5 read the other accumulator back with tcgen05.ld,
+// transpose it through shared memory and store coalesced rows of
+// y = acc * (a/127)[m] * s_w[n] (or add them into the residual stream).
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
+#include "kernels.cuh"
+
+namespace tmz {
+
+namespace {
+
+constexpr int BM = 128;
+constexpr int BK = 64;
+constexpr int STAGES = 4;
+constexpr int GEMM_THREADS = 192;
+constexpr int A_BYTES = BM * BK * 2;
+
+constexpr int EPI_WARPS = 4;
+constexpr int EPI_LD = 33;  // staging row stride (floats): conflict-free transpose
+
+template <int BN>
+struct GemmSmem {
+  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int EPI_OFF = STAGES * STAGE_BYTES;
+  static constexpr int EPI_BYTES = EPI_WARPS * 32 * EPI_LD * 4;
+  static constexpr int BAR_OFF = EPI_OFF + EPI_BYTES;
+  static constexpr int BYTES = BAR_OFF + 256 + 1024;  // barriers + alignment slack
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count));
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Waits for the phase with the given parity; false after kWaitNs.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (globaltimer_ns() - t0 > kWaitNs) return false;
+    __nanosleep(64);
+  }
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y,
+                                            uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"((uint64_t)map), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+
+// Shared-memory matrix descriptor (tcgen05): K-major, 128-byte swizzle,
+// 8-row atoms of 128 B stacked every 1024 B (SBO), version 1.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
+         ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+// Instruction descriptor: kind::f16, D = F32, A = B = BF16, K-major both.
+template <int BN>
+__device__ __forceinline__ uint32_t idesc_bf16() {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
+}
+
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
+        "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
+        "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
+        "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+// Persistent: CTA c processes tiles c, c + gridDim.x, ... (m fastest, so the
+// CTAs running together share the B tiles and sweep A through L2).  The
+// accumulator is double-buffered in tensor memory (2 x BN columns) so that
+// the epilogue of one tile overlaps the main loop of the next.
+template <int BN>
+__global__ void __launch_bounds__(GEMM_THREADS, 1)
+    k_bitlinear_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                     GemmArgs p) {
+  using L = GemmSmem<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  const uint32_t sbase = smem_u32(smem);
+  const uint32_t bar_full = sbase + L::BAR_OFF;        // STAGES x 8 B
+  const uint32_t bar_empty = bar_full + STAGES * 8;    // STAGES x 8 B
+  const uint32_t bar_tfull = bar_empty + STAGES * 8;   // 2 x 8 B: accumulator ready
+  const uint32_t bar_tempty = bar_tfull + 16;          // 2 x 8 B: accumulator drained
+  uint32_t* tmem_slot = (uint32_t*)(smem + L::BAR_OFF + 2 * STAGES * 8 + 32);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n_mt = (p.M + BM - 1) / BM, n_nt = (p.N + BN - 1) / BN;
+  const int tiles = n_mt * n_nt;
+  const int KB = (p.K + BK - 1) / BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(bar_full + 8 * s, 1);
+      mbar_init(bar_empty + 8 * s, 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(bar_tfull + 8 * b, 1);
+      mbar_init(bar_tempty + 8 * b, EPI_WARPS);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(2 * BN));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  const uint32_t tmem = *tmem_slot;
+  bool ok = true;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmA) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmB) : "memory");
+      uint32_t it = 0;
+      for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
+        const int m0 = (tile % n_mt) * BM, n0 = (tile / n_mt) * BN;
+        for (int kb = 0; kb < KB; ++kb, ++it) {
+          const uint32_t s = it % STAGES, use = it / STAGES;
+          if (it >= (uint32_t)STAGES && !(ok = mbar_wait(bar_empty + 8 * s, (use & 1u) ^ 1u))) break;
+          const uint32_t sa = sbase + s * L::STAGE_BYTES;
+          mbar_expect_tx(bar_full + 8 * s, L::STAGE_BYTES);
+          tma_load_2d(sa, &tmA, kb * BK, m0, bar_full + 8 * s);
+          tma_load_2d(sa + A_BYTES, &tmB, kb * BK, n0, bar_full + 8 * s);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16<BN>();
+      uint32_t it = 0, local = 0;
+      for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x, ++local) {
+        const uint32_t b = local & 1u, j = local >> 1;
+        if (j >= 1 && !(ok = mbar_wait(bar_tempty + 8 * b, (j & 1u) ^ 1u))) break;
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        const uint32_t d = tmem + b * BN;
+        for (int kb = 0; kb < KB; ++kb, ++it) {
+          const uint32_t s = it % STAGES;
+          if (!(ok = mbar_wait(bar_full + 8 * s, (it / STAGES) & 1u))) break;
+          asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+          const uint32_t sa = sbase + s * L::STAGE_BYTES;
+          const uint64_t da = sw128_desc(sa), db = sw128_desc(sa + A_BYTES);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            mma_bf16(d, da + (uint64_t)(2 * k), db + (uint64_t)(2 * k), idesc, (kb | k) ? 1u : 0u);
+          mma_commit(bar_empty + 8 * s);
+        }
+        if (!ok) break;
+        mma_commit(bar_tfull + 8 * b);
+      }
+    }
+  } else {
+    // Epilogue warps 2..5: warp w may access TMEM lanes 32*(w % 4) .. +31.
+    const int quarter = warp & 3;
+    float* stage = reinterpret_cast<float*>(smem + L::EPI_OFF) + (warp - 2) * 32 * EPI_LD;
+    const float s0 = p.sw[0], s1 = p.sw[1], s2 = p.sw[2];
+    uint32_t local = 0;
+    for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++local) {
+      const int m0 = (tile % n_mt) * BM, n0 = (tile / n_mt) * BN;
+      const uint32_t b = local & 1u, j = local >> 1;
+      ok = mbar_wait(bar_tfull + 8 * b, j & 1u);
+      if (!ok) break;
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      const int row0 = m0 + quarter * 32;
+      for (int c = 0; c < BN / 32; ++c) {
+        uint32_t r[32];
+        tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + b * BN + (uint32_t)(c * 32), r);
+#pragma unroll
+        for (int q = 0; q < 32; ++q) stage[lane * EPI_LD + q] = __uint_as_float(r[q]);
+        __syncwarp();
+        const int col = n0 + c * 32 + lane;
+        const float sw = col < p.n1 ? s0 : (col < p.n2 ? s1 : s2);
+        if (col < p.N) {
+          for (int rr = 0; rr < 32; ++rr) {
+            const int row = row0 + rr;
+            if (row >= p.M) break;
+            const float acc = stage[rr * EPI_LD + lane];
+            if (p.acc_out) p.acc_out[(size_t)row * p.N + col] = __float2int_rn(acc);
+            if (p.out) {
+              const float y = __fmul_rn(__fmul_rn(acc, p.deq[row]), sw);
+              float* o = p.out + (size_t)row * p.ldo + col;
+              *o = p.mode ? __fadd_rn(*o, y) : y;
+            }
+          }
+        }
+        __syncwarp();
+      }
+      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar_tempty + 8 * b);
+    }
+  }
+  if (!ok && p.err) atomicOr(p.err, ERR_TIMEOUT);
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  if (warp == 1) {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(2 * BN));
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = (PFN_cuTensorMapEncodeTiled_v12000)ptr;
+  }
+  return fn;
+}
+
+}  // namespace
+
+constexpr int GEMM_BN = 256;
+
+bool encode_bf16_kmajor(CUtensorMap* map, const void* base, uint64_t rows, uint64_t k, uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (!fn || (k * 2) % 16 != 0 || ((uintptr_t)base & 15)) return false;
+  cuuint64_t dims[2] = {k, rows};
+  cuuint64_t strides[1] = {k * 2};
+  cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+bool gemm_make_plan(GemmPlan* plan, const uint16_t* a, int M, int K, const uint16_t* b, int N) {
+  plan->M = M;
+  plan->N = N;
+  plan->K = K;
+  return encode_bf16_kmajor(&plan->a, a, (uint64_t)M, (uint64_t)K, BM) &&
+         encode_bf16_kmajor(&plan->b, b, (uint64_t)N, (uint64_t)K, GEMM_BN);
+}
+
+cudaError_t gemm_launch(const GemmPlan& plan, GemmArgs args, cudaStream_t stream) {
+  static bool attr_set = false;
+  constexpr int smem = GemmSmem<GEMM_BN>::BYTES;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(k_bitlinear_gemm<GEMM_BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  static int sms = 0;
+  if (!sms) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) sms = 148;
+  }
+  args.M = plan.M;
+  args.N = plan.N;
+  args.K = plan.K;
+  const int tiles = ((plan.N + GEMM_BN - 1) / GEMM_BN) * ((plan.M + BM - 1) / BM);
+  dim3 grid(tiles < sms ? tiles : sms);
+  ++kernel_launches();
+  k_bitlinear_gemm<GEMM_BN><<<grid, GEMM_THREADS, smem, stream>>>(plan.a, plan.b, args);
+  return cudaGetLastError();
+}
+
+}  // namespace tmz

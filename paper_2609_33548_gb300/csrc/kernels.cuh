@@ -1,0 +1,72 @@
+// Declarations shared by the TerMeZO translation units (host side).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "common.cuh"
+
+namespace tmz {
+
+// Kernels launched by the calling thread (every launcher adds its count).
+uint64_t& kernel_launches();
+
+// ---------------------------------------------------------------- GEMM ----
+struct GemmArgs {
+  int M, N, K;          // filled from the plan
+  float* out;           // fp32 [M, ldo] output (nullable)
+  int ldo;
+  int mode;             // 0: out = y; 1: out += y (residual stream)
+  int32_t* acc_out;     // raw int32 accumulators [M, N] (nullable)
+  const float* deq;     // [M] per-row activation scale a/127
+  const float* sw;      // three column-segment weight scales sw[0..2]
+  int n1, n2;           // segment bounds: [0,n1) sw[0], [n1,n2) sw[1], [n2,N) sw[2]
+  unsigned* err;        // device error word
+};
+
+struct GemmPlan {
+  CUtensorMap a, b;
+  int M, N, K;
+};
+
+bool gemm_make_plan(GemmPlan* plan, const uint16_t* a, int M, int K, const uint16_t* b, int N);
+cudaError_t gemm_launch(const GemmPlan& plan, GemmArgs args, cudaStream_t stream);
+
+// ------------------------------------------------------------ forward ----
+// Per-row absmax int8 quantisation of h = RMSNorm(x) (gain != nullptr) or
+// of h = x (gain == nullptr): q bf16 [M, D] (ld = D), deq[m] = a / 127.
+void launch_norm_quant(const float* x, const float* gain, int M, int D, uint16_t* q, float* deq,
+                       cudaStream_t s);
+// h = relu(gate)^2 * up for gu = [gate | up] fp32 [M, 2F]; quantised as above.
+void launch_relu2_quant(const float* gu, int M, int F, uint16_t* q, float* deq, cudaStream_t s);
+// Packed 2-bit codes [rows, K/16] -> bf16 {-1, 0, +1} [rows, K].
+void launch_expand_codes(const uint32_t* words, uint64_t rows, int K, uint16_t* out, cudaStream_t s);
+// x[t] = embed[tok[t]].
+void launch_embed(const int32_t* tok, const float* embed, int T, int D, int V, float* x, unsigned* err,
+                  cudaStream_t s);
+// Per-row absmax int8 quantisation of raw bf16 activations (no norm).
+void launch_norm_quant_bf16(const uint16_t* x, int M, int D, uint16_t* q, float* deq, cudaStream_t s);
+// RoPE tables cos/sin fp32 [S, hd/2] computed in float64, rounded to fp32.
+void launch_rope_tables(int S, int hd, float* cosb, float* sinb, cudaStream_t s);
+// qkv fp32 [B*S, (H + 2 KV) hd] -> Q bf16 [B, H, S, hd] (RoPE), K bf16
+// [B, KV, S, hd] (RoPE), Vt bf16 [B, KV, hd, S] (transposed).
+void launch_rope_pack(const float* qkv, const float* cosb, const float* sinb, int B, int S, int H, int KV,
+                      int hd, uint16_t* q, uint16_t* k, uint16_t* vt, cudaStream_t s);
+// Causal GQA attention -> out fp32 [B*S, H*hd].
+void launch_attention(const uint16_t* q, const uint16_t* k, const uint16_t* vt, int B, int S, int H, int KV,
+                      int hd, float* out, cudaStream_t s);
+// Final RMSNorm + LM head over the label tokens at the last position and
+// cross-entropy (loss mode 0): per_seq[b] (fp64), total = mean (fp64).
+void launch_head_ce_last(const float* x, const float* gain, const uint16_t* head, const int32_t* targets,
+                         int B, int S, int D, int V, int C, double* per_seq, double* total, cudaStream_t s);
+
+// ------------------------------------------------------ mask / sparse ----
+struct ProjTable {
+  int P;                      // number of projections
+  const uint64_t* base;       // [P+1] global base index of each projection (base[P] = d)
+  const uint32_t* blk_prefix; // [P+1] prefix of dense blocks per projection
+};
+
+}  // namespace tmz

@@ -1,0 +1,604 @@
+// Mask selection (Eqs. 2-5) and the sparse perturb / requantise / update
+// passes of Algorithm 1 over the sparse latent store.
+//
+// Dense passes (mask build) read the caller's dense latents in blocks of
+// 4096 elements that never straddle two projections.  Sparse passes read
+// the active-index list and its fp32 latents; each projection owns a fixed
+// number of blocks, each block a contiguous part of the projection's
+// segment of the (sorted) active list.  Per-projection sums of |w| are exact
+// (ExactSum), so tau and therefore every ternary code is independent of
+// the order in which blocks are reduced.
+#include "common.cuh"
+#include "kernels.cuh"
+#include "sparse.cuh"
+
+namespace tmz {
+
+namespace {
+
+constexpr int TPB = 256;
+constexpr uint32_t DENSE_CHUNK = 4096;  // elements per dense block (16 per thread)
+
+__device__ __forceinline__ int find_proj(const uint32_t* prefix, int P, uint32_t b) {
+  int lo = 0, hi = P - 1;  // largest p with prefix[p] <= b
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (prefix[mid] <= b) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+struct DenseRange {
+  int proj;
+  uint64_t start, end;
+};
+
+__device__ __forceinline__ DenseRange dense_range(const MaskArgs& a, uint32_t b) {
+  DenseRange r;
+  r.proj = find_proj(a.dpre, a.P, b);
+  r.start = a.base[r.proj] + (uint64_t)(b - a.dpre[r.proj]) * DENSE_CHUNK;
+  const uint64_t e = r.start + DENSE_CHUNK;
+  r.end = e < a.base[r.proj + 1] ? e : a.base[r.proj + 1];
+  return r;
+}
+
+struct SparseRange {
+  int proj;
+  uint32_t beg, end, seg_beg, seg_end;
+};
+
+__device__ __forceinline__ SparseRange sparse_range(const MaskArgs& a, const uint32_t* off, uint32_t b) {
+  SparseRange r;
+  r.proj = find_proj(a.spre, a.P, b);
+  const uint32_t nb = a.spre[r.proj + 1] - a.spre[r.proj];
+  const uint32_t j = b - a.spre[r.proj];
+  r.seg_beg = off[r.proj];
+  r.seg_end = off[r.proj + 1];
+  const uint32_t len = r.seg_end - r.seg_beg;
+  const uint32_t chunk = (len + nb - 1) / nb;
+  const uint64_t lo = (uint64_t)j * chunk, hi = (uint64_t)(j + 1) * chunk;
+  r.beg = r.seg_beg + (uint32_t)(lo < len ? lo : len);
+  r.end = r.seg_beg + (uint32_t)(hi < len ? hi : len);
+  return r;
+}
+
+__device__ __forceinline__ void load16(const float* w, uint64_t i, float (&v)[16]) {
+  const float4* p = reinterpret_cast<const float4*>(w + i);
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const float4 t = p[q];
+    v[4 * q] = t.x; v[4 * q + 1] = t.y; v[4 * q + 2] = t.z; v[4 * q + 3] = t.w;
+  }
+}
+
+// Exclusive block scan of one uint32 per thread (blockDim.x == TPB).
+__device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* sh, uint32_t* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint32_t x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  __syncthreads();
+  if (lane == 31) sh[warp] = x;
+  __syncthreads();
+  uint32_t wpre = 0, tot = 0;
+  for (int i = 0; i < TPB / 32; ++i) {
+    if (i < warp) wpre += sh[i];
+    tot += sh[i];
+  }
+  if (total) *total = tot;
+  return wpre + x - v;
+}
+
+// ----------------------------------------------------------- dense passes --
+
+__global__ void __launch_bounds__(TPB) k_dense_sum(MaskArgs a, const float* __restrict__ w) {
+  __shared__ ExactSum red[TPB / 32];
+  const DenseRange r = dense_range(a, blockIdx.x);
+  ExactSum s;
+  es_zero(s);
+  const uint64_t i0 = r.start + 16ull * threadIdx.x;
+  if (i0 < r.end) {
+    float v[16];
+    load16(w, i0, v);
+#pragma unroll
+    for (int j = 0; j < 16; ++j) es_add_abs(s, v[j]);
+  }
+  es_block_reduce(s, red);
+  if (threadIdx.x == 0) a.partials[blockIdx.x] = s;
+}
+
+// One block per projection: S = sum of the block partials [lo, hi) (+ add
+// when non-null), then gamma, tau, s_w of the projection.
+__global__ void k_reduce_proj(const ExactSum* __restrict__ parts, const uint32_t* __restrict__ pre, int stride,
+                              int slot, const ExactSum* __restrict__ add, const uint64_t* __restrict__ base,
+                              ExactSum* __restrict__ out_sum, float* gamma, float* tau, float* sw) {
+  __shared__ ExactSum red[TPB / 32];
+  const int p = blockIdx.x;
+  ExactSum s;
+  es_zero(s);
+  for (uint32_t b = pre[p] + threadIdx.x; b < pre[p + 1]; b += blockDim.x) es_merge(s, parts[(size_t)b * stride + slot]);
+  es_block_reduce(s, red);
+  if (threadIdx.x == 0) {
+    if (add) es_merge(s, add[p]);
+    if (out_sum) out_sum[p] = s;
+    if (tau) gamma_tau(s, base[p + 1] - base[p], &gamma[p], &tau[p], &sw[p]);
+  }
+}
+
+__device__ __forceinline__ bool key_filter(uint32_t key, int pass, uint32_t prefix, uint32_t* bin) {
+  if (pass == 0) { *bin = key >> 21; return true; }
+  if (pass == 1) { *bin = (key >> 10) & 0x7FFu; return (key >> 21) == prefix; }
+  *bin = key & 0x3FFu;
+  return (key >> 10) == prefix;
+}
+
+__global__ void __launch_bounds__(TPB) k_hist(MaskArgs a, const float* __restrict__ w, int pass) {
+  __shared__ uint32_t h[2048];
+  for (int i = threadIdx.x; i < 2048; i += TPB) h[i] = 0;
+  __syncthreads();
+  const DenseRange r = dense_range(a, blockIdx.x);
+  const float tau = a.tau_cur[r.proj];
+  const uint32_t prefix = a.sel->prefix;
+  const uint64_t i0 = r.start + 16ull * threadIdx.x;
+  if (i0 < r.end) {
+    float v[16];
+    load16(w, i0, v);
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      uint32_t bin;
+      if (key_filter(__float_as_uint(boundary_distance(v[j], tau)), pass, prefix, &bin)) atomicAdd(&h[bin], 1u);
+    }
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < 2048; i += TPB)
+    if (h[i]) atomicAdd(&a.hist[i], (unsigned long long)h[i]);
+}
+
+// Picks the radix bin that holds the krem-th smallest key (1-based).
+__global__ void k_select(MaskArgs a, int pass) {
+  if (threadIdx.x == 0) {
+    const int bins = pass < 2 ? 2048 : 1024;
+    const int bits = pass < 2 ? 11 : 10;
+    unsigned long long cum = 0, krem = a.sel->krem;
+    int B = bins - 1;
+    for (int i = 0; i < bins; ++i) {
+      if (cum + a.hist[i] >= krem) { B = i; break; }
+      cum += a.hist[i];
+    }
+    a.sel->krem = krem - cum;
+    a.sel->prefix = pass == 0 ? (uint32_t)B : ((a.sel->prefix << bits) | (uint32_t)B);
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < 2048; i += blockDim.x) a.hist[i] = 0;
+}
+
+__global__ void __launch_bounds__(TPB) k_count(MaskArgs a, const float* __restrict__ w) {
+  __shared__ uint32_t sh[TPB / 32];
+  const DenseRange r = dense_range(a, blockIdx.x);
+  const float tau = a.tau_cur[r.proj];
+  const uint32_t key_p = a.sel->prefix;
+  uint32_t less = 0, eq = 0;
+  const uint64_t i0 = r.start + 16ull * threadIdx.x;
+  if (i0 < r.end) {
+    float v[16];
+    load16(w, i0, v);
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const uint32_t key = __float_as_uint(boundary_distance(v[j], tau));
+      less += key < key_p;
+      eq += key == key_p;
+    }
+  }
+  uint32_t tl, te;
+  block_excl_scan(less, sh, &tl);
+  block_excl_scan(eq, sh, &te);
+  if (threadIdx.x == 0) {
+    a.blk_a[blockIdx.x] = tl;
+    a.blk_b[blockIdx.x] = te;
+  }
+}
+
+// Single block: per dense block b, ties before it (blk_d) and selected
+// weights before it (blk_c), selecting the first `krem` ties in index order.
+__device__ __forceinline__ unsigned long long scan1024(unsigned long long v, unsigned long long* sh) {
+  __syncthreads();
+  sh[threadIdx.x] = v;
+  __syncthreads();
+  for (int o = 1; o < 1024; o <<= 1) {
+    const unsigned long long t = threadIdx.x >= (unsigned)o ? sh[threadIdx.x - o] : 0;
+    __syncthreads();
+    sh[threadIdx.x] += t;
+    __syncthreads();
+  }
+  return sh[threadIdx.x] - v;  // exclusive
+}
+
+__global__ void __launch_bounds__(1024) k_scan_dense(MaskArgs a, uint32_t nblk) {
+  __shared__ unsigned long long sh[1024];
+  const unsigned long long ties = a.sel->krem;
+  const uint32_t per = (nblk + 1023) / 1024;
+  const uint32_t b0 = min(nblk, threadIdx.x * per), b1 = min(nblk, b0 + per);
+  unsigned long long eq = 0;
+  for (uint32_t b = b0; b < b1; ++b) eq += a.blk_b[b];
+  const unsigned long long tie_start = scan1024(eq, sh);
+  unsigned long long tie_before = tie_start, sel = 0;
+  for (uint32_t b = b0; b < b1; ++b) {
+    const unsigned long long e = a.blk_b[b];
+    unsigned long long take = tie_before >= ties ? 0 : (ties - tie_before);
+    if (take > e) take = e;
+    sel += a.blk_a[b] + take;
+    tie_before += e;
+  }
+  unsigned long long sel_before = scan1024(sel, sh);
+  tie_before = tie_start;
+  for (uint32_t b = b0; b < b1; ++b) {
+    a.blk_c[b] = (uint32_t)sel_before;
+    a.blk_d[b] = (uint32_t)tie_before;
+    const unsigned long long e = a.blk_b[b];
+    unsigned long long take = tie_before >= ties ? 0 : (ties - tie_before);
+    if (take > e) take = e;
+    sel_before += a.blk_a[b] + take;
+    tie_before += e;
+  }
+}
+
+// Writes S_0 (indices + latents, sorted) and the codes of every weight at tau_0.
+__global__ void __launch_bounds__(TPB) k_compact(MaskArgs a, const float* __restrict__ w) {
+  __shared__ uint32_t sh[TPB / 32];
+  const DenseRange r = dense_range(a, blockIdx.x);
+  const float tau = a.tau_cur[r.proj];
+  const uint32_t key_p = a.sel->prefix;
+  const unsigned long long ties = a.sel->krem;
+  const uint64_t i0 = r.start + 16ull * threadIdx.x;
+  const bool live = i0 < r.end;
+  float v[16];
+  uint32_t keys[16];
+  uint32_t eq = 0, word = 0;
+  if (live) {
+    load16(w, i0, v);
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      keys[j] = __float_as_uint(boundary_distance(v[j], tau));
+      eq += keys[j] == key_p;
+      word |= ternary_code(v[j], tau) << (2 * j);
+    }
+    a.packed[i0 >> 4] = word;
+  }
+  unsigned long long tie_rank = (unsigned long long)a.blk_d[blockIdx.x] + block_excl_scan(eq, sh, nullptr);
+  uint32_t selmask = 0, nsel = 0;
+  if (live) {
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      bool s = keys[j] < key_p;
+      if (keys[j] == key_p) {
+        s = tie_rank < ties;
+        ++tie_rank;
+      }
+      if (s) { selmask |= 1u << j; ++nsel; }
+    }
+  }
+  uint32_t pos = a.blk_c[blockIdx.x] + block_excl_scan(nsel, sh, nullptr);
+  if (live) {
+#pragma unroll
+    for (int j = 0; j < 16; ++j)
+      if (selmask & (1u << j)) {
+        a.idx[0][pos] = (uint32_t)(i0 + j);
+        a.lat[0][pos] = v[j];
+        ++pos;
+      }
+  }
+}
+
+__global__ void k_dense_offsets(MaskArgs a, uint32_t k0) {
+  for (int p = threadIdx.x; p <= a.P; p += blockDim.x) a.off[0][p] = p < a.P ? a.blk_c[a.dpre[p]] : k0;
+}
+
+// ---------------------------------------------------------- sparse passes --
+
+__global__ void __launch_bounds__(TPB) k_sparse_abs(MaskArgs a, int cur) {
+  __shared__ ExactSum red[TPB / 32];
+  const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
+  ExactSum s;
+  es_zero(s);
+  for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) es_add_abs(s, a.lat[cur][e]);
+  es_block_reduce(s, red);
+  if (threadIdx.x == 0) a.partials[blockIdx.x] = s;
+}
+
+// A = S_total - sum over active (bucket-wise; each bucket of the subset sum
+// is at most the bucket of the full sum).
+__global__ void k_frozen_init(MaskArgs a) {
+  __shared__ ExactSum red[TPB / 32];
+  const int p = blockIdx.x;
+  ExactSum s;
+  es_zero(s);
+  for (uint32_t b = a.spre[p] + threadIdx.x; b < a.spre[p + 1]; b += blockDim.x) es_merge(s, a.partials[b]);
+  es_block_reduce(s, red);
+  if (threadIdx.x == 0) {
+    ExactSum f = a.S_total[p];
+    for (int i = 0; i < 4; ++i) f.b[i] -= s.b[i];
+    a.A_frozen[p] = f;
+  }
+}
+
+__device__ __forceinline__ void perturbed(float w, float z, float eps, float* wp, float* wm, float* ee) {
+  *ee = __fmul_rn(eps, z);
+  *wp = __fadd_rn(w, *ee);
+  *wm = __fsub_rn(*wp, __fmul_rn(2.0f, *ee));
+}
+
+__global__ void __launch_bounds__(TPB) k_sparse_pm_sum(MaskArgs a, int cur, uint64_t seed, float eps) {
+  __shared__ ExactSum red[TPB / 32];
+  const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
+  ExactSum sp, sm;
+  es_zero(sp);
+  es_zero(sm);
+  for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) {
+    const float z = normal_at(seed, a.idx[cur][e]);
+    float wp, wm, ee;
+    perturbed(a.lat[cur][e], z, eps, &wp, &wm, &ee);
+    es_add_abs(sp, wp);
+    es_add_abs(sm, wm);
+  }
+  es_block_reduce(sp, red);
+  if (threadIdx.x == 0) a.partials[2 * (size_t)blockIdx.x] = sp;
+  es_block_reduce(sm, red);
+  if (threadIdx.x == 0) a.partials[2 * (size_t)blockIdx.x + 1] = sm;
+}
+
+// Rewrites the codes of the active weights.  sign +1: w + eps z at tau+;
+// sign -1: (w + eps z) - 2 eps z at tau- (and counts codes that differ from
+// the + pass); sign 0: w at tau_cur.  The first active element of each
+// packed word (the "leader") owns the read-modify-write of that word.
+__global__ void __launch_bounds__(TPB) k_sparse_requant(MaskArgs a, int cur, uint64_t seed, float eps, int sign) {
+  __shared__ unsigned long long cnt[3];
+  if (threadIdx.x < 3) cnt[threadIdx.x] = 0;
+  __syncthreads();
+  const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
+  const uint32_t* idx = a.idx[cur];
+  const float* lat = a.lat[cur];
+  const float* tau_sel = sign > 0 ? a.tau_plus : (sign < 0 ? a.tau_minus : a.tau_cur);
+  const float tau = tau_sel[r.proj];
+  const float taup = a.tau_plus[r.proj];
+  uint32_t flips = 0, jumps = 0, words = 0;
+  for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) {
+    const uint32_t i = idx[e];
+    if (e != r.seg_beg && (idx[e - 1] >> 4) == (i >> 4)) continue;  // not the leader
+    const uint32_t wi = i >> 4;
+    ++words;
+    uint32_t word = a.packed[wi];
+    for (uint32_t e2 = e; e2 < r.seg_end; ++e2) {
+      const uint32_t i2 = idx[e2];
+      if ((i2 >> 4) != wi) break;
+      const float w = lat[e2];
+      uint32_t code;
+      if (sign == 0) {
+        code = ternary_code(w, tau);
+      } else {
+        float wp, wm, ee;
+        perturbed(w, normal_at(seed, i2), eps, &wp, &wm, &ee);
+        code = ternary_code(sign > 0 ? wp : wm, tau);
+        if (sign < 0) {
+          const uint32_t cp = ternary_code(wp, taup);
+          flips += cp != code;
+          jumps += (cp ^ code) == 2u;  // 0 <-> 2 in the stored q+1 form
+        }
+      }
+      const uint32_t sh = 2 * (i2 & 15u);
+      word = (word & ~(3u << sh)) | (code << sh);
+    }
+    a.packed[wi] = word;
+  }
+  if (flips) atomicAdd(&cnt[0], (unsigned long long)flips);
+  if (jumps) atomicAdd(&cnt[1], (unsigned long long)jumps);
+  if (words) atomicAdd(&cnt[2], (unsigned long long)words);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    if (cnt[0]) atomicAdd(&a.counters[0], cnt[0]);
+    if (cnt[1]) atomicAdd(&a.counters[1], cnt[1]);
+    if (cnt[2]) atomicAdd(&a.counters[3], cnt[2]);
+  }
+}
+
+// Restore and update: w' = ((w + e) - 2e) + e; w <- w' - fl32(c z) with
+// c = (float)(lr * g); accumulates the exact sum of the new |w|.
+__global__ void __launch_bounds__(TPB) k_sparse_update(MaskArgs a, int cur, uint64_t seed, float eps, float lr,
+                                                       const double* g_dev, double g_host, int use_host) {
+  __shared__ ExactSum red[TPB / 32];
+  const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
+  const double g = use_host ? g_host : *g_dev;
+  const float c = (float)((double)lr * g);
+  ExactSum s;
+  es_zero(s);
+  for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) {
+    const float z = normal_at(seed, a.idx[cur][e]);
+    float wp, wm, ee;
+    perturbed(a.lat[cur][e], z, eps, &wp, &wm, &ee);
+    const float wr = __fadd_rn(wm, ee);
+    const float wn = __fsub_rn(wr, __fmul_rn(c, z));
+    a.lat[cur][e] = wn;
+    es_add_abs(s, wn);
+  }
+  es_block_reduce(s, red);
+  if (threadIdx.x == 0) a.partials[blockIdx.x] = s;
+}
+
+// Eq. 5 at tau_cur: marks dropped weights, writes their code at tau_cur,
+// sums their |w| and counts the kept ones per block.
+__global__ void __launch_bounds__(TPB) k_shrink_mark(MaskArgs a, int cur, float xi0) {
+  __shared__ ExactSum red[TPB / 32];
+  __shared__ uint32_t sh[TPB / 32];
+  const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
+  const uint32_t* idx = a.idx[cur];
+  const float* lat = a.lat[cur];
+  const float tau = a.tau_cur[r.proj];
+  ExactSum s;
+  es_zero(s);
+  uint32_t kept = 0, dropped = 0;
+  for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) {
+    const float w = lat[e];
+    if (boundary_distance(w, tau) <= xi0) {
+      ++kept;
+    } else {
+      ++dropped;
+      es_add_abs(s, w);
+    }
+    const uint32_t i = idx[e];
+    if (e != r.seg_beg && (idx[e - 1] >> 4) == (i >> 4)) continue;
+    const uint32_t wi = i >> 4;
+    uint32_t word = a.packed[wi];
+    bool touched = false;
+    for (uint32_t e2 = e; e2 < r.seg_end; ++e2) {
+      const uint32_t i2 = idx[e2];
+      if ((i2 >> 4) != wi) break;
+      const float w2 = lat[e2];
+      if (boundary_distance(w2, tau) > xi0) {
+        const uint32_t shf = 2 * (i2 & 15u);
+        word = (word & ~(3u << shf)) | (ternary_code(w2, tau) << shf);
+        touched = true;
+      }
+    }
+    if (touched) a.packed[wi] = word;
+  }
+  es_block_reduce(s, red);
+  if (threadIdx.x == 0) a.partials[blockIdx.x] = s;
+  uint32_t tk, td;
+  block_excl_scan(kept, sh, &tk);
+  block_excl_scan(dropped, sh, &td);
+  if (threadIdx.x == 0) {
+    a.blk_a[blockIdx.x] = tk;
+    if (td) atomicAdd(&a.counters[2], (unsigned long long)td);
+  }
+}
+
+__global__ void k_frozen_add(MaskArgs a) {
+  __shared__ ExactSum red[TPB / 32];
+  const int p = blockIdx.x;
+  ExactSum s;
+  es_zero(s);
+  for (uint32_t b = a.spre[p] + threadIdx.x; b < a.spre[p + 1]; b += blockDim.x) es_merge(s, a.partials[b]);
+  es_block_reduce(s, red);
+  if (threadIdx.x == 0) es_merge(a.A_frozen[p], s);
+}
+
+// Single block exclusive scan of blk_a[0..n) into blk_c; total into *total.
+__global__ void __launch_bounds__(1024) k_scan_simple(MaskArgs a, uint32_t n, uint32_t* total) {
+  __shared__ unsigned long long sh[1024];
+  const uint32_t per = (n + 1023) / 1024;
+  const uint32_t b0 = min(n, threadIdx.x * per), b1 = min(n, b0 + per);
+  unsigned long long s = 0;
+  for (uint32_t b = b0; b < b1; ++b) s += a.blk_a[b];
+  unsigned long long run = scan1024(s, sh);
+  if (threadIdx.x == 1023) *total = (uint32_t)(run + s);
+  for (uint32_t b = b0; b < b1; ++b) {
+    a.blk_c[b] = (uint32_t)run;
+    run += a.blk_a[b];
+  }
+}
+
+__global__ void __launch_bounds__(TPB) k_shrink_scatter(MaskArgs a, int cur, float xi0) {
+  __shared__ uint32_t sh[TPB / 32];
+  const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
+  const float tau = a.tau_cur[r.proj];
+  uint32_t pos = a.blk_c[blockIdx.x];
+  for (uint32_t base = r.beg; base < r.end; base += TPB) {
+    const uint32_t e = base + threadIdx.x;
+    bool keep = false;
+    float w = 0.f;
+    uint32_t i = 0;
+    if (e < r.end) {
+      w = a.lat[cur][e];
+      i = a.idx[cur][e];
+      keep = boundary_distance(w, tau) <= xi0;
+    }
+    uint32_t tot;
+    const uint32_t rank = block_excl_scan(keep ? 1u : 0u, sh, &tot);
+    if (keep) {
+      a.idx[cur ^ 1][pos + rank] = i;
+      a.lat[cur ^ 1][pos + rank] = w;
+    }
+    pos += tot;
+  }
+}
+
+__global__ void k_sparse_offsets(MaskArgs a, int out, const uint32_t* total) {
+  for (int p = threadIdx.x; p <= a.P; p += blockDim.x) a.off[out][p] = p < a.P ? a.blk_c[a.spre[p]] : *total;
+}
+
+__global__ void k_grad(const double* loss, float eps, double* g) {
+  if (threadIdx.x == 0) *g = (loss[0] - loss[1]) / (2.0 * (double)eps);
+}
+
+__global__ void k_normal(uint64_t seed, const uint32_t* idx, uint64_t n, float* z) {
+  const uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) z[i] = normal_at(seed, idx[i]);
+}
+
+}  // namespace
+
+// ----------------------------------------------------------- host side ----
+
+void mask_build(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_t s) {
+  kernel_launches() += 12;
+  k_dense_sum<<<a.NBD, TPB, 0, s>>>(a, w);
+  k_reduce_proj<<<a.P, TPB, 0, s>>>(a.partials, a.dpre, 1, 0, nullptr, a.base, a.S_total, a.gamma_cur, a.tau_cur,
+                                    a.sw_cur);
+  for (int pass = 0; pass < 3; ++pass) {
+    k_hist<<<a.NBD, TPB, 0, s>>>(a, w, pass);
+    k_select<<<1, 256, 0, s>>>(a, pass);
+  }
+  k_count<<<a.NBD, TPB, 0, s>>>(a, w);
+  k_scan_dense<<<1, 1024, 0, s>>>(a, a.NBD);
+  k_compact<<<a.NBD, TPB, 0, s>>>(a, w);
+  k_dense_offsets<<<1, 256, 0, s>>>(a, (uint32_t)k0);
+}
+
+void mask_finish(const MaskArgs& a, cudaStream_t s) {
+  kernel_launches() += 2;
+  k_sparse_abs<<<a.NBS, TPB, 0, s>>>(a, 0);
+  k_frozen_init<<<a.P, TPB, 0, s>>>(a);
+}
+
+void sparse_pm_taus(const MaskArgs& a, int cur, uint64_t seed, float eps, cudaStream_t s) {
+  kernel_launches() += 3;
+  k_sparse_pm_sum<<<a.NBS, TPB, 0, s>>>(a, cur, seed, eps);
+  k_reduce_proj<<<a.P, TPB, 0, s>>>(a.partials, a.spre, 2, 0, a.A_frozen, a.base, nullptr, a.gamma_plus, a.tau_plus,
+                                    a.sw_plus);
+  k_reduce_proj<<<a.P, TPB, 0, s>>>(a.partials, a.spre, 2, 1, a.A_frozen, a.base, nullptr, a.gamma_minus,
+                                    a.tau_minus, a.sw_minus);
+}
+
+void sparse_requant(const MaskArgs& a, int cur, uint64_t seed, float eps, int sign, cudaStream_t s) {
+  kernel_launches() += 1;
+  k_sparse_requant<<<a.NBS, TPB, 0, s>>>(a, cur, seed, eps, sign);
+}
+
+void sparse_update(const MaskArgs& a, int cur, uint64_t seed, float eps, float lr, const double* g_dev, double g_host,
+                   int use_host, cudaStream_t s) {
+  kernel_launches() += 2;
+  k_sparse_update<<<a.NBS, TPB, 0, s>>>(a, cur, seed, eps, lr, g_dev, g_host, use_host);
+  k_reduce_proj<<<a.P, TPB, 0, s>>>(a.partials, a.spre, 1, 0, a.A_frozen, a.base, nullptr, a.gamma_cur, a.tau_cur,
+                                    a.sw_cur);
+}
+
+void sparse_shrink(const MaskArgs& a, int cur, float xi0, uint32_t* d_total, cudaStream_t s) {
+  kernel_launches() += 5;
+  k_shrink_mark<<<a.NBS, TPB, 0, s>>>(a, cur, xi0);
+  k_frozen_add<<<a.P, TPB, 0, s>>>(a);
+  k_scan_simple<<<1, 1024, 0, s>>>(a, a.NBS, d_total);
+  k_shrink_scatter<<<a.NBS, TPB, 0, s>>>(a, cur, xi0);
+  k_sparse_offsets<<<1, 256, 0, s>>>(a, cur ^ 1, d_total);
+}
+
+void launch_grad(const double* loss, float eps, double* g, cudaStream_t s) {
+  kernel_launches() += 1; k_grad<<<1, 32, 0, s>>>(loss, eps, g); }
+
+void launch_normal(uint64_t seed, const uint32_t* idx, uint64_t n, float* z, cudaStream_t s) {
+  if (n) ++kernel_launches();
+  if (n) k_normal<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(seed, idx, n, z);
+}
+
+}  // namespace tmz

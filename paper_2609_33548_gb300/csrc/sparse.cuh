@@ -1,0 +1,53 @@
+// Device state of the mask and of the sparse latent store (host side view).
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "common.cuh"
+
+namespace tmz {
+
+struct SelectState {
+  unsigned long long krem;  // rank still to find (1-based); after the last pass: ties to take
+  uint32_t prefix;          // radix prefix found so far; after the last pass: the key of xi_0
+  uint32_t pad;
+};
+
+// Everything the mask / sparse kernels touch.  Passed by value to kernels.
+struct MaskArgs {
+  int P;                        // projections
+  const uint64_t* base;         // [P+1] first global index of each projection
+  const uint32_t* dpre;         // [P+1] dense-block prefix (4096 elements per block)
+  uint32_t NBD;                 // dense blocks
+  const uint32_t* spre;         // [P+1] sparse-block prefix
+  uint32_t NBS;                 // sparse blocks
+  uint32_t* packed;             // [d/16] 2-bit codes
+  uint32_t* idx[2];             // active global indices (double buffer)
+  float* lat[2];                // active latents
+  uint32_t* off[2];             // [P+1] segment offsets into idx/lat
+  ExactSum* S_total;            // [P] exact sum of |w_0|
+  ExactSum* A_frozen;           // [P] exact sum of |w| over frozen weights
+  ExactSum* partials;           // per-block partial sums
+  float *gamma_cur, *tau_cur, *sw_cur;       // [P+2] of the current latents
+  float *gamma_plus, *tau_plus, *sw_plus;    // [P+2] of w + eps z
+  float *gamma_minus, *tau_minus, *sw_minus; // [P+2] of w - eps z
+  unsigned long long* hist;     // [2048]
+  SelectState* sel;
+  uint32_t *blk_a, *blk_b, *blk_c, *blk_d;   // per-block scratch
+  unsigned long long* counters; // [0] flipped, [1] jumps, [2] dropped, [3] packed words rewritten
+  unsigned* err;
+};
+
+void mask_build(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_t s);
+void mask_finish(const MaskArgs& a, cudaStream_t s);
+void sparse_pm_taus(const MaskArgs& a, int cur, uint64_t seed, float eps, cudaStream_t s);
+void sparse_requant(const MaskArgs& a, int cur, uint64_t seed, float eps, int sign, cudaStream_t s);
+void sparse_update(const MaskArgs& a, int cur, uint64_t seed, float eps, float lr, const double* g_dev,
+                   double g_host, int use_host, cudaStream_t s);
+void sparse_shrink(const MaskArgs& a, int cur, float xi0, uint32_t* d_total, cudaStream_t s);
+void launch_grad(const double* loss, float eps, double* g, cudaStream_t s);
+void launch_normal(uint64_t seed, const uint32_t* idx, uint64_t n, float* z, cudaStream_t s);
+
+}  // namespace tmz

@@ -1,0 +1,124 @@
+"""GPU parity of the single-projection ("BitLinear op") workload against the
+oracle: z generation, exact absmean and mask selection (Eqs. 2-4),
+perturb/requantise (Alg. 1), restore/update, and the int8 x ternary GEMM.
+Calls go through the C ABI."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import bitnet, philox, ternary, termezo as otz
+from paper_2609_33548_gb300 import synth
+from paper_2609_33548_gb300 import termezo as tz
+
+from helpers import ulp_diff
+
+pytestmark = pytest.mark.gpu
+
+N, K, M = synth.BITLINEAR_OP["N"], synth.BITLINEAR_OP["K"], synth.BITLINEAR_OP["M"]
+
+
+@pytest.fixture(scope="module")
+def op_latents():
+    return synth.op_latents(N, K).numpy().reshape(-1)
+
+
+def _ctx(w, density, n=N, k=K, m=M):
+    ctx = tz.Context(tz.op_cfg(n, k, m), density)
+    wd = torch.from_numpy(w).cuda()
+    ctx.termezo_load_params(wd)
+    return ctx, wd
+
+
+def test_normal_matches_oracle():
+    rng = np.random.default_rng(0)
+    idx = np.concatenate([np.arange(4096), rng.integers(0, 2**32 - 1, 100000, dtype=np.uint64)]).astype(np.uint32)
+    for seed in (0, 1001, 2**40 + 7):
+        z_gpu = torch.empty(idx.size, dtype=torch.float32, device="cuda")
+        tz.termezo_normal(seed, torch.from_numpy(idx.astype(np.int32)).cuda(), z_gpu)
+        z = z_gpu.cpu().numpy()
+        zo = philox.normal(seed, idx.astype(np.uint64))
+        err = np.abs(z.astype(np.float64) - zo)
+        assert np.all(err <= 4e-7 * np.maximum(1.0, np.abs(zo)) + 1e-7), err.max()
+        assert np.median(ulp_diff(z, zo)) <= 1
+
+
+@pytest.mark.parametrize("density", synth.BITLINEAR_OP["densities"])
+def test_mask_build_bit_exact(op_latents, density):
+    w = op_latents
+    ctx, _ = _ctx(w, density)
+    k0, xi0 = ctx.termezo_build_mask(density)
+    st = ctx.termezo_export_state()
+    reg = otz.single_registry(N, K)
+    sel, xi0_o, k0_o, tau_o = otz.initial_mask(w, reg, density)
+    assert k0 == k0_o == int(np.floor(density * N * K))
+    assert np.float32(xi0).view(np.uint32) == np.float32(xi0_o).view(np.uint32)
+    assert st["tau_cur"][0].view(np.uint32) == tau_o[0].view(np.uint32)
+    np.testing.assert_array_equal(st["idx"], sel.astype(np.uint32))
+    np.testing.assert_array_equal(st["latents"], w[sel])
+    np.testing.assert_array_equal(st["packed"], ternary.pack_codes(ternary.quantize(w, tau_o[0])))
+
+
+def test_perturb_requantize_update(op_latents):
+    density, seed, eps, lr, g = 0.01, 1000, np.float32(1e-3), np.float32(1e-3), -5.25
+    w = op_latents
+    ctx, _ = _ctx(w, density)
+    ctx.termezo_build_mask(density)
+    reg = otz.single_registry(N, K)
+    state = otz.build(w, reg, density)
+    act = state.active
+    z = philox.normal(seed, act)
+    e = (eps * z).astype(np.float32)
+
+    def check(sign, wp):
+        st = ctx.termezo_export_state()
+        codes, tau, sw = otz.requantize(wp, reg)
+        key = "tau_plus" if sign > 0 else "tau_minus"
+        assert ulp_diff(st[key][:1], tau[:1])[0] <= 1
+        got = ternary.unpack_codes(st["packed"])
+        near = otz.near_threshold(wp[act], tau[np.zeros(act.size, int)], sw[np.zeros(act.size, int)])
+        bad = np.nonzero(got != codes)[0]
+        frozen_bad = np.setdiff1d(bad, act)
+        assert frozen_bad.size == 0
+        act_bad = np.isin(act, bad)
+        assert np.all(near[act_bad]), (act_bad.sum(), near.sum())
+        return near.sum()
+
+    ctx.termezo_requantize(seed, float(eps), +1)
+    w_plus = w.copy()
+    w_plus[act] = (w[act] + e).astype(np.float32)
+    check(+1, w_plus)
+    ctx.termezo_requantize(seed, float(eps), -1)
+    w_minus = w_plus.copy()
+    w_minus[act] = (w_plus[act] - np.float32(2) * e).astype(np.float32)
+    check(-1, w_minus)
+    ctx.termezo_update(seed, float(eps), float(lr), g)
+    st = ctx.termezo_export_state(packed=False)
+    w_rest = (w_minus[act] + e).astype(np.float32)
+    c = np.float32(float(lr) * g)
+    expect = (w_rest - (c * z).astype(np.float32)).astype(np.float32)
+    np.testing.assert_array_equal(st["idx"], act.astype(np.uint32))
+    # z agrees to a few ulp; the restore ((w+e)-2e)+e rounds at the scale of
+    # |w| + 2|e|, so the tolerance is relative to that scale
+    tol = 1e-5 * (np.abs(expect).astype(np.float64) + 2 * np.abs(e))
+    assert np.all(np.abs(st["latents"].astype(np.float64) - expect) <= tol)
+
+
+@pytest.mark.parametrize("shape", [(N, K, M), (688, 688, 200), (256, 2560, 130)])
+def test_bitlinear_int32_accumulators_bit_exact(shape):
+    n, k, m = shape
+    w = synth.op_latents(n, k, seed=11).numpy().reshape(-1)
+    ctx, _ = _ctx(w, 0.01, n, k, max(m, 128))
+    ctx.termezo_build_mask(0.01)
+    x = synth.op_activations(m, k, seed=12)
+    acc = torch.zeros(m, n, dtype=torch.int32, device="cuda")
+    y = torch.zeros(m, n, dtype=torch.float32, device="cuda")
+    ctx.termezo_bitlinear(0, x.cuda(), acc, y)
+    torch.cuda.synchronize()
+    reg = otz.single_registry(n, k)
+    _, tau, sw = otz.thresholds(w, reg)
+    codes = ternary.quantize(w, tau[0]).reshape(n, k)
+    q, a = bitnet.act_quant(x.float().numpy())
+    acc_o = bitnet.int_matmul(q, codes)
+    np.testing.assert_array_equal(acc.cpu().numpy(), acc_o)
+    y_o = acc_o.astype(np.float64) * (a.astype(np.float64)[:, None] / 127.0) * float(sw[0])
+    np.testing.assert_allclose(y.cpu().numpy(), y_o, rtol=2e-6, atol=1e-30)

@@ -1,0 +1,153 @@
+"""Whole-step GPU parity on the tiny BitNet workload (2 layers, d 256,
+seq 64, batch 4, density 1%, eps 1e-3, lr 1e-6) against the dense oracle on
+the same seeded inputs.  Calls go through the C ABI.
+
+Tolerances:
+* F+ and F-: 1e-3 relative (the stated bound).
+* g = (F+ - F-) / (2 eps): the quantised forward turns 1-ulp differences of
+  fp32 intermediates into int8 / bf16 code flips, so two valid fp32
+  evaluation orders disagree on g by about 1%.  The oracle is therefore
+  evaluated under several alternative valid roundings (each BitLinear
+  output moved by at most one ulp) and the GPU's g must lie inside that
+  ensemble's range widened by its spread; it must also agree within 1e-3
+  when that spread happens to be smaller.
+* latents: |dw| <= 1e-5 (|w| + 2 eps |z|) + lr |dg| |z| (the restore
+  ((w+e)-2e)+e rounds at the scale of |w| + 2|e|, and a g difference moves
+  the update by lr dg z).
+* codes: bit-exact except active latents within 1e-5 s_w of a threshold.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import bitnet, philox, rounding, ternary, termezo as otz
+from paper_2609_33548_gb300 import synth
+from paper_2609_33548_gb300 import termezo as tz
+
+from helpers import rel_err
+
+pytestmark = pytest.mark.gpu
+
+CFG = synth.TINY
+DENSITY, EPS, LR = 0.01, 1e-3, 1e-6
+
+
+@pytest.fixture(scope="module")
+def inputs():
+    w = synth.latents(CFG)
+    emb, gains, head = synth.theta(CFG)
+    tok, tgt = synth.batch(CFG)
+    return w, emb, gains, head, tok, tgt
+
+
+def _gpu_ctx(inputs):
+    w, emb, gains, head, tok, tgt = inputs
+    ctx = tz.Context(tz.make_cfg(CFG), DENSITY)
+    dev = [t.cuda() for t in (w, emb, gains, head, tok, tgt)]
+    ctx.termezo_load_params(dev[0], dev[1], dev[2], dev[3])
+    return ctx, dev
+
+
+def _theta_np(inputs):
+    return (inputs[1].numpy(), inputs[2].numpy(), inputs[3].float().numpy(), inputs[4].numpy(),
+            inputs[5].numpy())
+
+
+def _split(codes, reg):
+    return [codes[p.base:p.base + p.n].reshape(p.N, p.K) for p in reg]
+
+
+def test_forward_loss_matches_oracle(inputs):
+    ctx, dev = _gpu_ctx(inputs)
+    ctx.termezo_build_mask(DENSITY)
+    loss, per = ctx.termezo_forward_loss(dev[4], dev[5])
+    loss2, per2 = ctx.termezo_forward_loss(dev[4], dev[5])
+    assert loss == loss2 and np.array_equal(per, per2)          # deterministic
+    reg = otz.registry(CFG)
+    codes, tau, sw = otz.requantize(inputs[0].numpy(), reg)
+    per_o, mean_o = bitnet.batch_loss(CFG, _split(codes, reg), sw, *_theta_np(inputs))
+    assert rel_err(loss, mean_o) < 1e-3
+    np.testing.assert_allclose(per, per_o, rtol=3e-3)
+
+
+def test_one_step_matches_oracle(inputs):
+    ctx, dev = _gpu_ctx(inputs)
+    k0, xi0 = ctx.termezo_build_mask(DENSITY)
+    reg = otz.registry(CFG)
+    state = otz.build(inputs[0].numpy(), reg, DENSITY)
+    fn = otz.bitnet_loss_fn(CFG, *_theta_np(inputs))
+    assert k0 == state.k0 and np.float32(xi0) == state.xi0
+    w_before = state.w.copy()
+    act = state.active.copy()
+    seed = synth.step_seed(0)
+    out = ctx.termezo_step(seed, EPS, LR, DENSITY, dev[4], dev[5])
+    rec = otz.step(state, fn, seed, EPS, LR)
+    assert rel_err(out["loss_plus"], rec["loss_plus"]) < 1e-3
+    assert rel_err(out["loss_minus"], rec["loss_minus"]) < 1e-3
+    # g against the ensemble of valid roundings
+    z = philox.normal(seed, act)
+    e = (np.float32(EPS) * z).astype(np.float32)
+    wp = w_before.copy(); wp[act] = (w_before[act] + e).astype(np.float32)
+    wm = wp.copy(); wm[act] = (wp[act] - np.float32(2) * e).astype(np.float32)
+    cp, _, swp = otz.requantize(wp, reg)
+    cm, _, swm = otz.requantize(wm, reg)
+    ens = rounding.g_ensemble(CFG, (_split(cp, reg), swp), (_split(cm, reg), swm), _theta_np(inputs), EPS)
+    assert rounding.g_within_ensemble(out["g"], rec["g"], ens), (out["g"], rec["g"], ens)
+    # counters
+    assert out["k_active"] == rec["k"] == act.size
+    assert out["n_jumps"] == rec["n_jumps"]
+    n_near = int(rec["near_plus"].sum() + rec["near_minus"].sum())
+    assert abs(int(out["n_flipped"]) - rec["n_flipped"]) <= n_near
+    # state after the update
+    st = ctx.termezo_export_state()
+    np.testing.assert_array_equal(st["idx"], act.astype(np.uint32))
+    dg = abs(out["g"] - rec["g"])
+    tol = 1e-5 * (np.abs(w_before[act]) + 2 * np.abs(e)) + float(np.float32(LR)) * dg * np.abs(z) * 1.01
+    assert np.all(np.abs(st["latents"].astype(np.float64) - state.w[act]) <= tol)
+    got = ternary.unpack_codes(st["packed"])
+    bad = np.nonzero(got != rec["codes_minus"])[0]
+    assert rec["frozen_mismatch"] == 0
+    assert np.all(np.isin(bad, act[rec["near_minus"]]))
+    np.testing.assert_array_equal(st["tau_minus"].view(np.uint32), rec["tau_minus"].view(np.uint32))
+    np.testing.assert_array_equal(st["tau_plus"].view(np.uint32), rec["tau_plus"].view(np.uint32))
+
+
+def test_mask_and_update_replay_many_steps(inputs):
+    """Mask shrink, perturb and update over 30 iterations with a given g
+    sequence (the oracle's g is fed to both sides), large enough that the
+    active set shrinks: indices bit-exact, latents within the rounding of
+    the restore arithmetic."""
+    w0 = inputs[0].numpy()
+    reg = otz.registry(CFG)
+    ctx, dev = _gpu_ctx(inputs)
+    ctx.termezo_build_mask(DENSITY)
+    state = otz.build(w0, reg, DENSITY)
+    eps, lr = np.float32(EPS), np.float32(2e-3)
+    rng = np.random.default_rng(5)
+    sizes = []
+    for t in range(30):
+        g = float(rng.standard_normal() * 20.0)
+        seed = synth.step_seed(t)
+        if t:
+            ctx.termezo_shrink()
+            kept, tau_t = otz.shrink(state.w, reg, state.active, state.xi0)
+            state.active = kept
+        act = state.active
+        ctx.termezo_requantize(seed, float(eps), +1)
+        ctx.termezo_requantize(seed, float(eps), -1)
+        ctx.termezo_update(seed, float(eps), float(lr), g)
+        z = philox.normal(seed, act)
+        w_next, *_ = otz.masked_spsa(state.w, act, z, eps, 0.0, lambda v: 0.0)
+        c = np.float32(float(lr) * g)
+        state.w = w_next
+        state.w[act] = (state.w[act] - (c * z).astype(np.float32)).astype(np.float32)
+        st = ctx.termezo_export_state(packed=False)
+        np.testing.assert_array_equal(st["idx"], act.astype(np.uint32))
+        # z agrees to a few ulp, so the latents agree to the rounding of the
+        # restore arithmetic, accumulated over the iterations so far
+        e = np.abs(eps * z)
+        tol = (t + 1) * 1e-5 * (np.abs(state.w[act]) + 2 * e)
+        assert np.all(np.abs(st["latents"].astype(np.float64) - state.w[act]) <= tol)
+        sizes.append(act.size)
+    assert sizes[-1] < sizes[0]
+    assert all(a >= b for a, b in zip(sizes, sizes[1:]))
