@@ -156,6 +156,26 @@ int termezo_export_state(termezo_ctx* ctx, uint32_t* h_idx, float* h_latents, ui
  * to d_z fp32 [n].  Stateless; ordered on `stream`. */
 int termezo_normal(uint64_t seed, const uint32_t* d_idx, uint64_t n, float* d_z, void* stream);
 
+/* Allocation-free absmean.  The paper has no counterpart: this is an
+ * interface for callers that cannot allocate device memory -- code inside a
+ * host framework that owns all of the GPU's memory (a serving engine that
+ * reserves it up front, or one that forbids cudaMalloc on its hot path
+ * because it synchronises the device) and so cannot pass a workspace to
+ * termezo_create.
+ * Computes, for one fp32 latent tensor d_w[n] (device), the exact
+ * gamma = mean |w| (Sec. 3, same arithmetic as termezo_build_mask),
+ * tau = 0.5 (gamma + 1e-5) and s_w = gamma + 1e-5, written to the device
+ * floats d_out[0], d_out[1], d_out[2], ordered on `stream`.
+ * Scratch: a fixed array of TERMEZO_NOALLOC_MAX_ELEMS / 4096 partial sums
+ * (4 MiB) inside the library; every GPU that loads the library holds it
+ * until the process exits.  n > TERMEZO_NOALLOC_MAX_ELEMS returns
+ * TERMEZO_EINVAL (with a message on stderr).  The first call on a device
+ * looks up that device's address of the array; make it before any stream
+ * capture.  Calls share the array: calls that overlap on the GPU race.
+ * Each call overwrites every partial sum it reads.  Allocates nothing. */
+#define TERMEZO_NOALLOC_MAX_ELEMS (1ull << 28)
+int termezo_absmean_noalloc(const float* d_w, uint64_t n, float* d_out, void* stream);
+
 /* Kernel timing of a context.  enable = 1 resets the totals and starts
  * recording CUDA events (on the context's stream) around every BitLinear
  * GEMM, attention and sparse-pass launch; enable = 0 stops recording;

@@ -22,7 +22,7 @@ EXPORTS = (
     "termezo_workspace_bytes", "termezo_create", "termezo_load_params", "termezo_build_mask",
     "termezo_forward_loss", "termezo_step", "termezo_shrink", "termezo_requantize", "termezo_update",
     "termezo_bitlinear", "termezo_state_sizes", "termezo_export_state", "termezo_normal",
-    "termezo_profile", "termezo_destroy", "termezo_strerror",
+    "termezo_absmean_noalloc", "termezo_profile", "termezo_destroy", "termezo_strerror",
 )
 
 
@@ -92,6 +92,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         "termezo_state_sizes": (I32, [P, ctypes.POINTER(U64), ctypes.POINTER(U64), ctypes.POINTER(I32)]),
         "termezo_export_state": (I32, [P, P, P, P, P]),
         "termezo_normal": (I32, [U64, P, U64, P, P]),
+        "termezo_absmean_noalloc": (I32, [P, U64, P, P]),
         "termezo_profile": (I32, [P, I32, ctypes.POINTER(ProfileOut)]),
         "termezo_destroy": (None, [P]),
         "termezo_strerror": (ctypes.c_char_p, [I32]),
@@ -242,3 +243,11 @@ class Context:
 def termezo_normal(seed: int, idx_u32, z_out, stream=None):
     _check("termezo_normal", load().termezo_normal(seed, _ptr(idx_u32), idx_u32.numel(), _ptr(z_out),
                                                    _stream(stream)))
+
+
+def termezo_absmean_noalloc(w, out, stream=None):
+    """gamma, tau, s_w of the fp32 device tensor w into the 3-float device
+    tensor out, without any device allocation (for callers that cannot
+    allocate: the library's fixed scratch array is used)."""
+    _check("termezo_absmean_noalloc", load().termezo_absmean_noalloc(_ptr(w), w.numel(), _ptr(out),
+                                                                     _stream(stream)))
