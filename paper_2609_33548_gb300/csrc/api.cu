@@ -160,7 +160,8 @@ size_t xq_cols(const Shape& s) {
 size_t wexp_elems(const Shape& s) {
   size_t m = 0;
   if (s.op) return (size_t)s.N[0] * s.K[0];
-  const size_t qkv = (size_t)(s.H + 2 * s.KV) * s.hd * s.D, o = (size_t)s.D * s.H * s.hd, gu = (size_t)2 * s.F * s.D,
+  const size_t qkv = (size_t)(s.H + 2 * s.KV) * s.hd * s.D, o = (size_t)s.D * s.H * s.hd,
+               gu = (size_t)256 * ((s.F + 127) / 128) * s.D,
                dn = (size_t)s.D * s.F;
   m = qkv;
   if (o > m) m = o;
@@ -336,18 +337,21 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
     }
     // MLP block
     tmz::launch_norm_quant(c->x, c->gains + (size_t)(2 * l + 1) * D, T, D, c->xq, c->deq, st);
-    tmz::launch_expand_codes(c->ma.packed + s.base[pg] / 16, (uint64_t)(2 * F), D, c->wexp, st);
-    a.out = c->gu;
-    a.ldo = 2 * F;
+    tmz::launch_expand_gate_up(c->ma.packed + s.base[pg] / 16, c->ma.packed + s.base[pg + 1] / 16, F, D, c->wexp,
+                               st);
+    a.out = c->gu;  // hid = relu(gate)^2 * up, fp32 [T, F]
+    a.ldo = F;
     a.mode = 0;
     a.sw = sw + pg;
-    a.n1 = F;
-    a.n2 = 2 * F;
+    a.n1 = a.n2 = a.N;
+    a.relu2 = 1;
+    a.n_out = F;
     {
-      ProfScope ps(c, 0, gemm_flops(c->plan_gu));
+      ProfScope ps(c, 0, 2.0 * T * (2.0 * F) * D);
       if (tmz::gemm_launch(c->plan_gu, a, st) != cudaSuccess) return TERMEZO_ECUDA;
     }
-    tmz::launch_relu2_quant(c->gu, T, F, c->xq, c->deq, st);
+    a.relu2 = 0;
+    tmz::launch_norm_quant(c->gu, nullptr, T, F, c->xq, c->deq, st);
     tmz::launch_expand_codes(c->ma.packed + s.base[pd] / 16, (uint64_t)D, F, c->wexp, st);
     a.out = c->x;
     a.ldo = D;
@@ -431,7 +435,7 @@ int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspa
     const int T = s.T, D = s.D, F = s.F, hq = s.H * s.hd, hkv = s.KV * s.hd;
     bool ok = tmz::gemm_make_plan(&c->plan_qkv, c->xq, T, D, c->wexp, hq + 2 * hkv) &&
               tmz::gemm_make_plan(&c->plan_o, c->xq, T, hq, c->wexp, D) &&
-              tmz::gemm_make_plan(&c->plan_gu, c->xq, T, D, c->wexp, 2 * F) &&
+              tmz::gemm_make_plan(&c->plan_gu, c->xq, T, D, c->wexp, 256 * ((F + 127) / 128)) &&
               tmz::gemm_make_plan(&c->plan_down, c->xq, T, F, c->wexp, D);
     if (!ok) {
       delete c;

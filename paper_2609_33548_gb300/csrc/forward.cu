@@ -48,6 +48,7 @@ __device__ __forceinline__ float quant_code(float h, float s) {
 
 // One block per row.  h_k = (x_k * r) * g_k with r = 1/sqrt(mean(x^2)+1e-5)
 // (RMSNorm) or h_k = x_k; a = max(max|h|, 1e-5); q_k = rint(h_k * (127/a)).
+// Generic version (any D, any input type): three passes over the row.
 template <typename In>
 __global__ void k_norm_quant(const In* __restrict__ x, const float* __restrict__ gain, int D,
                              uint16_t* __restrict__ q, float* __restrict__ deq) {
@@ -81,32 +82,69 @@ __global__ void k_norm_quant(const In* __restrict__ x, const float* __restrict__
   if (threadIdx.x == 0) deq[row] = __fdiv_rn(a, 127.f);
 }
 
+// Same arithmetic for fp32 rows with D % 4 == 0 and D <= 4 * 256 * VPT: the
+// row is read once (float4) and kept in registers.
+template <int VPT>
+__global__ void __launch_bounds__(256) k_norm_quant_vec(const float* __restrict__ x, const float* __restrict__ gain,
+                                                        int D, uint16_t* __restrict__ q, float* __restrict__ deq) {
+  __shared__ float red[32];
+  const size_t row = blockIdx.x;
+  const float4* xr = reinterpret_cast<const float4*>(x + row * (size_t)D);
+  const float4* gr = reinterpret_cast<const float4*>(gain);
+  const int D4 = D >> 2;
+  float4 v[VPT];
+#pragma unroll
+  for (int i = 0; i < VPT; ++i) {
+    const int k = i * 256 + threadIdx.x;
+    v[i] = k < D4 ? xr[k] : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  float r = 1.f;
+  if (gain) {
+    float ss = 0.f;
+#pragma unroll
+    for (int i = 0; i < VPT; ++i) {
+      ss = __fadd_rn(ss, __fmul_rn(v[i].x, v[i].x));
+      ss = __fadd_rn(ss, __fmul_rn(v[i].y, v[i].y));
+      ss = __fadd_rn(ss, __fmul_rn(v[i].z, v[i].z));
+      ss = __fadd_rn(ss, __fmul_rn(v[i].w, v[i].w));
+    }
+    ss = block_sum(ss, red);
+    r = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(__fdiv_rn(ss, (float)D), 1e-5f)));
+#pragma unroll
+    for (int i = 0; i < VPT; ++i) {
+      const int k = i * 256 + threadIdx.x;
+      if (k < D4) {
+        const float4 g = gr[k];
+        v[i].x = __fmul_rn(__fmul_rn(v[i].x, r), g.x);
+        v[i].y = __fmul_rn(__fmul_rn(v[i].y, r), g.y);
+        v[i].z = __fmul_rn(__fmul_rn(v[i].z, r), g.z);
+        v[i].w = __fmul_rn(__fmul_rn(v[i].w, r), g.w);
+      }
+    }
+  }
+  float amax = 0.f;
+#pragma unroll
+  for (int i = 0; i < VPT; ++i)
+    amax = fmaxf(fmaxf(fmaxf(amax, fabsf(v[i].x)), fmaxf(fabsf(v[i].y), fabsf(v[i].z))), fabsf(v[i].w));
+  const float a = fmaxf(block_max(amax, red), 1e-5f);
+  const float s = __fdiv_rn(127.f, a);
+  uint2* qr = reinterpret_cast<uint2*>(q + row * (size_t)D);
+#pragma unroll
+  for (int i = 0; i < VPT; ++i) {
+    const int k = i * 256 + threadIdx.x;
+    if (k < D4) {
+      const uint32_t b0 = int_to_bf16_bits(quant_code(v[i].x, s)), b1 = int_to_bf16_bits(quant_code(v[i].y, s));
+      const uint32_t b2 = int_to_bf16_bits(quant_code(v[i].z, s)), b3 = int_to_bf16_bits(quant_code(v[i].w, s));
+      qr[k] = make_uint2(b0 | (b1 << 16), b2 | (b3 << 16));
+    }
+  }
+  if (threadIdx.x == 0) deq[row] = __fdiv_rn(a, 127.f);
+}
+
 struct Bf16In {
   uint16_t bits;
   __device__ __forceinline__ explicit operator float() const { return __uint_as_float((uint32_t)bits << 16); }
 };
-
-// h_k = relu(gate_k)^2 * up_k, then per-row absmax int8.
-__global__ void k_relu2_quant(const float* __restrict__ gu, int F, uint16_t* __restrict__ q,
-                              float* __restrict__ deq) {
-  __shared__ float red[32];
-  const size_t row = blockIdx.x;
-  const float* g = gu + row * (size_t)(2 * F);
-  const float* u = g + F;
-  float amax = 0.f;
-  for (int k = threadIdx.x; k < F; k += blockDim.x) {
-    const float gr = fmaxf(g[k], 0.f);
-    amax = fmaxf(amax, fabsf(__fmul_rn(__fmul_rn(gr, gr), u[k])));
-  }
-  const float a = fmaxf(block_max(amax, red), 1e-5f);
-  const float s = __fdiv_rn(127.f, a);
-  uint16_t* qr = q + row * (size_t)F;
-  for (int k = threadIdx.x; k < F; k += blockDim.x) {
-    const float gr = fmaxf(g[k], 0.f);
-    qr[k] = int_to_bf16_bits(quant_code(__fmul_rn(__fmul_rn(gr, gr), u[k]), s));
-  }
-  if (threadIdx.x == 0) deq[row] = __fdiv_rn(a, 127.f);
-}
 
 // One thread per packed word: 16 codes -> 16 bf16 values (32 bytes).
 __global__ void k_expand_codes(const uint32_t* __restrict__ words, uint64_t n_words, uint16_t* __restrict__ out) {
@@ -124,6 +162,34 @@ __global__ void k_expand_codes(const uint32_t* __restrict__ words, uint64_t n_wo
   uint4* o = reinterpret_cast<uint4*>(out + i * 16);
   o[0] = make_uint4(v[0], v[1], v[2], v[3]);
   o[1] = make_uint4(v[4], v[5], v[6], v[7]);
+}
+
+__device__ __forceinline__ void expand_word(uint32_t w, uint16_t* dst) {
+  uint32_t v[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const uint32_t c0 = (w >> (4 * j)) & 3u, c1 = (w >> (4 * j + 2)) & 3u;
+    const uint32_t b0 = c0 == 2u ? 0x3F80u : (c0 == 0u ? 0xBF80u : 0u);
+    const uint32_t b1 = c1 == 2u ? 0x3F80u : (c1 == 0u ? 0xBF80u : 0u);
+    v[j] = b0 | (b1 << 16);
+  }
+  uint4* o = reinterpret_cast<uint4*>(dst);
+  o[0] = make_uint4(v[0], v[1], v[2], v[3]);
+  o[1] = make_uint4(v[4], v[5], v[6], v[7]);
+}
+
+// One thread per (interleaved row, word).
+__global__ void k_expand_gate_up(const uint32_t* __restrict__ gw, const uint32_t* __restrict__ uw, int F, int wpr,
+                                 uint64_t n_words, uint16_t* __restrict__ out) {
+  const uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n_words) return;
+  const uint64_t r = i / wpr;
+  const int jw = (int)(i % wpr);
+  const int blk = (int)(r / 256), within = (int)(r % 256);
+  const int src = blk * 128 + (within & 127);
+  uint32_t w = 0x55555555u;  // code 1 (value 0) in every slot
+  if (src < F) w = (within < 128 ? gw : uw)[(size_t)src * wpr + jw];
+  expand_word(w, out + i * 16);
 }
 
 __global__ void k_embed(const int32_t* __restrict__ tok, const float* __restrict__ embed, int D, int V,
@@ -216,16 +282,43 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 __device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
 
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(smem)),
+               "l"(gmem)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3, const void* p) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"((uint32_t)__cvta_generic_to_shared(p)));
+}
+
 // Causal attention, two passes over the keys: pass 1 finds the exact row
 // maximum of the scores, pass 2 forms P = bf16(exp(s - max)), l = sum P and
-// O = P V / l.  4 warps x 16 query rows per block; bf16 mma.sync tiles.
+// O = P V / l.  4 warps x 16 query rows per block; bf16 mma.sync tiles fed
+// by ldmatrix from a double-buffered cp.async ring of 64-key K / V^T tiles.
+template <int HD>
+struct AttnSmem {
+  static constexpr int KP = HD + 8, VP = 64 + 8;
+  static constexpr int K_ELEMS = 64 * KP, V_ELEMS = HD * VP;
+  static constexpr int BYTES = 2 * (K_ELEMS + V_ELEMS) * 2;
+};
+
 template <int HD>
 __global__ void __launch_bounds__(128) k_attention(const uint16_t* __restrict__ Q, const uint16_t* __restrict__ K,
                                                    const uint16_t* __restrict__ Vt, int S, int H, int KV,
                                                    float scale, float* __restrict__ out) {
-  constexpr int KP = HD + 8, VP = 64 + 8;
-  __shared__ __align__(16) uint16_t Ks[64 * KP];
-  __shared__ __align__(16) uint16_t Vs[HD * VP];
+  using L = AttnSmem<HD>;
+  constexpr int KP = L::KP, VP = L::VP;
+  extern __shared__ __align__(16) uint16_t att_smem[];
+  uint16_t* Ks = att_smem;                      // [2][64][KP]
+  uint16_t* Vs = att_smem + 2 * L::K_ELEMS;     // [2][HD][VP]
   const int qblk = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int kvh = h / (H / KV);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -248,31 +341,50 @@ __global__ void __launch_bounds__(128) k_attention(const uint16_t* __restrict__ 
   const int r0 = q0 + g, r1 = q0 + g + 8;
   float mx0 = -FLT_MAX, mx1 = -FLT_MAX;
 
-  auto load_k = [&](int kb) {
+  auto load_k = [&](int kb, int buf) {
+    uint16_t* dst = Ks + buf * L::K_ELEMS;
     for (int i = threadIdx.x; i < 64 * (HD / 8); i += 128) {
       const int r = i / (HD / 8), c8 = i % (HD / 8);
-      *reinterpret_cast<uint4*>(&Ks[r * KP + c8 * 8]) =
-          *reinterpret_cast<const uint4*>(Kp + (size_t)(kb * 64 + r) * HD + c8 * 8);
+      cp_async16(&dst[r * KP + c8 * 8], Kp + (size_t)(kb * 64 + r) * HD + c8 * 8);
     }
   };
-  auto scores = [&](float (&sacc)[8][4]) {
+  auto load_v = [&](int kb, int buf) {
+    uint16_t* dst = Vs + buf * L::V_ELEMS;
+    for (int i = threadIdx.x; i < HD * 8; i += 128) {
+      const int d = i / 8, c8 = i % 8;
+      cp_async16(&dst[d * VP + c8 * 8], Vp + (size_t)d * S + kb * 64 + c8 * 8);
+    }
+  };
+  // ldmatrix lane -> row address: lanes 8m..8m+7 address the rows of matrix m.
+  const int lm_row = lane & 7, lm_mat = lane >> 3;
+  auto scores = [&](const uint16_t* ks, float (&sacc)[8][4]) {
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       sacc[j][0] = sacc[j][1] = sacc[j][2] = sacc[j][3] = 0.f;
 #pragma unroll
-      for (int kk = 0; kk < HD / 16; ++kk) {
-        const uint16_t* kr = &Ks[(j * 8 + g) * KP + kk * 16 + 2 * c];
-        mma_16816(sacc[j], qa[kk], *reinterpret_cast<const uint32_t*>(kr), *reinterpret_cast<const uint32_t*>(kr + 8));
+      for (int kk = 0; kk < HD / 16; kk += 2) {
+        // matrices: (kk, lo8), (kk, hi8), (kk+1, lo8), (kk+1, hi8) of key rows j*8..j*8+7
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4(b0, b1, b2, b3, &ks[(j * 8 + lm_row) * KP + (kk + (lm_mat >> 1)) * 16 + (lm_mat & 1) * 8]);
+        mma_16816(sacc[j], qa[kk], b0, b1);
+        if (kk + 1 < HD / 16) mma_16816(sacc[j], qa[kk + 1], b2, b3);
       }
     }
   };
 
+  load_k(0, 0);
+  cp_async_commit();
   for (int kb = 0; kb < nkb; ++kb) {
-    __syncthreads();
-    load_k(kb);
+    if (kb + 1 < nkb) {
+      load_k(kb + 1, (kb + 1) & 1);
+      cp_async_commit();
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
     __syncthreads();
     float sacc[8][4];
-    scores(sacc);
+    scores(Ks + (kb & 1) * L::K_ELEMS, sacc);
 #pragma unroll
     for (int j = 0; j < 8; ++j)
 #pragma unroll
@@ -284,6 +396,7 @@ __global__ void __launch_bounds__(128) k_attention(const uint16_t* __restrict__ 
           if (e < 2) mx0 = fmaxf(mx0, s); else mx1 = fmaxf(mx1, s);
         }
       }
+    __syncthreads();
   }
 #pragma unroll
   for (int o = 1; o <= 2; o <<= 1) {
@@ -295,17 +408,22 @@ __global__ void __launch_bounds__(128) k_attention(const uint16_t* __restrict__ 
 #pragma unroll
   for (int n = 0; n < HD / 8; ++n) oacc[n][0] = oacc[n][1] = oacc[n][2] = oacc[n][3] = 0.f;
   float l0 = 0.f, l1 = 0.f;
+  load_k(0, 0);
+  load_v(0, 0);
+  cp_async_commit();
   for (int kb = 0; kb < nkb; ++kb) {
-    __syncthreads();
-    load_k(kb);
-    for (int i = threadIdx.x; i < HD * 8; i += 128) {
-      const int d = i / 8, c8 = i % 8;
-      *reinterpret_cast<uint4*>(&Vs[d * VP + c8 * 8]) =
-          *reinterpret_cast<const uint4*>(Vp + (size_t)d * S + kb * 64 + c8 * 8);
+    if (kb + 1 < nkb) {
+      load_k(kb + 1, (kb + 1) & 1);
+      load_v(kb + 1, (kb + 1) & 1);
+      cp_async_commit();
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
     }
     __syncthreads();
+    const uint16_t* vs = Vs + (kb & 1) * L::V_ELEMS;
     float sacc[8][4];
-    scores(sacc);
+    scores(Ks + (kb & 1) * L::K_ELEMS, sacc);
     uint32_t pf[8][2];
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
@@ -325,11 +443,15 @@ __global__ void __launch_bounds__(128) k_attention(const uint16_t* __restrict__ 
     for (int kc = 0; kc < 4; ++kc) {
       const uint32_t a[4] = {pf[2 * kc][0], pf[2 * kc][1], pf[2 * kc + 1][0], pf[2 * kc + 1][1]};
 #pragma unroll
-      for (int n = 0; n < HD / 8; ++n) {
-        const uint16_t* vr = &Vs[(n * 8 + g) * VP + kc * 16 + 2 * c];
-        mma_16816(oacc[n], a, *reinterpret_cast<const uint32_t*>(vr), *reinterpret_cast<const uint32_t*>(vr + 8));
+      for (int n = 0; n < HD / 8; n += 2) {
+        // matrices: (n, keys lo8), (n, keys hi8), (n+1, lo8), (n+1, hi8) of this key chunk
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4(b0, b1, b2, b3, &vs[((n + (lm_mat >> 1)) * 8 + lm_row) * VP + kc * 16 + (lm_mat & 1) * 8]);
+        mma_16816(oacc[n], a, b0, b1);
+        mma_16816(oacc[n + 1], a, b2, b3);
       }
     }
+    __syncthreads();
   }
 #pragma unroll
   for (int o = 1; o <= 2; o <<= 1) {
@@ -408,7 +530,23 @@ uint64_t& kernel_launches() {
 
 void launch_norm_quant(const float* x, const float* gain, int M, int D, uint16_t* q, float* deq, cudaStream_t s) {
   kernel_launches() += 1;
-  k_norm_quant<float><<<M, 256, 0, s>>>(x, gain, D, q, deq);
+  const int vpt = (D + 1023) / 1024;
+  const bool aligned = (D % 4 == 0) && ((uintptr_t)x % 16 == 0) && ((uintptr_t)q % 8 == 0) &&
+                       (!gain || (uintptr_t)gain % 16 == 0);
+  if (!aligned || vpt > 8) {
+    k_norm_quant<float><<<M, 256, 0, s>>>(x, gain, D, q, deq);
+    return;
+  }
+  switch (vpt) {
+    case 1: k_norm_quant_vec<1><<<M, 256, 0, s>>>(x, gain, D, q, deq); break;
+    case 2: k_norm_quant_vec<2><<<M, 256, 0, s>>>(x, gain, D, q, deq); break;
+    case 3: k_norm_quant_vec<3><<<M, 256, 0, s>>>(x, gain, D, q, deq); break;
+    case 4: k_norm_quant_vec<4><<<M, 256, 0, s>>>(x, gain, D, q, deq); break;
+    case 5: k_norm_quant_vec<5><<<M, 256, 0, s>>>(x, gain, D, q, deq); break;
+    case 6: k_norm_quant_vec<6><<<M, 256, 0, s>>>(x, gain, D, q, deq); break;
+    case 7: k_norm_quant_vec<7><<<M, 256, 0, s>>>(x, gain, D, q, deq); break;
+    default: k_norm_quant_vec<8><<<M, 256, 0, s>>>(x, gain, D, q, deq); break;
+  }
 }
 
 void launch_norm_quant_bf16(const uint16_t* x, int M, int D, uint16_t* q, float* deq, cudaStream_t s) {
@@ -416,15 +554,19 @@ void launch_norm_quant_bf16(const uint16_t* x, int M, int D, uint16_t* q, float*
   k_norm_quant<Bf16In><<<M, 256, 0, s>>>(reinterpret_cast<const Bf16In*>(x), nullptr, D, q, deq);
 }
 
-void launch_relu2_quant(const float* gu, int M, int F, uint16_t* q, float* deq, cudaStream_t s) {
-  kernel_launches() += 1;
-  k_relu2_quant<<<M, 256, 0, s>>>(gu, F, q, deq);
-}
-
 void launch_expand_codes(const uint32_t* words, uint64_t rows, int K, uint16_t* out, cudaStream_t s) {
   kernel_launches() += 1;
   const uint64_t n = rows * (uint64_t)(K / 16);
   k_expand_codes<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(words, n, out);
+}
+
+void launch_expand_gate_up(const uint32_t* gate_words, const uint32_t* up_words, int F, int K, uint16_t* out,
+                           cudaStream_t s) {
+  kernel_launches() += 1;
+  const int wpr = K / 16;
+  const uint64_t rows = 256ull * (uint64_t)((F + 127) / 128);
+  const uint64_t n = rows * (uint64_t)wpr;
+  k_expand_gate_up<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(gate_words, up_words, F, wpr, n, out);
 }
 
 void launch_embed(const int32_t* tok, const float* embed, int T, int D, int V, float* x, unsigned* err,
@@ -447,15 +589,26 @@ void launch_rope_pack(const float* qkv, const float* cosb, const float* sinb, in
   k_pack_vt<<<grid, dim3(32, 8), 0, s>>>(qkv, S, H, KV, hd, vt);
 }
 
+template <int HD>
+void attention_hd(const uint16_t* q, const uint16_t* k, const uint16_t* vt, int B, int S, int H, int KV, float scale,
+                  float* out, cudaStream_t s) {
+  static bool attr = false;
+  if (!attr) {
+    cudaFuncSetAttribute(k_attention<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, AttnSmem<HD>::BYTES);
+    attr = true;
+  }
+  dim3 grid(S / 64, H, B);
+  k_attention<HD><<<grid, 128, AttnSmem<HD>::BYTES, s>>>(q, k, vt, S, H, KV, scale, out);
+}
+
 void launch_attention(const uint16_t* q, const uint16_t* k, const uint16_t* vt, int B, int S, int H, int KV, int hd,
                       float* out, cudaStream_t s) {
   kernel_launches() += 1;
-  dim3 grid(S / 64, H, B);
   const float scale = 1.0f / sqrtf((float)hd);
   switch (hd) {
-    case 64: k_attention<64><<<grid, 128, 0, s>>>(q, k, vt, S, H, KV, scale, out); break;
-    case 96: k_attention<96><<<grid, 128, 0, s>>>(q, k, vt, S, H, KV, scale, out); break;
-    case 128: k_attention<128><<<grid, 128, 0, s>>>(q, k, vt, S, H, KV, scale, out); break;
+    case 64: attention_hd<64>(q, k, vt, B, S, H, KV, scale, out, s); break;
+    case 96: attention_hd<96>(q, k, vt, B, S, H, KV, scale, out, s); break;
+    case 128: attention_hd<128>(q, k, vt, B, S, H, KV, scale, out, s); break;
     default: break;
   }
 }

@@ -40,7 +40,7 @@ struct GemmSmem {
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int EPI_OFF = STAGES * STAGE_BYTES;
-  static constexpr int EPI_BYTES = EPI_WARPS * 32 * EPI_LD * 4;
+  static constexpr int EPI_BYTES = EPI_WARPS * 32 * (EPI_LD + 1) * 4;
   static constexpr int BAR_OFF = EPI_OFF + EPI_BYTES;
   static constexpr int BYTES = BAR_OFF + 256 + 1024;  // barriers + alignment slack
 };
@@ -220,35 +220,84 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     }
   } else {
     // Epilogue warps 2..5: warp w may access TMEM lanes 32*(w % 4) .. +31.
+    // Lane l owns row row0 + l when reading TMEM and column col0 + l when
+    // writing: the 32 x 32 block is transposed through shared memory so that
+    // every store (and residual load) is one coalesced 128-byte row segment.
     const int quarter = warp & 3;
-    float* stage = reinterpret_cast<float*>(smem + L::EPI_OFF) + (warp - 2) * 32 * EPI_LD;
+    float* stage = reinterpret_cast<float*>(smem + L::EPI_OFF) + (warp - 2) * 32 * (EPI_LD + 1);
+    float* dqs = stage + 32 * EPI_LD;  // the 32 rows' activation scales
     const float s0 = p.sw[0], s1 = p.sw[1], s2 = p.sw[2];
     uint32_t local = 0;
     for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++local) {
       const int m0 = (tile % n_mt) * BM, n0 = (tile / n_mt) * BN;
       const uint32_t b = local & 1u, j = local >> 1;
+      const int row0 = m0 + quarter * 32;
+      const int nrows = min(32, p.M - row0);
+      dqs[lane] = (lane < nrows) ? p.deq[row0 + lane] : 0.f;
       ok = mbar_wait(bar_tfull + 8 * b, j & 1u);
       if (!ok) break;
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-      const int row0 = m0 + quarter * 32;
-      for (int c = 0; c < BN / 32; ++c) {
-        uint32_t r[32];
-        tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + b * BN + (uint32_t)(c * 32), r);
+      if (p.relu2) {
+        // TMEM columns [0, BN/2) hold gate features f0.., [BN/2, BN) the up
+        // features f0..; lane = row: hid = relu(g)^2 * u, then transposed.
+        const int f0 = (n0 / BN) * (BN / 2);
+        const float dql = dqs[lane];
+        for (int c = 0; c < BN / 64; ++c) {
+          {
+            uint32_t g[32], u[32];
+            const uint32_t tb = tmem + ((uint32_t)(quarter * 32) << 16) + b * BN;
+            tmem_ld32(tb + (uint32_t)(c * 32), g);
+            tmem_ld32(tb + (uint32_t)(BN / 2 + c * 32), u);
 #pragma unroll
-        for (int q = 0; q < 32; ++q) stage[lane * EPI_LD + q] = __uint_as_float(r[q]);
+            for (int q = 0; q < 32; ++q) {
+              const float gv = fmaxf(__fmul_rn(__fmul_rn(__uint_as_float(g[q]), dql), s0), 0.f);
+              const float uv = __fmul_rn(__fmul_rn(__uint_as_float(u[q]), dql), s1);
+              stage[lane * EPI_LD + q] = __fmul_rn(__fmul_rn(gv, gv), uv);
+            }
+          }
+          __syncwarp();
+          const int col = f0 + c * 32 + lane;
+          if (col < p.n_out && nrows > 0) {
+            float* o = p.out + (size_t)row0 * p.ldo + col;
+#pragma unroll 8
+            for (int rr = 0; rr < 32; ++rr)
+              if (rr < nrows) o[(size_t)rr * p.ldo] = stage[rr * EPI_LD + lane];
+          }
+          __syncwarp();
+        }
+      }
+      for (int c = 0; c < (p.relu2 ? 0 : BN / 32); ++c) {
+        {
+          uint32_t r[32];
+          tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + b * BN + (uint32_t)(c * 32), r);
+#pragma unroll
+          for (int q = 0; q < 32; ++q) stage[lane * EPI_LD + q] = __uint_as_float(r[q]);
+        }
         __syncwarp();
         const int col = n0 + c * 32 + lane;
-        const float sw = col < p.n1 ? s0 : (col < p.n2 ? s1 : s2);
-        if (col < p.N) {
-          for (int rr = 0; rr < 32; ++rr) {
-            const int row = row0 + rr;
-            if (row >= p.M) break;
-            const float acc = stage[rr * EPI_LD + lane];
-            if (p.acc_out) p.acc_out[(size_t)row * p.N + col] = __float2int_rn(acc);
-            if (p.out) {
-              const float y = __fmul_rn(__fmul_rn(acc, p.deq[row]), sw);
-              float* o = p.out + (size_t)row * p.ldo + col;
-              *o = p.mode ? __fadd_rn(*o, y) : y;
+        if (col < p.N && nrows > 0) {
+          if (p.acc_out) {
+            int32_t* ao = p.acc_out + (size_t)row0 * p.N + col;
+#pragma unroll 8
+            for (int rr = 0; rr < 32; ++rr)
+              if (rr < nrows) ao[(size_t)rr * p.N] = __float2int_rn(stage[rr * EPI_LD + lane]);
+          }
+          if (p.out) {
+            const float sw = col < p.n1 ? s0 : (col < p.n2 ? s1 : s2);
+            float* o = p.out + (size_t)row0 * p.ldo + col;
+            if (p.mode) {
+              float prev[32];
+#pragma unroll
+              for (int rr = 0; rr < 32; ++rr) prev[rr] = rr < nrows ? o[(size_t)rr * p.ldo] : 0.f;
+#pragma unroll
+              for (int rr = 0; rr < 32; ++rr)
+                if (rr < nrows)
+                  o[(size_t)rr * p.ldo] =
+                      __fadd_rn(prev[rr], __fmul_rn(__fmul_rn(stage[rr * EPI_LD + lane], dqs[rr]), sw));
+            } else {
+#pragma unroll 8
+              for (int rr = 0; rr < 32; ++rr)
+                if (rr < nrows) o[(size_t)rr * p.ldo] = __fmul_rn(__fmul_rn(stage[rr * EPI_LD + lane], dqs[rr]), sw);
             }
           }
         }

@@ -23,6 +23,10 @@ struct GemmArgs {
   const float* deq;     // [M] per-row activation scale a/127
   const float* sw;      // three column-segment weight scales sw[0..2]
   int n1, n2;           // segment bounds: [0,n1) sw[0], [n1,n2) sw[1], [n2,N) sw[2]
+  int relu2;            // fused gate/up: B rows interleave 128 gate and 128 up rows per
+                        // 256-row tile; out[m, f] = relu(g)^2 * u with g scaled by sw[0],
+                        // u by sw[1]; f < n_out (out is [M, ldo])
+  int n_out;
   unsigned* err;        // device error word
 };
 
@@ -39,10 +43,13 @@ cudaError_t gemm_launch(const GemmPlan& plan, GemmArgs args, cudaStream_t stream
 // of h = x (gain == nullptr): q bf16 [M, D] (ld = D), deq[m] = a / 127.
 void launch_norm_quant(const float* x, const float* gain, int M, int D, uint16_t* q, float* deq,
                        cudaStream_t s);
-// h = relu(gate)^2 * up for gu = [gate | up] fp32 [M, 2F]; quantised as above.
-void launch_relu2_quant(const float* gu, int M, int F, uint16_t* q, float* deq, cudaStream_t s);
 // Packed 2-bit codes [rows, K/16] -> bf16 {-1, 0, +1} [rows, K].
 void launch_expand_codes(const uint32_t* words, uint64_t rows, int K, uint16_t* out, cudaStream_t s);
+// gate, up codes (two [F, K/16] word matrices) -> bf16 [256 * ceil(F/128), K]
+// with 256-row tiles [gate rows 128b..128b+127 | up rows 128b..128b+127]
+// (rows beyond F are zero).
+void launch_expand_gate_up(const uint32_t* gate_words, const uint32_t* up_words, int F, int K, uint16_t* out,
+                           cudaStream_t s);
 // x[t] = embed[tok[t]].
 void launch_embed(const int32_t* tok, const float* embed, int T, int D, int V, float* x, unsigned* err,
                   cudaStream_t s);
