@@ -41,6 +41,7 @@ WORKLOADS = {
     "2b": (synth.BITNET_2B, 0.01),
     "2b-0.1": (synth.BITNET_2B, 0.001),
     "0.7b": (synth.BITNET_07B, 0.01),
+    "2b-long": (synth.BITNET_2B_LONG, 0.05),
     "tiny": (synth.TINY, 0.01),
 }
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}

@@ -59,8 +59,8 @@ int make_shape(const termezo_model_cfg* c, Shape* s) {
     if (s->hd != 64 && s->hd != 96 && s->hd != 128) return TERMEZO_EINVAL;
     if (c->seq % 64) return TERMEZO_EINVAL;
     if (c->vocab <= 0) return TERMEZO_EINVAL;
-    if (c->loss_mode != 0) return TERMEZO_EINVAL;  // token-level loss: not provided by this build
-    if (c->n_labels < 1 || c->n_labels > 64 || c->n_labels > c->vocab) return TERMEZO_EINVAL;
+    if (c->loss_mode != 0 && c->loss_mode != 1) return TERMEZO_EINVAL;
+    if (c->loss_mode == 0 && (c->n_labels < 1 || c->n_labels > 64 || c->n_labels > c->vocab)) return TERMEZO_EINVAL;
     const int Hq = s->H * s->hd, Hkv = s->KV * s->hd;
     const int n[7] = {Hq, Hkv, Hkv, s->D, s->F, s->F, s->D};
     const int k[7] = {s->D, s->D, s->D, Hq, s->D, s->D, s->F};
@@ -73,7 +73,7 @@ int make_shape(const termezo_model_cfg* c, Shape* s) {
   }
   for (int p = 0; p < s->P; ++p) s->base.push_back(s->base.back() + (uint64_t)s->N[p] * (uint64_t)s->K[p]);
   s->d = s->base.back();
-  if (s->d >= (1ull << 32)) return TERMEZO_EINVAL;
+  if (s->d >= (1ull << 32) || s->P > 65535) return TERMEZO_EINVAL;
   return TERMEZO_OK;
 }
 
@@ -126,7 +126,13 @@ struct termezo_ctx {
   double* per_seq = nullptr;  // [2B]
   double* loss = nullptr;     // [2]
   double* g = nullptr;        // [1]
-  GemmPlan plan_qkv{}, plan_o{}, plan_gu{}, plan_down{};
+  GemmPlan plan_qkv{}, plan_o{}, plan_gu{}, plan_down{}, plan_head{};
+  bool head_plan_ok = false;
+  // loss mode 1 (token-level cross-entropy over the vocabulary)
+  uint16_t* hfin = nullptr;   // bf16 [T, D]
+  float2* part = nullptr;     // [T, ceil(V/256)]
+  float* tlogit = nullptr;    // [T]
+  double* tok_loss = nullptr; // [T]
   const float* code_sw = nullptr;  // s_w array matching the codes now in the packed store
   uint64_t pm_seed = 0;
   float pm_eps = 0.f;
@@ -178,6 +184,8 @@ void carve(termezo_ctx* c, Carver& cv) {
   a.base = cv.take<uint64_t>(P + 1);
   a.dpre = cv.take<uint32_t>(P + 1);
   a.spre = cv.take<uint32_t>(P + 1);
+  a.dproj = cv.take<uint16_t>(c->dpre.empty() ? 1 : c->dpre.back());
+  a.sproj = cv.take<uint16_t>(c->NBS_max);
   a.packed = cv.take<uint32_t>(s.d / 16);
   for (int i = 0; i < 2; ++i) {
     a.idx[i] = cv.take<uint32_t>(c->k_cap);
@@ -216,6 +224,12 @@ void carve(termezo_ctx* c, Carver& cv) {
     c->gu = cv.take<float>(T * 2 * (size_t)s.F);
     c->cosb = cv.take<float>((size_t)s.S * s.hd / 2);
     c->sinb = cv.take<float>((size_t)s.S * s.hd / 2);
+    if (s.mode == 1) {
+      c->hfin = cv.take<uint16_t>(T * s.D);
+      c->part = cv.take<float2>(T * (size_t)tmz::gemm_col_tiles(s.V));
+      c->tlogit = cv.take<float>(T);
+      c->tok_loss = cv.take<double>(T);
+    }
   }
   c->per_seq = cv.take<double>(2 * (size_t)s.B);
   c->loss = cv.take<double>(2);
@@ -363,8 +377,26 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
       if (tmz::gemm_launch(c->plan_down, a, st) != cudaSuccess) return TERMEZO_ECUDA;
     }
   }
-  tmz::launch_head_ce_last(c->x, c->gains + (size_t)(2 * s.L) * D, c->head, targets, s.B, s.S, D, s.V, s.C,
-                           c->per_seq + (size_t)slot * s.B, c->loss + slot, st);
+  if (s.mode == 0) {
+    tmz::launch_head_ce_last(c->x, c->gains + (size_t)(2 * s.L) * D, c->head, targets, s.B, s.S, D, s.V, s.C,
+                             c->per_seq + (size_t)slot * s.B, c->loss + slot, st);
+  } else {
+    if (!c->head_plan_ok) return TERMEZO_ESTATE;
+    tmz::launch_final_norm_bf16(c->x, c->gains + (size_t)(2 * s.L) * D, T, D, c->hfin, st);
+    GemmArgs h{};
+    h.lse = 1;
+    h.part = c->part;
+    h.tlogit = c->tlogit;
+    h.target = targets;
+    h.sw = sw;  // unused by the cross-entropy epilogue
+    h.err = c->ma.err;
+    {
+      ProfScope ps(c, 0, gemm_flops(c->plan_head));
+      if (tmz::gemm_launch(c->plan_head, h, st) != cudaSuccess) return TERMEZO_ECUDA;
+    }
+    tmz::launch_ce_reduce(c->part, tmz::gemm_col_tiles(s.V), c->tlogit, targets, s.B, s.S, s.V, c->tok_loss,
+                          c->per_seq + (size_t)slot * s.B, c->loss + slot, c->ma.err, st);
+  }
   return cuda_status(c);
 }
 
@@ -425,6 +457,12 @@ int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspa
   cudaStream_t st = c->stream;
   cudaMemcpyAsync((void*)c->ma.base, s.base.data(), (s.P + 1) * sizeof(uint64_t), cudaMemcpyHostToDevice, st);
   cudaMemcpyAsync((void*)c->ma.dpre, c->dpre.data(), (s.P + 1) * sizeof(uint32_t), cudaMemcpyHostToDevice, st);
+  {
+    std::vector<uint16_t> dproj(c->dpre.back());
+    for (int p = 0; p < s.P; ++p)
+      for (uint32_t b = c->dpre[p]; b < c->dpre[p + 1]; ++b) dproj[b] = (uint16_t)p;
+    cudaMemcpy((void*)c->ma.dproj, dproj.data(), dproj.size() * sizeof(uint16_t), cudaMemcpyHostToDevice);
+  }
   cudaMemsetAsync(c->ma.err, 0, sizeof(unsigned), st);
   cudaMemsetAsync(c->ma.counters, 0, 4 * sizeof(unsigned long long), st);
   for (float* f : {c->ma.gamma_cur, c->ma.tau_cur, c->ma.sw_cur, c->ma.gamma_plus, c->ma.tau_plus, c->ma.sw_plus,
@@ -461,6 +499,10 @@ int termezo_load_params(termezo_ctx* c, const float* d_latents, const float* d_e
   c->embed = d_embed;
   c->gains = d_gains;
   c->head = d_head;
+  if (!c->sh.op && c->sh.mode == 1) {
+    c->head_plan_ok = tmz::gemm_make_plan(&c->plan_head, c->hfin, c->sh.T, c->sh.D, d_head, c->sh.V);
+    if (!c->head_plan_ok) return TERMEZO_EINVAL;  // head must be 16-byte aligned
+  }
   return TERMEZO_OK;
 }
 
@@ -496,6 +538,10 @@ int termezo_build_mask(termezo_ctx* c, double density, uint64_t* k0_out, float* 
   if (spre[s.P] > c->NBS_max) return TERMEZO_ECUDA;
   c->ma.NBS = spre[s.P];
   cudaMemcpyAsync((void*)c->ma.spre, spre.data(), (s.P + 1) * sizeof(uint32_t), cudaMemcpyHostToDevice, st);
+  std::vector<uint16_t> sproj(spre[s.P]);
+  for (int p = 0; p < s.P; ++p)
+    for (uint32_t b = spre[p]; b < spre[p + 1]; ++b) sproj[b] = (uint16_t)p;
+  cudaMemcpyAsync((void*)c->ma.sproj, sproj.data(), sproj.size() * sizeof(uint16_t), cudaMemcpyHostToDevice, st);
   tmz::mask_finish(c->ma, st);
   c->cur = 0;
   c->k0 = k0;

@@ -47,6 +47,48 @@ __device__ __forceinline__ void es_merge(ExactSum& a, const ExactSum& o) {
   for (int i = 0; i < 4; ++i) a.b[i] += o.b[i];
 }
 
+// Per-thread accumulator with a fast path for |w| in [2^-63, 2) (biased
+// exponent 64..127, bucket 1): m << (e - 64) is split into two 64-bit words
+// (shift < 32, and shift - 32 for the rest, weighted 2^32), flushed into the
+// 128-bit bucket every 16 values (16 * 2^55 < 2^63).  Other values take
+// es_add_abs.  The result is the same exact integer.
+struct ExactAcc {
+  ExactSum s;
+  uint64_t a0, a1;
+  int cnt;
+};
+
+__device__ __forceinline__ void ea_zero(ExactAcc& a) {
+  es_zero(a.s);
+  a.a0 = a.a1 = 0;
+  a.cnt = 0;
+}
+
+__device__ __forceinline__ void ea_flush(ExactAcc& a) {
+  a.s.b[1] += (u128)a.a0 + ((u128)a.a1 << 32);
+  a.a0 = a.a1 = 0;
+  a.cnt = 0;
+}
+
+__device__ __forceinline__ void ea_add_abs(ExactAcc& a, float w) {
+  const uint32_t bits = __float_as_uint(w) & 0x7FFFFFFFu;
+  const uint32_t e = bits >> 23;
+  if (e >= 64u && e < 128u) {
+    const uint64_t m = (uint64_t)((bits & 0x7FFFFFu) | 0x800000u);
+    const uint32_t sh = e - 64u;
+    const uint64_t v = m << (sh & 31u);
+    if (sh < 32u) a.a0 += v; else a.a1 += v;
+    if (++a.cnt == 16) ea_flush(a);
+  } else {
+    es_add_abs(a.s, w);
+  }
+}
+
+__device__ __forceinline__ const ExactSum& ea_result(ExactAcc& a) {
+  ea_flush(a);
+  return a.s;
+}
+
 __device__ __forceinline__ u128 shfl_xor_u128(u128 v, int mask) {
   uint64_t lo = (uint64_t)v, hi = (uint64_t)(v >> 64);
   lo = __shfl_xor_sync(0xffffffffu, lo, mask);
@@ -54,11 +96,13 @@ __device__ __forceinline__ u128 shfl_xor_u128(u128 v, int mask) {
   return ((u128)hi << 64) | lo;
 }
 
+// Buckets that are zero in every lane (usually all but bucket 1) are skipped.
 __device__ __forceinline__ void es_warp_reduce(ExactSum& s) {
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
+  for (int i = 0; i < 4; ++i) {
+    if (!__any_sync(0xffffffffu, s.b[i] != 0)) continue;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) s.b[i] += shfl_xor_u128(s.b[i], off);
+    for (int off = 16; off > 0; off >>= 1) s.b[i] += shfl_xor_u128(s.b[i], off);
   }
 }
 

@@ -513,6 +513,66 @@ __global__ void k_head_ce_last(const float* __restrict__ x, const float* __restr
   }
 }
 
+// Final RMSNorm of one row per block, rounded to bf16 (the LM-head operand).
+__global__ void k_final_norm_bf16(const float* __restrict__ x, const float* __restrict__ gain, int D,
+                                  uint16_t* __restrict__ h) {
+  __shared__ float red[32];
+  const size_t row = blockIdx.x;
+  const float* xr = x + row * (size_t)D;
+  float ss = 0.f;
+  for (int k = threadIdx.x; k < D; k += blockDim.x) ss = __fadd_rn(ss, __fmul_rn(xr[k], xr[k]));
+  ss = block_sum(ss, red);
+  const float r = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(__fdiv_rn(ss, (float)D), 1e-5f)));
+  for (int k = threadIdx.x; k < D; k += blockDim.x) {
+    __nv_bfloat16 v = __float2bfloat16_rn(__fmul_rn(__fmul_rn(xr[k], r), gain[k]));
+    h[row * (size_t)D + k] = *reinterpret_cast<uint16_t*>(&v);
+  }
+}
+
+// One warp per row: log-sum-exp over the tiles' partials in float64.
+__global__ void k_ce_rows(const float2* __restrict__ part, int ntiles, const float* __restrict__ tlogit,
+                          const int32_t* __restrict__ target, int T, int V, double* __restrict__ tok_loss,
+                          unsigned* err) {
+  const int row = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= T) return;
+  const float2* pr = part + (size_t)row * ntiles;
+  float m = -INFINITY;
+  for (int j = lane; j < ntiles; j += 32) m = fmaxf(m, pr[j].x);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+  double acc = 0.0;
+  for (int j = lane; j < ntiles; j += 32) acc += (double)pr[j].y * exp((double)pr[j].x - (double)m);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+  if (lane == 0) {
+    const int tg = target[row];
+    if (tg < 0 || tg >= V) {
+      atomicOr(err, ERR_BOUNDS);
+      tok_loss[row] = 0.0;
+    } else {
+      tok_loss[row] = (double)m + log(acc) - (double)tlogit[row];
+    }
+  }
+}
+
+// Per-sequence mean of the token losses (fixed order, float64).
+__global__ void k_seq_mean(const double* __restrict__ tok_loss, int S, double* __restrict__ per_seq) {
+  __shared__ double red[32];
+  const int b = blockIdx.x;
+  double s = 0.0;
+  for (int i = threadIdx.x; i < S; i += blockDim.x) s += tok_loss[(size_t)b * S + i];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
+    per_seq[b] = t / (double)S;
+  }
+}
+
 __global__ void k_mean(const double* __restrict__ v, int n, double* __restrict__ out) {
   if (threadIdx.x == 0 && blockIdx.x == 0) {
     double t = 0.0;
@@ -611,6 +671,20 @@ void launch_attention(const uint16_t* q, const uint16_t* k, const uint16_t* vt, 
     case 128: attention_hd<128>(q, k, vt, B, S, H, KV, scale, out, s); break;
     default: break;
   }
+}
+
+void launch_final_norm_bf16(const float* x, const float* gain, int M, int D, uint16_t* h, cudaStream_t s) {
+  kernel_launches() += 1;
+  k_final_norm_bf16<<<M, 256, 0, s>>>(x, gain, D, h);
+}
+
+void launch_ce_reduce(const float2* part, int ntiles, const float* tlogit, const int32_t* target, int B, int S,
+                      int V, double* tok_loss, double* per_seq, double* total, unsigned* err, cudaStream_t s) {
+  kernel_launches() += 3;
+  const int T = B * S;
+  k_ce_rows<<<(T + 7) / 8, 256, 0, s>>>(part, ntiles, tlogit, target, T, V, tok_loss, err);
+  k_seq_mean<<<B, 256, 0, s>>>(tok_loss, S, per_seq);
+  k_mean<<<1, 32, 0, s>>>(per_seq, B, total);
 }
 
 void launch_head_ce_last(const float* x, const float* gain, const uint16_t* head, const int32_t* targets, int B,

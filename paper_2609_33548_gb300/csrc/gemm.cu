@@ -233,11 +233,42 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       const uint32_t b = local & 1u, j = local >> 1;
       const int row0 = m0 + quarter * 32;
       const int nrows = min(32, p.M - row0);
-      dqs[lane] = (lane < nrows) ? p.deq[row0 + lane] : 0.f;
+      dqs[lane] = (lane < nrows && p.deq) ? p.deq[row0 + lane] : 0.f;
       ok = mbar_wait(bar_tfull + 8 * b, j & 1u);
       if (!ok) break;
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-      if (p.relu2) {
+      if (p.lse) {
+        // lane = row: running max and sum of exp over this tile's columns
+        const int row = row0 + lane;
+        const int tg = (lane < nrows) ? p.target[row] : -1;
+        float m = -INFINITY, se = 0.f;
+        for (int c = 0; c < BN / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + b * BN + (uint32_t)(c * 32), r);
+          const int col0 = n0 + c * 32;
+          float cm = -INFINITY;
+#pragma unroll
+          for (int q = 0; q < 32; ++q)
+            if (col0 + q < p.N) cm = fmaxf(cm, __uint_as_float(r[q]));
+          const float mn = fmaxf(m, cm);
+          if (mn != -INFINITY) {
+            float t = (m == -INFINITY) ? 0.f : __fmul_rn(se, expf(__fsub_rn(m, mn)));
+#pragma unroll
+            for (int q = 0; q < 32; ++q)
+              if (col0 + q < p.N) t = __fadd_rn(t, expf(__fsub_rn(__uint_as_float(r[q]), mn)));
+            se = t;
+            m = mn;
+          }
+          if (tg >= col0 && tg < col0 + 32) {
+            float tv = 0.f;
+#pragma unroll
+            for (int q = 0; q < 32; ++q)
+              if (col0 + q == tg) tv = __uint_as_float(r[q]);
+            p.tlogit[row] = tv;
+          }
+        }
+        if (lane < nrows) p.part[(size_t)row * n_nt + (n0 / BN)] = make_float2(m, se);
+      } else if (p.relu2) {
         // TMEM columns [0, BN/2) hold gate features f0.., [BN/2, BN) the up
         // features f0..; lane = row: hid = relu(g)^2 * u, then transposed.
         const int f0 = (n0 / BN) * (BN / 2);
@@ -266,7 +297,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           __syncwarp();
         }
       }
-      for (int c = 0; c < (p.relu2 ? 0 : BN / 32); ++c) {
+      for (int c = 0; c < ((p.relu2 || p.lse) ? 0 : BN / 32); ++c) {
         {
           uint32_t r[32];
           tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + b * BN + (uint32_t)(c * 32), r);
@@ -354,6 +385,8 @@ bool gemm_make_plan(GemmPlan* plan, const uint16_t* a, int M, int K, const uint1
   return encode_bf16_kmajor(&plan->a, a, (uint64_t)M, (uint64_t)K, BM) &&
          encode_bf16_kmajor(&plan->b, b, (uint64_t)N, (uint64_t)K, GEMM_BN);
 }
+
+int gemm_col_tiles(int N) { return (N + GEMM_BN - 1) / GEMM_BN; }
 
 cudaError_t gemm_launch(const GemmPlan& plan, GemmArgs args, cudaStream_t stream) {
   static bool attr_set = false;

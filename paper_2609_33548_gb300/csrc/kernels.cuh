@@ -27,8 +27,17 @@ struct GemmArgs {
                         // 256-row tile; out[m, f] = relu(g)^2 * u with g scaled by sw[0],
                         // u by sw[1]; f < n_out (out is [M, ldo])
   int n_out;
+  int lse;              // LM-head cross-entropy partials instead of an output matrix:
+                        // part[m * ceil(N/BN) + j] = (max, sum exp(acc - max)) over the
+                        // columns n < N of tile j; tlogit[m] = acc[m, target[m]]
+  float2* part;
+  float* tlogit;
+  const int32_t* target;
   unsigned* err;        // device error word
 };
+
+// Column tiles of the GEMM (the stride of GemmArgs::part).
+int gemm_col_tiles(int N);
 
 struct GemmPlan {
   CUtensorMap a, b;
@@ -64,6 +73,13 @@ void launch_rope_pack(const float* qkv, const float* cosb, const float* sinb, in
 // Causal GQA attention -> out fp32 [B*S, H*hd].
 void launch_attention(const uint16_t* q, const uint16_t* k, const uint16_t* vt, int B, int S, int H, int KV,
                       int hd, float* out, cudaStream_t s);
+// Final RMSNorm of every row, rounded to bf16: h bf16 [M, D].
+void launch_final_norm_bf16(const float* x, const float* gain, int M, int D, uint16_t* h, cudaStream_t s);
+// Loss mode 1: combines the per-tile (max, sum exp) partials of each row into
+// the log-sum-exp (float64), subtracts the target logit, and averages the
+// token losses of each sequence (per_seq[b], float64) and of the batch.
+void launch_ce_reduce(const float2* part, int ntiles, const float* tlogit, const int32_t* target, int B, int S,
+                      int V, double* tok_loss, double* per_seq, double* total, unsigned* err, cudaStream_t s);
 // Final RMSNorm + LM head over the label tokens at the last position and
 // cross-entropy (loss mode 0): per_seq[b] (fp64), total = mean (fp64).
 void launch_head_ce_last(const float* x, const float* gain, const uint16_t* head, const int32_t* targets,

@@ -27,13 +27,14 @@ static __device__ __align__(256) tmz::ExactSum g_partials[kMaxBlocks];
 __global__ void __launch_bounds__(kThreads) k_noalloc_partial(const float* __restrict__ w, uint64_t n,
                                                               tmz::ExactSum* __restrict__ parts) {
   __shared__ tmz::ExactSum red[kThreads / 32];
-  tmz::ExactSum s;
-  tmz::es_zero(s);
+  tmz::ExactAcc acc;
+  tmz::ea_zero(acc);
   const uint64_t start = (uint64_t)blockIdx.x * kChunk;
   for (uint32_t j = threadIdx.x; j < kChunk; j += kThreads) {
     const uint64_t i = start + j;
-    if (i < n) tmz::es_add_abs(s, w[i]);
+    if (i < n) tmz::ea_add_abs(acc, w[i]);
   }
+  tmz::ExactSum s = tmz::ea_result(acc);
   tmz::es_block_reduce(s, red);
   if (threadIdx.x == 0) parts[blockIdx.x] = s;
 }

@@ -19,15 +19,6 @@ namespace {
 constexpr int TPB = 256;
 constexpr uint32_t DENSE_CHUNK = 4096;  // elements per dense block (16 per thread)
 
-__device__ __forceinline__ int find_proj(const uint32_t* prefix, int P, uint32_t b) {
-  int lo = 0, hi = P - 1;  // largest p with prefix[p] <= b
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (prefix[mid] <= b) lo = mid; else hi = mid - 1;
-  }
-  return lo;
-}
-
 struct DenseRange {
   int proj;
   uint64_t start, end;
@@ -35,7 +26,7 @@ struct DenseRange {
 
 __device__ __forceinline__ DenseRange dense_range(const MaskArgs& a, uint32_t b) {
   DenseRange r;
-  r.proj = find_proj(a.dpre, a.P, b);
+  r.proj = a.dproj[b];
   r.start = a.base[r.proj] + (uint64_t)(b - a.dpre[r.proj]) * DENSE_CHUNK;
   const uint64_t e = r.start + DENSE_CHUNK;
   r.end = e < a.base[r.proj + 1] ? e : a.base[r.proj + 1];
@@ -49,7 +40,7 @@ struct SparseRange {
 
 __device__ __forceinline__ SparseRange sparse_range(const MaskArgs& a, const uint32_t* off, uint32_t b) {
   SparseRange r;
-  r.proj = find_proj(a.spre, a.P, b);
+  r.proj = a.sproj[b];
   const uint32_t nb = a.spre[r.proj + 1] - a.spre[r.proj];
   const uint32_t j = b - a.spre[r.proj];
   r.seg_beg = off[r.proj];
@@ -92,20 +83,37 @@ __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* sh, ui
   return wpre + x - v;
 }
 
+// Loads the 4096-element chunk of a dense block with a coalesced pattern
+// (thread t reads float4 number q * 256 + t); for passes where the order of
+// elements within the block does not matter.
+__device__ __forceinline__ int load16_coalesced(const float* w, const DenseRange& r, float (&v)[16]) {
+  int n = 0;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const uint64_t i = r.start + 4ull * (q * TPB + threadIdx.x);
+    float4 t = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (i < r.end) {
+      t = *reinterpret_cast<const float4*>(w + i);
+      n = 4 * (q + 1);
+    }
+    v[4 * q] = t.x; v[4 * q + 1] = t.y; v[4 * q + 2] = t.z; v[4 * q + 3] = t.w;
+  }
+  return n;  // valid values are a prefix of v (chunk lengths are multiples of 16)
+}
+
 // ----------------------------------------------------------- dense passes --
 
 __global__ void __launch_bounds__(TPB) k_dense_sum(MaskArgs a, const float* __restrict__ w) {
   __shared__ ExactSum red[TPB / 32];
   const DenseRange r = dense_range(a, blockIdx.x);
-  ExactSum s;
-  es_zero(s);
-  const uint64_t i0 = r.start + 16ull * threadIdx.x;
-  if (i0 < r.end) {
-    float v[16];
-    load16(w, i0, v);
+  ExactAcc acc;
+  ea_zero(acc);
+  float v[16];
+  const int n = load16_coalesced(w, r, v);
 #pragma unroll
-    for (int j = 0; j < 16; ++j) es_add_abs(s, v[j]);
-  }
+  for (int j = 0; j < 16; ++j)
+    if (j < n) ea_add_abs(acc, v[j]);
+  ExactSum s = ea_result(acc);
   es_block_reduce(s, red);
   if (threadIdx.x == 0) a.partials[blockIdx.x] = s;
 }
@@ -135,26 +143,40 @@ __device__ __forceinline__ bool key_filter(uint32_t key, int pass, uint32_t pref
   return (key >> 10) == prefix;
 }
 
+// Radix histogram.  Pass 0 (top 10 bits of the key: the distances crowd a
+// few exponent bins) counts into per-warp shared histograms to spread the
+// shared-memory atomics; passes 1-2 see few matching keys and share one.
 __global__ void __launch_bounds__(TPB) k_hist(MaskArgs a, const float* __restrict__ w, int pass) {
-  __shared__ uint32_t h[2048];
-  for (int i = threadIdx.x; i < 2048; i += TPB) h[i] = 0;
+  constexpr int NB0 = 1024;  // keys of non-negative floats have bit 31 clear
+  __shared__ uint32_t h[(TPB / 32) * NB0];
+  const int warp = threadIdx.x >> 5;
+  for (int i = threadIdx.x; i < (TPB / 32) * NB0; i += TPB) h[i] = 0;
   __syncthreads();
   const DenseRange r = dense_range(a, blockIdx.x);
   const float tau = a.tau_cur[r.proj];
   const uint32_t prefix = a.sel->prefix;
+  float v[16];
   const uint64_t i0 = r.start + 16ull * threadIdx.x;
-  if (i0 < r.end) {
-    float v[16];
-    load16(w, i0, v);
+  const int n = i0 < r.end ? 16 : 0;
+  if (n) load16(w, i0, v);
+  uint32_t* hw = pass == 0 ? h + warp * NB0 : h;
 #pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      uint32_t bin;
-      if (key_filter(__float_as_uint(boundary_distance(v[j], tau)), pass, prefix, &bin)) atomicAdd(&h[bin], 1u);
-    }
+  for (int j = 0; j < 16; ++j) {
+    uint32_t bin;
+    if (j < n && key_filter(__float_as_uint(boundary_distance(v[j], tau)), pass, prefix, &bin))
+      atomicAdd(&hw[bin], 1u);
   }
   __syncthreads();
-  for (int i = threadIdx.x; i < 2048; i += TPB)
-    if (h[i]) atomicAdd(&a.hist[i], (unsigned long long)h[i]);
+  if (pass == 0) {
+    for (int i = threadIdx.x; i < NB0; i += TPB) {
+      uint32_t t = 0;
+      for (int ww = 0; ww < TPB / 32; ++ww) t += h[ww * NB0 + i];
+      if (t) atomicAdd(&a.hist[i], (unsigned long long)t);
+    }
+  } else {
+    for (int i = threadIdx.x; i < 2048; i += TPB)
+      if (h[i]) atomicAdd(&a.hist[i], (unsigned long long)h[i]);
+  }
 }
 
 // Picks the radix bin that holds the krem-th smallest key (1-based).
@@ -181,12 +203,13 @@ __global__ void __launch_bounds__(TPB) k_count(MaskArgs a, const float* __restri
   const float tau = a.tau_cur[r.proj];
   const uint32_t key_p = a.sel->prefix;
   uint32_t less = 0, eq = 0;
+  float v[16];
   const uint64_t i0 = r.start + 16ull * threadIdx.x;
-  if (i0 < r.end) {
-    float v[16];
-    load16(w, i0, v);
+  const int n = i0 < r.end ? 16 : 0;
+  if (n) load16(w, i0, v);
 #pragma unroll
-    for (int j = 0; j < 16; ++j) {
+  for (int j = 0; j < 16; ++j) {
+    if (j < n) {
       const uint32_t key = __float_as_uint(boundary_distance(v[j], tau));
       less += key < key_p;
       eq += key == key_p;
@@ -301,9 +324,10 @@ __global__ void k_dense_offsets(MaskArgs a, uint32_t k0) {
 __global__ void __launch_bounds__(TPB) k_sparse_abs(MaskArgs a, int cur) {
   __shared__ ExactSum red[TPB / 32];
   const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
-  ExactSum s;
-  es_zero(s);
-  for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) es_add_abs(s, a.lat[cur][e]);
+  ExactAcc acc;
+  ea_zero(acc);
+  for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) ea_add_abs(acc, a.lat[cur][e]);
+  ExactSum s = ea_result(acc);
   es_block_reduce(s, red);
   if (threadIdx.x == 0) a.partials[blockIdx.x] = s;
 }
@@ -333,16 +357,29 @@ __device__ __forceinline__ void perturbed(float w, float z, float eps, float* wp
 __global__ void __launch_bounds__(TPB) k_sparse_pm_sum(MaskArgs a, int cur, uint64_t seed, float eps) {
   __shared__ ExactSum red[TPB / 32];
   const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
-  ExactSum sp, sm;
-  es_zero(sp);
-  es_zero(sm);
-  for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) {
-    const float z = normal_at(seed, a.idx[cur][e]);
-    float wp, wm, ee;
-    perturbed(a.lat[cur][e], z, eps, &wp, &wm, &ee);
-    es_add_abs(sp, wp);
-    es_add_abs(sm, wm);
+  ExactAcc ap, am;
+  ea_zero(ap);
+  ea_zero(am);
+  // four independent elements per iteration so the Philox chains overlap
+  for (uint32_t e0 = r.beg + threadIdx.x; e0 < r.end; e0 += 4 * TPB) {
+    float wp[4], wm[4];
+    bool live[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const uint32_t e = e0 + u * TPB;
+      live[u] = e < r.end;
+      float ee;
+      perturbed(live[u] ? a.lat[cur][e] : 0.f, normal_at(seed, live[u] ? a.idx[cur][e] : 0u), eps, &wp[u], &wm[u],
+                &ee);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+      if (live[u]) {
+        ea_add_abs(ap, wp[u]);
+        ea_add_abs(am, wm[u]);
+      }
   }
+  ExactSum sp = ea_result(ap), sm = ea_result(am);
   es_block_reduce(sp, red);
   if (threadIdx.x == 0) a.partials[2 * (size_t)blockIdx.x] = sp;
   es_block_reduce(sm, red);
@@ -351,19 +388,55 @@ __global__ void __launch_bounds__(TPB) k_sparse_pm_sum(MaskArgs a, int cur, uint
 
 // Rewrites the codes of the active weights.  sign +1: w + eps z at tau+;
 // sign -1: (w + eps z) - 2 eps z at tau- (and counts codes that differ from
-// the + pass); sign 0: w at tau_cur.  The first active element of each
-// packed word (the "leader") owns the read-modify-write of that word.
+// the + pass); sign 0: w at tau_cur.  Phase 1 computes the code of every
+// element of the block's range in parallel (into shared memory); phase 2 has
+// the first active element of each packed word (the "leader") read-modify-
+// write that word, so no two threads write the same word.
+constexpr uint32_t RQ_MAX = 4096;  // elements per sparse block (see the host's block plan)
+
+__device__ __forceinline__ void requant_codes(const MaskArgs& a, int sign, uint64_t seed, float eps, float tau,
+                                              float taup, uint32_t i, float w, uint32_t* code, uint32_t* code_p) {
+  if (sign == 0) {
+    *code = ternary_code(w, tau);
+    *code_p = *code;
+    return;
+  }
+  float wp, wm, ee;
+  perturbed(w, normal_at(seed, i), eps, &wp, &wm, &ee);
+  *code = ternary_code(sign > 0 ? wp : wm, tau);
+  *code_p = ternary_code(wp, taup);
+}
+
 __global__ void __launch_bounds__(TPB) k_sparse_requant(MaskArgs a, int cur, uint64_t seed, float eps, int sign) {
+  __shared__ uint8_t sc[RQ_MAX];
   __shared__ unsigned long long cnt[3];
   if (threadIdx.x < 3) cnt[threadIdx.x] = 0;
-  __syncthreads();
   const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
   const uint32_t* idx = a.idx[cur];
   const float* lat = a.lat[cur];
   const float* tau_sel = sign > 0 ? a.tau_plus : (sign < 0 ? a.tau_minus : a.tau_cur);
   const float tau = tau_sel[r.proj];
   const float taup = a.tau_plus[r.proj];
+  const uint32_t n = r.end - r.beg;
+  if (n > RQ_MAX) {  // cannot happen with the host's block plan; recorded, never silent
+    if (threadIdx.x == 0) atomicOr(a.err, ERR_BOUNDS);
+    return;
+  }
   uint32_t flips = 0, jumps = 0, words = 0;
+  // phase 1: codes of the block's own elements (bits 0-1: this pass, 2-3: + pass)
+  for (uint32_t j0 = threadIdx.x; j0 < n; j0 += 4 * TPB) {
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const uint32_t j = j0 + u * TPB;
+      if (j < n) {
+        uint32_t c, cp;
+        requant_codes(a, sign, seed, eps, tau, taup, idx[r.beg + j], lat[r.beg + j], &c, &cp);
+        sc[j] = (uint8_t)(c | (cp << 2));
+      }
+    }
+  }
+  __syncthreads();
+  // phase 2: leaders rewrite their words
   for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) {
     const uint32_t i = idx[e];
     if (e != r.seg_beg && (idx[e - 1] >> 4) == (i >> 4)) continue;  // not the leader
@@ -373,19 +446,17 @@ __global__ void __launch_bounds__(TPB) k_sparse_requant(MaskArgs a, int cur, uin
     for (uint32_t e2 = e; e2 < r.seg_end; ++e2) {
       const uint32_t i2 = idx[e2];
       if ((i2 >> 4) != wi) break;
-      const float w = lat[e2];
-      uint32_t code;
-      if (sign == 0) {
-        code = ternary_code(w, tau);
-      } else {
-        float wp, wm, ee;
-        perturbed(w, normal_at(seed, i2), eps, &wp, &wm, &ee);
-        code = ternary_code(sign > 0 ? wp : wm, tau);
-        if (sign < 0) {
-          const uint32_t cp = ternary_code(wp, taup);
-          flips += cp != code;
-          jumps += (cp ^ code) == 2u;  // 0 <-> 2 in the stored q+1 form
-        }
+      uint32_t code, cp;
+      if (e2 < r.end) {
+        const uint32_t v = sc[e2 - r.beg];
+        code = v & 3u;
+        cp = v >> 2;
+      } else {  // follower in the next block's range
+        requant_codes(a, sign, seed, eps, tau, taup, i2, lat[e2], &code, &cp);
+      }
+      if (sign < 0) {
+        flips += cp != code;
+        jumps += (cp ^ code) == 2u;  // 0 <-> 2 in the stored q+1 form
       }
       const uint32_t sh = 2 * (i2 & 15u);
       word = (word & ~(3u << sh)) | (code << sh);
@@ -411,17 +482,27 @@ __global__ void __launch_bounds__(TPB) k_sparse_update(MaskArgs a, int cur, uint
   const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
   const double g = use_host ? g_host : *g_dev;
   const float c = (float)((double)lr * g);
-  ExactSum s;
-  es_zero(s);
-  for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) {
-    const float z = normal_at(seed, a.idx[cur][e]);
-    float wp, wm, ee;
-    perturbed(a.lat[cur][e], z, eps, &wp, &wm, &ee);
-    const float wr = __fadd_rn(wm, ee);
-    const float wn = __fsub_rn(wr, __fmul_rn(c, z));
-    a.lat[cur][e] = wn;
-    es_add_abs(s, wn);
+  ExactAcc acc;
+  ea_zero(acc);
+  for (uint32_t e0 = r.beg + threadIdx.x; e0 < r.end; e0 += 4 * TPB) {
+    float wn[4];
+    bool live[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const uint32_t e = e0 + u * TPB;
+      live[u] = e < r.end;
+      const float z = normal_at(seed, live[u] ? a.idx[cur][e] : 0u);
+      float wp, wm, ee;
+      perturbed(live[u] ? a.lat[cur][e] : 0.f, z, eps, &wp, &wm, &ee);
+      const float wr = __fadd_rn(wm, ee);
+      wn[u] = __fsub_rn(wr, __fmul_rn(c, z));
+      if (live[u]) a.lat[cur][e] = wn[u];
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+      if (live[u]) ea_add_abs(acc, wn[u]);
   }
+  ExactSum s = ea_result(acc);
   es_block_reduce(s, red);
   if (threadIdx.x == 0) a.partials[blockIdx.x] = s;
 }
@@ -435,8 +516,8 @@ __global__ void __launch_bounds__(TPB) k_shrink_mark(MaskArgs a, int cur, float 
   const uint32_t* idx = a.idx[cur];
   const float* lat = a.lat[cur];
   const float tau = a.tau_cur[r.proj];
-  ExactSum s;
-  es_zero(s);
+  ExactAcc acc;
+  ea_zero(acc);
   uint32_t kept = 0, dropped = 0;
   for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) {
     const float w = lat[e];
@@ -444,7 +525,7 @@ __global__ void __launch_bounds__(TPB) k_shrink_mark(MaskArgs a, int cur, float 
       ++kept;
     } else {
       ++dropped;
-      es_add_abs(s, w);
+      ea_add_abs(acc, w);
     }
     const uint32_t i = idx[e];
     if (e != r.seg_beg && (idx[e - 1] >> 4) == (i >> 4)) continue;
@@ -463,6 +544,7 @@ __global__ void __launch_bounds__(TPB) k_shrink_mark(MaskArgs a, int cur, float 
     }
     if (touched) a.packed[wi] = word;
   }
+  ExactSum s = ea_result(acc);
   es_block_reduce(s, red);
   if (threadIdx.x == 0) a.partials[blockIdx.x] = s;
   uint32_t tk, td;

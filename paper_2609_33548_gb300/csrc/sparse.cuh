@@ -20,8 +20,10 @@ struct MaskArgs {
   int P;                        // projections
   const uint64_t* base;         // [P+1] first global index of each projection
   const uint32_t* dpre;         // [P+1] dense-block prefix (4096 elements per block)
+  const uint16_t* dproj;        // [NBD] projection of each dense block
   uint32_t NBD;                 // dense blocks
   const uint32_t* spre;         // [P+1] sparse-block prefix
+  const uint16_t* sproj;        // [NBS] projection of each sparse block
   uint32_t NBS;                 // sparse blocks
   uint32_t* packed;             // [d/16] 2-bit codes
   uint32_t* idx[2];             // active global indices (double buffer)

@@ -16,6 +16,8 @@ Tolerances:
   the update by lr dg z).
 * codes: bit-exact except active latents within 1e-5 s_w of a threshold.
 """
+import dataclasses
+
 import numpy as np
 import pytest
 import torch
@@ -28,20 +30,23 @@ from helpers import rel_err
 
 pytestmark = pytest.mark.gpu
 
-CFG = synth.TINY
+# the tiny decoder with the classification loss, and with the token-level
+# loss over a vocabulary that is not a multiple of the 256-column tile
+TINY_SFT = dataclasses.replace(synth.TINY, name="tiny-2L-d256-sft", vocab=1000, loss_mode=1, n_labels=0)
 DENSITY, EPS, LR = 0.01, 1e-3, 1e-6
 
 
-@pytest.fixture(scope="module")
-def inputs():
-    w = synth.latents(CFG)
-    emb, gains, head = synth.theta(CFG)
-    tok, tgt = synth.batch(CFG)
-    return w, emb, gains, head, tok, tgt
+@pytest.fixture(scope="module", params=[synth.TINY, TINY_SFT], ids=["last-token", "token-level"])
+def inputs(request):
+    cfg = request.param
+    w = synth.latents(cfg)
+    emb, gains, head = synth.theta(cfg)
+    tok, tgt = synth.batch(cfg)
+    return w, emb, gains, head, tok, tgt, cfg
 
 
 def _gpu_ctx(inputs):
-    w, emb, gains, head, tok, tgt = inputs
+    w, emb, gains, head, tok, tgt, CFG = inputs
     ctx = tz.Context(tz.make_cfg(CFG), DENSITY)
     dev = [t.cuda() for t in (w, emb, gains, head, tok, tgt)]
     ctx.termezo_load_params(dev[0], dev[1], dev[2], dev[3])
@@ -51,6 +56,10 @@ def _gpu_ctx(inputs):
 def _theta_np(inputs):
     return (inputs[1].numpy(), inputs[2].numpy(), inputs[3].float().numpy(), inputs[4].numpy(),
             inputs[5].numpy())
+
+
+def _cfg(inputs):
+    return inputs[6]
 
 
 def _split(codes, reg):
@@ -63,9 +72,9 @@ def test_forward_loss_matches_oracle(inputs):
     loss, per = ctx.termezo_forward_loss(dev[4], dev[5])
     loss2, per2 = ctx.termezo_forward_loss(dev[4], dev[5])
     assert loss == loss2 and np.array_equal(per, per2)          # deterministic
-    reg = otz.registry(CFG)
+    reg = otz.registry(_cfg(inputs))
     codes, tau, sw = otz.requantize(inputs[0].numpy(), reg)
-    per_o, mean_o = bitnet.batch_loss(CFG, _split(codes, reg), sw, *_theta_np(inputs))
+    per_o, mean_o = bitnet.batch_loss(_cfg(inputs), _split(codes, reg), sw, *_theta_np(inputs))
     assert rel_err(loss, mean_o) < 1e-3
     np.testing.assert_allclose(per, per_o, rtol=3e-3)
 
@@ -73,9 +82,9 @@ def test_forward_loss_matches_oracle(inputs):
 def test_one_step_matches_oracle(inputs):
     ctx, dev = _gpu_ctx(inputs)
     k0, xi0 = ctx.termezo_build_mask(DENSITY)
-    reg = otz.registry(CFG)
+    reg = otz.registry(_cfg(inputs))
     state = otz.build(inputs[0].numpy(), reg, DENSITY)
-    fn = otz.bitnet_loss_fn(CFG, *_theta_np(inputs))
+    fn = otz.bitnet_loss_fn(_cfg(inputs), *_theta_np(inputs))
     assert k0 == state.k0 and np.float32(xi0) == state.xi0
     w_before = state.w.copy()
     act = state.active.copy()
@@ -91,7 +100,7 @@ def test_one_step_matches_oracle(inputs):
     wm = wp.copy(); wm[act] = (wp[act] - np.float32(2) * e).astype(np.float32)
     cp, _, swp = otz.requantize(wp, reg)
     cm, _, swm = otz.requantize(wm, reg)
-    ens = rounding.g_ensemble(CFG, (_split(cp, reg), swp), (_split(cm, reg), swm), _theta_np(inputs), EPS)
+    ens = rounding.g_ensemble(_cfg(inputs), (_split(cp, reg), swp), (_split(cm, reg), swm), _theta_np(inputs), EPS)
     assert rounding.g_within_ensemble(out["g"], rec["g"], ens), (out["g"], rec["g"], ens)
     # counters
     assert out["k_active"] == rec["k"] == act.size
@@ -118,7 +127,7 @@ def test_mask_and_update_replay_many_steps(inputs):
     active set shrinks: indices bit-exact, latents within the rounding of
     the restore arithmetic."""
     w0 = inputs[0].numpy()
-    reg = otz.registry(CFG)
+    reg = otz.registry(_cfg(inputs))
     ctx, dev = _gpu_ctx(inputs)
     ctx.termezo_build_mask(DENSITY)
     state = otz.build(w0, reg, DENSITY)
