@@ -28,9 +28,13 @@ library routine or brute force in tests/test_oracle_bitnet.py):
 * loss mode 0: cross-entropy of the last position over the label tokens
   vocab-C .. vocab-1 (logits = bf16(h) . W_head[label]); loss mode 1:
   token-level cross-entropy over the full vocabulary at every position;
-* every value the kernels store in fp32 (residual stream, BitLinear
-  outputs, attention output, MLP hidden) is rounded to fp32 at the same
-  point here; all other arithmetic is float64.
+* precision: every value that is stored between kernels and feeds a
+  quantizer (the residual stream, RMSNorm output, BitLinear outputs, RoPE,
+  attention scores / probabilities / output, the MLP hidden) is computed in
+  float32, the kernels' precision, with plain numpy float32 operations in
+  the order the definition writes them (reductions in numpy's own order):
+  an int8 or bf16 code is decided on a float32 value on both sides.  The
+  LM-head logits of the last position and every cross-entropy are float64.
 """
 from __future__ import annotations
 
@@ -49,10 +53,15 @@ def bf16_round(x) -> np.ndarray:
     return (r & np.uint64(0xFFFFFFFF)).astype(np.uint32).view(np.float32)
 
 
+F32 = np.float32
+
+
 def rmsnorm(x: np.ndarray, gain: np.ndarray) -> np.ndarray:
-    x64 = x.astype(np.float64)
-    r = 1.0 / np.sqrt(np.mean(x64 * x64, axis=-1, keepdims=True) + RMS_EPS)
-    return (x64 * r * gain.astype(np.float64)).astype(np.float32)
+    """x * r * g with r = 1 / sqrt(mean(x^2) + 1e-5), float32."""
+    x = np.asarray(x, dtype=F32)
+    ms = (np.sum(x * x, axis=-1, keepdims=True, dtype=F32) / F32(x.shape[-1])).astype(F32)
+    r = (F32(1.0) / np.sqrt(ms + F32(RMS_EPS))).astype(F32)
+    return ((x * r).astype(F32) * np.asarray(gain, dtype=F32)).astype(F32)
 
 
 def act_quant(x: np.ndarray):
@@ -72,22 +81,27 @@ def int_matmul(q: np.ndarray, codes: np.ndarray) -> np.ndarray:
 
 
 def bitlinear(x: np.ndarray, codes: np.ndarray, s_w) -> np.ndarray:
+    """y = (acc * (a / 127)) * s_w in float32 (acc is an exact integer)."""
     q, a = act_quant(x)
-    acc = int_matmul(q, codes)
-    return (acc.astype(np.float64) * (a.astype(np.float64)[:, None] / 127.0)
-            * float(s_w)).astype(np.float32)
+    acc = int_matmul(q, codes).astype(F32)          # exact: |acc| < 2^24
+    dq = (a / F32(127.0)).astype(F32)
+    return ((acc * dq[:, None]).astype(F32) * F32(s_w)).astype(F32)
 
 
 def rope(x: np.ndarray, hd: int) -> np.ndarray:
-    """x: [S, nh, hd] fp32 at positions 0..S-1 -> rotated fp32."""
+    """x: [S, nh, hd] fp32 at positions 0..S-1 -> rotated fp32.  The angles
+    pos * 10000^(-2j/hd) and their cos / sin are float64, rounded to float32;
+    the rotation (x1 c - x2 s, x2 c + x1 s) is float32."""
     S = x.shape[0]
     half = hd // 2
     inv = ROPE_BASE ** (-(2.0 * np.arange(half)) / hd)
     ang = np.arange(S, dtype=np.float64)[:, None] * inv[None, :]
-    c, s = np.cos(ang)[:, None, :], np.sin(ang)[:, None, :]
-    x1 = x[..., :half].astype(np.float64)
-    x2 = x[..., half:].astype(np.float64)
-    return np.concatenate([x1 * c - x2 * s, x2 * c + x1 * s], axis=-1).astype(np.float32)
+    c = np.cos(ang).astype(F32)[:, None, :]
+    s = np.sin(ang).astype(F32)[:, None, :]
+    x1 = np.asarray(x[..., :half], dtype=F32)
+    x2 = np.asarray(x[..., half:], dtype=F32)
+    return np.concatenate([((x1 * c).astype(F32) - (x2 * s).astype(F32)).astype(F32),
+                           ((x2 * c).astype(F32) + (x1 * s).astype(F32)).astype(F32)], axis=-1)
 
 
 def attention(q: np.ndarray, k: np.ndarray, v: np.ndarray) -> np.ndarray:
@@ -95,17 +109,18 @@ def attention(q: np.ndarray, k: np.ndarray, v: np.ndarray) -> np.ndarray:
     q: [S, H, hd], k, v: [S, KV, hd] (fp32) -> [S, H*hd] fp32."""
     S, H, hd = q.shape
     KV = k.shape[1]
-    qb, kb, vb = (bf16_round(t).astype(np.float64) for t in (q, k, v))
-    scale = 1.0 / np.sqrt(hd)
+    qb, kb, vb = (bf16_round(t) for t in (q, k, v))
+    scale = F32(1.0) / np.sqrt(F32(hd))
     causal = np.tril(np.ones((S, S), dtype=bool))
-    out = np.empty((S, H, hd), dtype=np.float32)
+    out = np.empty((S, H, hd), dtype=F32)
     for h in range(H):
         j = h // (H // KV)
-        s = (qb[:, h, :] @ kb[:, j, :].T) * scale
-        s = np.where(causal, s, -np.inf)
-        p = np.exp(s - s.max(axis=1, keepdims=True))
-        pb = bf16_round(p.astype(np.float32)).astype(np.float64)
-        out[:, h, :] = ((pb @ vb[:, j, :]) / pb.sum(axis=1, keepdims=True)).astype(np.float32)
+        s = ((qb[:, h, :] @ kb[:, j, :].T).astype(F32) * scale).astype(F32)
+        s = np.where(causal, s, F32(-np.inf))
+        p = np.exp((s - s.max(axis=1, keepdims=True)).astype(F32)).astype(F32)
+        pb = bf16_round(p)
+        l = np.sum(pb, axis=1, keepdims=True, dtype=F32)
+        out[:, h, :] = ((pb @ vb[:, j, :]).astype(F32) / l).astype(F32)
     return out.reshape(S, H * hd)
 
 
@@ -137,9 +152,9 @@ def sequence_loss(cfg, codes, s_w, embed, gains, head, tokens, target) -> float:
         a = attention(rope(q, hd), rope(k, hd), v)
         x = (x + bitlinear(a, co, so)).astype(np.float32)
         h = rmsnorm(x, gains[2 * l + 1])
-        g = bitlinear(h, cg, sg).astype(np.float64)
-        u = bitlinear(h, cu, su).astype(np.float64)
-        hid = (np.maximum(g, 0.0) ** 2 * u).astype(np.float32)
+        g = np.maximum(bitlinear(h, cg, sg), F32(0.0))
+        u = bitlinear(h, cu, su)
+        hid = ((g * g).astype(F32) * u).astype(F32)
         x = (x + bitlinear(hid, cd, sd)).astype(np.float32)
     h = bf16_round(rmsnorm(x, gains[2 * cfg.layers])).astype(np.float64)
     W = np.asarray(head, dtype=np.float64)
@@ -147,7 +162,7 @@ def sequence_loss(cfg, codes, s_w, embed, gains, head, tokens, target) -> float:
         C = cfg.n_labels
         logits = h[S - 1:S] @ W[cfg.vocab - C:].T
         return float(cross_entropy(logits, np.array([int(target)]))[0])
-    logits = h @ W.T
+    logits = (h.astype(F32) @ W.astype(F32).T).astype(F32)   # tensor-core logits: bf16 x bf16, fp32 sums
     return float(cross_entropy(logits, np.asarray(target, dtype=np.int64)).mean())
 
 

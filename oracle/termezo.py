@@ -98,16 +98,24 @@ def keep_count(rho0: float, d: int) -> int:
     return int(math.floor(float(rho0) * float(d)))
 
 
+def select_smallest(d: np.ndarray, k0: int):
+    """The k0 smallest (d_i, i) pairs: xi = the k0-th smallest distance;
+    every i with d_i < xi, then the lowest indices with d_i == xi.
+    Returns (sorted indices, xi)."""
+    if k0 == 0:
+        return np.zeros(0, dtype=np.int64), np.float32(0.0)
+    xi = np.float32(np.partition(d, k0 - 1)[k0 - 1])
+    below = np.flatnonzero(d < xi)
+    ties = np.flatnonzero(d == xi)[:k0 - below.size]
+    return np.sort(np.concatenate([below, ties])).astype(np.int64), xi
+
+
 def initial_mask(w: np.ndarray, reg, rho0: float):
     """Returns (S_0 as sorted int64 global indices, xi_0 float32, k0, tau_0)."""
     _, tau, _ = thresholds(w, reg)
     d = all_distances(w, reg, tau)
     k0 = keep_count(rho0, d.size)
-    if k0 == 0:
-        return np.zeros(0, dtype=np.int64), np.float32(0.0), 0, tau
-    order = np.argsort(d, kind="stable")  # equal distances: lower index first
-    sel = np.sort(order[:k0]).astype(np.int64)
-    xi0 = np.float32(d[order[k0 - 1]])
+    sel, xi0 = select_smallest(d, k0)
     return sel, xi0, k0, tau
 
 

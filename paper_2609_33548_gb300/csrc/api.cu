@@ -799,6 +799,14 @@ int termezo_profile(termezo_ctx* c, int enable, termezo_profile_out* out) {
   return TERMEZO_OK;
 }
 
+int termezo_attention(const uint16_t* d_q, const uint16_t* d_k, const uint16_t* d_vt, int32_t B, int32_t S,
+                      int32_t H, int32_t KV, int32_t hd, float* d_out, void* stream) {
+  if (!d_q || !d_k || !d_vt || !d_out || B <= 0 || S <= 0 || S % 64 || H <= 0 || KV <= 0 || H % KV) return TERMEZO_EINVAL;
+  if (hd != 64 && hd != 96 && hd != 128) return TERMEZO_EINVAL;
+  tmz::launch_attention(d_q, d_k, d_vt, B, S, H, KV, hd, d_out, reinterpret_cast<cudaStream_t>(stream));
+  return cudaGetLastError() == cudaSuccess ? TERMEZO_OK : TERMEZO_ECUDA;
+}
+
 void termezo_destroy(termezo_ctx* c) { delete c; }
 
 const char* termezo_strerror(int status) {

@@ -150,7 +150,8 @@ __global__ void __launch_bounds__(TPB) k_hist(MaskArgs a, const float* __restric
   constexpr int NB0 = 1024;  // keys of non-negative floats have bit 31 clear
   __shared__ uint32_t h[(TPB / 32) * NB0];
   const int warp = threadIdx.x >> 5;
-  for (int i = threadIdx.x; i < (TPB / 32) * NB0; i += TPB) h[i] = 0;
+  const int nz = pass == 0 ? (TPB / 32) * NB0 : 2048;
+  for (int i = threadIdx.x; i < nz; i += TPB) h[i] = 0;
   __syncthreads();
   const DenseRange r = dense_range(a, blockIdx.x);
   const float tau = a.tau_cur[r.proj];
@@ -360,24 +361,12 @@ __global__ void __launch_bounds__(TPB) k_sparse_pm_sum(MaskArgs a, int cur, uint
   ExactAcc ap, am;
   ea_zero(ap);
   ea_zero(am);
-  // four independent elements per iteration so the Philox chains overlap
-  for (uint32_t e0 = r.beg + threadIdx.x; e0 < r.end; e0 += 4 * TPB) {
-    float wp[4], wm[4];
-    bool live[4];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const uint32_t e = e0 + u * TPB;
-      live[u] = e < r.end;
-      float ee;
-      perturbed(live[u] ? a.lat[cur][e] : 0.f, normal_at(seed, live[u] ? a.idx[cur][e] : 0u), eps, &wp[u], &wm[u],
-                &ee);
-    }
-#pragma unroll
-    for (int u = 0; u < 4; ++u)
-      if (live[u]) {
-        ea_add_abs(ap, wp[u]);
-        ea_add_abs(am, wm[u]);
-      }
+  for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) {
+    const float z = normal_at(seed, a.idx[cur][e]);
+    float wp, wm, ee;
+    perturbed(a.lat[cur][e], z, eps, &wp, &wm, &ee);
+    ea_add_abs(ap, wp);
+    ea_add_abs(am, wm);
   }
   ExactSum sp = ea_result(ap), sm = ea_result(am);
   es_block_reduce(sp, red);
@@ -484,23 +473,14 @@ __global__ void __launch_bounds__(TPB) k_sparse_update(MaskArgs a, int cur, uint
   const float c = (float)((double)lr * g);
   ExactAcc acc;
   ea_zero(acc);
-  for (uint32_t e0 = r.beg + threadIdx.x; e0 < r.end; e0 += 4 * TPB) {
-    float wn[4];
-    bool live[4];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const uint32_t e = e0 + u * TPB;
-      live[u] = e < r.end;
-      const float z = normal_at(seed, live[u] ? a.idx[cur][e] : 0u);
-      float wp, wm, ee;
-      perturbed(live[u] ? a.lat[cur][e] : 0.f, z, eps, &wp, &wm, &ee);
-      const float wr = __fadd_rn(wm, ee);
-      wn[u] = __fsub_rn(wr, __fmul_rn(c, z));
-      if (live[u]) a.lat[cur][e] = wn[u];
-    }
-#pragma unroll
-    for (int u = 0; u < 4; ++u)
-      if (live[u]) ea_add_abs(acc, wn[u]);
+  for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) {
+    const float z = normal_at(seed, a.idx[cur][e]);
+    float wp, wm, ee;
+    perturbed(a.lat[cur][e], z, eps, &wp, &wm, &ee);
+    const float wr = __fadd_rn(wm, ee);
+    const float wn = __fsub_rn(wr, __fmul_rn(c, z));
+    a.lat[cur][e] = wn;
+    ea_add_abs(acc, wn);
   }
   ExactSum s = ea_result(acc);
   es_block_reduce(s, red);

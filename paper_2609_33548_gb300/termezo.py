@@ -22,7 +22,7 @@ EXPORTS = (
     "termezo_workspace_bytes", "termezo_create", "termezo_load_params", "termezo_build_mask",
     "termezo_forward_loss", "termezo_step", "termezo_shrink", "termezo_requantize", "termezo_update",
     "termezo_bitlinear", "termezo_state_sizes", "termezo_export_state", "termezo_normal",
-    "termezo_absmean_noalloc", "termezo_profile", "termezo_destroy", "termezo_strerror",
+    "termezo_absmean_noalloc", "termezo_attention", "termezo_profile", "termezo_destroy", "termezo_strerror",
 )
 
 
@@ -93,6 +93,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         "termezo_export_state": (I32, [P, P, P, P, P]),
         "termezo_normal": (I32, [U64, P, U64, P, P]),
         "termezo_absmean_noalloc": (I32, [P, U64, P, P]),
+        "termezo_attention": (I32, [P, P, P, I32, I32, I32, I32, I32, P, P]),
         "termezo_profile": (I32, [P, I32, ctypes.POINTER(ProfileOut)]),
         "termezo_destroy": (None, [P]),
         "termezo_strerror": (ctypes.c_char_p, [I32]),
@@ -251,3 +252,12 @@ def termezo_absmean_noalloc(w, out, stream=None):
     allocate: the library's fixed scratch array is used)."""
     _check("termezo_absmean_noalloc", load().termezo_absmean_noalloc(_ptr(w), w.numel(), _ptr(out),
                                                                      _stream(stream)))
+
+
+def termezo_attention(q, k, vt, out, stream=None):
+    """Causal attention op: q bf16 [B, H, S, hd], k bf16 [B, KV, S, hd],
+    vt bf16 [B, KV, hd, S] -> out fp32 [B*S, H*hd]."""
+    B, H, S, hd = q.shape
+    KV = k.shape[1]
+    _check("termezo_attention", load().termezo_attention(_ptr(q), _ptr(k), _ptr(vt), B, S, H, KV, hd, _ptr(out),
+                                                         _stream(stream)))

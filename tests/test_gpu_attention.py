@@ -1,0 +1,36 @@
+"""The attention kernel against the oracle's attention (causal, grouped KV
+heads, bf16 Q/K/V and P, exact row maximum) on bf16-exact inputs, across
+sequence lengths (several 64-key blocks), head dims and GQA ratios."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import bitnet
+from paper_2609_33548_gb300 import termezo as tz
+
+pytestmark = pytest.mark.gpu
+
+CASES = [(1, 64, 4, 4, 64), (2, 256, 4, 4, 64), (1, 192, 4, 2, 128), (1, 128, 4, 4, 96), (1, 512, 4, 1, 64),
+         (1, 512, 20, 5, 128), (1, 2048, 2, 1, 128)]
+
+
+@pytest.mark.parametrize("B,S,H,KV,hd", CASES)
+def test_attention_matches_oracle(B, S, H, KV, hd):
+    g = torch.Generator().manual_seed(S * 1000 + hd)
+    q = torch.randn(B, H, S, hd, generator=g).to(torch.bfloat16)
+    k = torch.randn(B, KV, S, hd, generator=g).to(torch.bfloat16)
+    v = torch.randn(B, KV, S, hd, generator=g).to(torch.bfloat16)
+    out = torch.empty(B * S, H * hd, dtype=torch.float32, device="cuda")
+    tz.termezo_attention(q.cuda(), k.cuda(), v.transpose(2, 3).contiguous().cuda(), out)
+    torch.cuda.synchronize()
+    got = out.cpu().numpy().reshape(B, S, H * hd)
+    for b in range(B):
+        ref = bitnet.attention(q[b].float().permute(1, 0, 2).numpy(), k[b].float().permute(1, 0, 2).numpy(),
+                               v[b].float().permute(1, 0, 2).numpy())
+        err = np.abs(got[b] - ref)
+        # fp32 sums in another order; a P that rounds to the other bf16 value
+        # moves its row by at most 2^-8 * P * |v| / sum P
+        assert np.median(err) < 1e-5, np.median(err)
+        assert err.max() < 2e-2, err.max()
+        rel = np.abs(got[b] - ref).sum(axis=1) / (np.abs(ref).sum(axis=1) + 1e-30)
+        assert np.percentile(rel, 99) < 2e-4

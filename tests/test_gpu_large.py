@@ -1,0 +1,141 @@
+"""GPU parity at the full model-shaped workloads (0.7B-, 2B- and 2B-long-
+shaped: 24-30 layers, d 1536-2560, 0.68-2.08 G latents) in the launch
+configuration bench.py times.
+
+* Mask (Eqs. 2-4) at full size: S_0, xi_0 and tau_0 of every projection
+  bit-exact against the oracle's global selection, and the packed codes of
+  every weight bit for bit.
+* Perturb / requantise (Eq. 2, Algorithm 1) after one full step, on sampled
+  projections: tau+ and tau- bit-exact, codes of the - pass bit-exact except
+  latents within 1e-5 s_w of a threshold.
+* BitLinear GEMM at the 2B shapes (M 8192 tokens): int32 accumulators of
+  sampled rows bit-exact.
+* One step on the 0.7B model: the loss of each sequence depends only on that
+  sequence, so sampled sequences are evaluated by the oracle at +eps z and
+  -eps z (1e-3, or inside the spread of valid fp32 roundings).
+Inputs are drawn on the host by the seeded generator (so the oracle can
+redraw them anywhere) and copied to the device."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import bitnet, philox, rounding, ternary, termezo as otz
+from paper_2609_33548_gb300 import synth
+from paper_2609_33548_gb300 import termezo as tz
+
+pytestmark = pytest.mark.gpu
+
+EPS, LR = 1e-3, 1e-6
+
+
+def _setup(cfg, density):
+    w = synth.latents(cfg)
+    emb, gains, head = synth.theta(cfg)
+    tok, tgt = synth.batch(cfg)
+    ctx = tz.Context(tz.make_cfg(cfg), density)
+    dev = [t.cuda() for t in (w, emb, gains, head, tok, tgt)]
+    ctx.termezo_load_params(dev[0], dev[1], dev[2], dev[3])
+    return ctx, dev, (w.numpy(), emb.numpy(), gains.numpy(), head.float().numpy(), tok.numpy(), tgt.numpy())
+
+
+def _mask_exact(ctx, w, reg, density):
+    k0, xi0 = ctx.termezo_build_mask(density)
+    st = ctx.termezo_export_state()
+    sel, xi0_o, k0_o, tau = otz.initial_mask(w, reg, density)
+    assert k0 == k0_o
+    assert np.float32(xi0).view(np.uint32) == np.float32(xi0_o).view(np.uint32)
+    np.testing.assert_array_equal(st["tau_cur"].view(np.uint32), tau.view(np.uint32))
+    np.testing.assert_array_equal(st["idx"], sel.astype(np.uint32))
+    np.testing.assert_array_equal(st["latents"], w[sel])
+    for j, p in enumerate(reg):  # packed codes, projection by projection
+        np.testing.assert_array_equal(st["packed"][p.base // 16:(p.base + p.n) // 16],
+                                      ternary.pack_codes(ternary.quantize(w[p.base:p.base + p.n], tau[j])))
+    return sel
+
+
+def _requant_sampled(ctx, w, reg, act, seed, picks):
+    st = ctx.termezo_export_state()
+    z_all = philox.normal(seed, act)
+    for j in picks:
+        p = reg[j]
+        lo, hi = np.searchsorted(act, [p.base, p.base + p.n])
+        a, z = act[lo:hi], z_all[lo:hi]
+        e = (np.float32(EPS) * z).astype(np.float32)
+        v = w[p.base:p.base + p.n].copy()
+        v[a - p.base] = (v[a - p.base] + e).astype(np.float32)
+        gp = ternary.absmean(v)
+        tp = ternary.threshold(gp)
+        v[a - p.base] = (v[a - p.base] - np.float32(2) * e).astype(np.float32)
+        gm = ternary.absmean(v)
+        tm, swm = ternary.threshold(gm), ternary.weight_scale(gm)
+        assert st["tau_plus"][j].view(np.uint32) == tp.view(np.uint32), (p, st["tau_plus"][j], tp)
+        assert st["tau_minus"][j].view(np.uint32) == tm.view(np.uint32), (p, st["tau_minus"][j], tm)
+        got = ternary.unpack_codes(st["packed"][p.base // 16:(p.base + p.n) // 16])
+        want = ternary.quantize(v, tm)
+        bad = np.flatnonzero(got != want) + p.base
+        near = a[otz.near_threshold(v[a - p.base], np.full(a.size, tm), np.full(a.size, swm))]
+        assert np.all(np.isin(bad, near)), (p, bad.size)
+
+
+@pytest.mark.parametrize("name", ["2b", "2b-long"])
+def test_full_size_mask_requant_and_gemm(name):
+    cfg, density = {"2b": (synth.BITNET_2B, 0.01), "2b-long": (synth.BITNET_2B_LONG, 0.05)}[name]
+    ctx, dev, (w, *_r) = _setup(cfg, density)
+    reg = otz.registry(cfg)
+    act = _mask_exact(ctx, w, reg, density)
+    seed = synth.step_seed(0)
+    out = ctx.termezo_step(seed, EPS, LR, density, dev[4], dev[5])
+    assert out["k_active"] == act.size and out["n_jumps"] == 0
+    picks = [0, 7 * 14 + 4, len(reg) - 1]          # layer 0 q, layer 14 gate, last down
+    _requant_sampled(ctx, w, reg, act, seed, picks)
+    if name == "2b":
+        # the BitLinear GEMM at the model's token count, on codes at tau_0
+        ctx2 = tz.Context(tz.make_cfg(cfg), density)
+        ctx2.termezo_load_params(dev[0], dev[1], dev[2], dev[3])
+        ctx2.termezo_build_mask(density)
+        j = 7 * 14 + 4
+        p = reg[j]
+        x = synth.op_activations(cfg.tokens, p.K, seed=31)
+        acc = torch.zeros(cfg.tokens, p.N, dtype=torch.int32, device="cuda")
+        ctx2.termezo_bitlinear(j, x.cuda(), acc, None)
+        torch.cuda.synchronize()
+        tau = ternary.threshold(ternary.absmean(w[p.base:p.base + p.n]))
+        codes = ternary.quantize(w[p.base:p.base + p.n], tau).reshape(p.N, p.K)
+        rows = np.random.default_rng(3).choice(cfg.tokens, 64, replace=False)
+        q, _ = bitnet.act_quant(x.float().numpy()[rows])
+        np.testing.assert_array_equal(acc.cpu().numpy()[rows], bitnet.int_matmul(q, codes))
+
+
+def test_step_sampled_sequences_0_7b():
+    cfg, density = synth.BITNET_07B, 0.01
+    ctx, dev, (w, emb, gains, head, tok, tgt) = _setup(cfg, density)
+    reg = otz.registry(cfg)
+    act = _mask_exact(ctx, w, reg, density)
+    seed = synth.step_seed(0)
+    out = ctx.termezo_step(seed, EPS, LR, density, dev[4], dev[5])
+    z = philox.normal(seed, act)
+    e = (np.float32(EPS) * z).astype(np.float32)
+    wp = w.copy()
+    wp[act] = (w[act] + e).astype(np.float32)
+    wm = wp.copy()
+    wm[act] = (wp[act] - np.float32(2) * e).astype(np.float32)
+    cp, tp, swp = otz.requantize(wp, reg)
+    cm, tm, swm = otz.requantize(wm, reg)
+    st = ctx.termezo_export_state(packed=False)
+    np.testing.assert_array_equal(st["tau_plus"].view(np.uint32), tp.view(np.uint32))
+    np.testing.assert_array_equal(st["tau_minus"].view(np.uint32), tm.view(np.uint32))
+    split = lambda c: [c[p.base:p.base + p.n].reshape(p.N, p.K) for p in reg]
+    th = (emb, gains, head, tok, tgt)
+    rows = [0, 1]
+    per_p, _ = bitnet.batch_loss(cfg, split(cp), swp, *th, rows=rows)
+    per_m, _ = bitnet.batch_loss(cfg, split(cm), swm, *th, rows=rows)
+    ens_p = rounding.loss_ensemble(cfg, (split(cp), swp), th, n=6, rows=rows)
+    ens_m = rounding.loss_ensemble(cfg, (split(cm), swm), th, n=6, rows=rows)
+    two_eps = 2 * float(np.float32(EPS))
+    for i, b in enumerate(rows):
+        assert rounding.within(out["per_seq_plus"][b], per_p[i], ens_p[:, i]), (b, out["per_seq_plus"][b], per_p[i])
+        assert rounding.within(out["per_seq_minus"][b], per_m[i], ens_m[:, i])
+        g_gpu = (out["per_seq_plus"][b] - out["per_seq_minus"][b]) / two_eps
+        g_ref = (per_p[i] - per_m[i]) / two_eps
+        assert rounding.within(g_gpu, g_ref, (ens_p[:, i] - ens_m[:, i]) / two_eps), (b, g_gpu, g_ref)
+    assert out["n_jumps"] == 0 and out["k_active"] == act.size
