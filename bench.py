@@ -394,13 +394,54 @@ def run_op(args):
     print(json.dumps(line), flush=True)
 
 
+ATTN_WORKLOADS = {"attn-2b": synth.BITNET_2B, "attn-2b-long": synth.BITNET_2B_LONG}
+
+
+def run_attn(args):
+    """Causal attention op at a model's attention shape (q [B, H, S, hd],
+    k and V^T of the KV heads), the kernel one forward launches per layer;
+    seeded normal bf16 inputs."""
+    from paper_2609_33548_gb300 import termezo as tz
+
+    cfg = ATTN_WORKLOADS[args.workload]
+    B, S, H, KV, hd = cfg.batch, cfg.seq, cfg.heads, cfg.kv_heads, cfg.head_dim
+    dev = torch.device("cuda", 0)
+    g = torch.Generator(device=dev).manual_seed(77)
+    q = torch.randn(B, H, S, hd, generator=g, device=dev).to(torch.bfloat16)
+    k = torch.randn(B, KV, S, hd, generator=g, device=dev).to(torch.bfloat16)
+    vt = torch.randn(B, KV, hd, S, generator=g, device=dev).to(torch.bfloat16)
+    out = torch.empty(B * S, H * hd, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        tz.termezo_attention(q, k, vt, out, stream)
+    ts = []
+    for _ in range(args.steps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        tz.termezo_attention(q, k, vt, out, stream)
+        b.record(stream)
+        torch.cuda.synchronize()
+        ts.append(a.elapsed_time(b))
+    ms = statistics.median(ts)
+    flops = 4.0 * B * H * hd * (0.5 * S * (S + 1.0))
+    pk, how = peaks()
+    line = {"metric": "causal attention op (exact row max, bf16 P)", "value": flops / (ms / 1e3) / 1e12,
+            "unit": "TFLOP/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic",
+            "config": {"workload": f"attention B{B} S{S} H{H} KV{KV} hd{hd}",
+                       "flops": "4 B H hd S(S+1)/2 (causal QK^T and PV)"},
+            "peak_bf16_tflops": float(pk.get("bf16_tflops", 1900.0)), "peak_source": how}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=("mine", "reference"), default="mine")
-    ap.add_argument("--workload", choices=sorted(WORKLOADS) + ["op"], default="2b")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS) + ["op"] + sorted(ATTN_WORKLOADS), default="2b")
     ap.add_argument("--op-density", type=float, default=0.01)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
@@ -410,6 +451,8 @@ def main():
         run_reference(args)
     elif args.workload == "op":
         run_op(args)
+    elif args.workload in ATTN_WORKLOADS:
+        run_attn(args)
     else:
         run_mine(args)
 

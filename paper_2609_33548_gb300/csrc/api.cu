@@ -127,6 +127,8 @@ struct termezo_ctx {
   double* loss = nullptr;     // [2]
   double* g = nullptr;        // [1]
   GemmPlan plan_qkv{}, plan_o{}, plan_gu{}, plan_down{}, plan_head{};
+  tmz::AttnPlan att_plan{};
+  bool att_tc = false;
   bool head_plan_ok = false;
   // loss mode 1 (token-level cross-entropy over the vocabulary)
   uint16_t* hfin = nullptr;   // bf16 [T, D]
@@ -336,7 +338,12 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
     tmz::launch_rope_pack(c->qkv, c->cosb, c->sinb, s.B, s.S, s.H, s.KV, s.hd, c->qb, c->kb, c->vt, st);
     {
       ProfScope ps(c, 1, 4.0 * s.B * s.H * (double)s.hd * (0.5 * s.S * (s.S + 1.0)));
-      tmz::launch_attention(c->qb, c->kb, c->vt, s.B, s.S, s.H, s.KV, s.hd, c->attn, st);
+      if (c->att_tc) {
+        if (tmz::attention_tc_launch(c->att_plan, s.B, s.S, s.H, s.KV, s.hd, c->attn, c->ma.err, st) != cudaSuccess)
+          return TERMEZO_ECUDA;
+      } else {
+        tmz::launch_attention(c->qb, c->kb, c->vt, s.B, s.S, s.H, s.KV, s.hd, c->attn, st);
+      }
     }
     tmz::launch_norm_quant(c->attn, nullptr, T, hq, c->xq, c->deq, st);
     tmz::launch_expand_codes(c->ma.packed + s.base[po] / 16, (uint64_t)D, hq, c->wexp, st);
@@ -479,6 +486,8 @@ int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspa
       delete c;
       return TERMEZO_ECUDA;
     }
+    c->att_tc = tmz::attention_tc_supported(s.S, s.hd) &&
+                tmz::attention_tc_plan(&c->att_plan, c->qb, c->kb, c->vt, s.B, s.S, s.H, s.KV, s.hd);
   }
   c->code_sw = c->ma.sw_cur;
   rc = sync_status(c);
@@ -803,7 +812,12 @@ int termezo_attention(const uint16_t* d_q, const uint16_t* d_k, const uint16_t* 
                       int32_t H, int32_t KV, int32_t hd, float* d_out, void* stream) {
   if (!d_q || !d_k || !d_vt || !d_out || B <= 0 || S <= 0 || S % 64 || H <= 0 || KV <= 0 || H % KV) return TERMEZO_EINVAL;
   if (hd != 64 && hd != 96 && hd != 128) return TERMEZO_EINVAL;
-  tmz::launch_attention(d_q, d_k, d_vt, B, S, H, KV, hd, d_out, reinterpret_cast<cudaStream_t>(stream));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  tmz::AttnPlan plan;
+  if (tmz::attention_tc_supported(S, hd) && tmz::attention_tc_plan(&plan, d_q, d_k, d_vt, B, S, H, KV, hd))
+    return tmz::attention_tc_launch(plan, B, S, H, KV, hd, d_out, nullptr, st) == cudaSuccess ? TERMEZO_OK
+                                                                                             : TERMEZO_ECUDA;
+  tmz::launch_attention(d_q, d_k, d_vt, B, S, H, KV, hd, d_out, st);
   return cudaGetLastError() == cudaSuccess ? TERMEZO_OK : TERMEZO_ECUDA;
 }
 
