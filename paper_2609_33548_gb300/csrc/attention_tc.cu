@@ -15,7 +15,7 @@
 // Warp 0 issues TMA loads (Q_A, Q_B; a ring of K and V^T tiles, 128-byte
 // swizzle); one thread of warp 1 issues tcgen05.mma: S_t = Q_t K^T into TMEM
 // buffer t (M 128, N 128, K hd) and O_t += P_t V (M 128, N hd, K 128) with P_t
-// from shared memory.  Warps 2-5 own tile A, warps 6-9 tile B (thread = query
+// from shared memory.  Warps 4-7 own tile A, warps 8-11 tile B (thread = query
 // row): they read S_t with tcgen05.ld, release the buffer at once (so S_t of
 // the next key block is computed while they work), reduce the row maximum
 // (pass 1) or form bf16 P rows in the swizzled K-major layout (pass 2), and at
@@ -32,7 +32,12 @@ namespace tmz {
 
 namespace {
 
-constexpr int ATT_THREADS = 320;  // warp 0 TMA, warp 1 MMA, warps 2-5 tile A, warps 6-9 tile B
+// Warp 0 TMA, warp 1 MMA (warps 2-3 idle): 136 registers a thread; warps 4-7
+// tile A, warps 8-11 tile B: 184.  128 x 136 + 256 x 184 = 384 x 168, the
+// registers the block is launched with.
+constexpr int ATT_THREADS = 384;
+constexpr int REG_CTRL = 136, REG_SOFTMAX = 184;
+static_assert(128 * REG_CTRL + 256 * REG_SOFTMAX == ATT_THREADS * 168, "register split");
 constexpr int BQ = 128, BKEY = 128;
 constexpr int ATOM = 128 * 128;  // one 128-row x 64-element bf16 swizzle atom block
 
@@ -112,6 +117,59 @@ __device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, uint32_t* r) {
   for (int c = 0; c < NC; ++c) tmem_tie32(r + 32 * c);
 }
 
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// Paired fp32 arithmetic (one instruction for two lanes of a float2), each
+// lane rounded to nearest like its scalar form.
+__device__ __forceinline__ float2 mul2(float2 a, float2 b) {
+  float2 d;
+  asm("{\n .reg .b64 x, y, z;\n mov.b64 x, {%2, %3};\n mov.b64 y, {%4, %5};\n mul.rn.f32x2 z, x, y;\n"
+      " mov.b64 {%0, %1}, z;\n}\n"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+__device__ __forceinline__ float2 sub2(float2 a, float2 b) {
+  float2 d;
+  asm("{\n .reg .b64 x, y, z;\n mov.b64 x, {%2, %3};\n mov.b64 y, {%4, %5};\n sub.rn.f32x2 z, x, y;\n"
+      " mov.b64 {%0, %1}, z;\n}\n"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+__device__ __forceinline__ float2 add2(float2 a, float2 b) {
+  float2 d;
+  asm("{\n .reg .b64 x, y, z;\n mov.b64 x, {%2, %3};\n mov.b64 y, {%4, %5};\n add.rn.f32x2 z, x, y;\n"
+      " mov.b64 {%0, %1}, z;\n}\n"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+
+// Keys c > row of the diagonal block are outside the causal window: their
+// accumulator becomes -inf, which the maximum ignores and exp maps to 0.
+__device__ __forceinline__ void causal_mask(uint32_t* sv, int row) {
+#pragma unroll
+  for (int c = 0; c < BKEY; ++c) sv[c] = c <= row ? sv[c] : 0xff800000u;
+}
+
+// P for keys c0 .. c0+7 of one row: 4 words of bf16 pairs; l2 += P (fp32).
+__device__ __forceinline__ uint4 p_chunk(const uint32_t* sv, int c0, float2 sc, float2 m2, float2& l2) {
+  uint32_t w[4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float2 x = sub2(mul2(make_float2(__uint_as_float(sv[c0 + 2 * e]), __uint_as_float(sv[c0 + 2 * e + 1])), sc), m2);
+    const __nv_bfloat162 b = __floats2bfloat162_rn(expf(x.x), expf(x.y));
+    w[e] = *reinterpret_cast<const uint32_t*>(&b);
+    l2 = add2(l2, make_float2(__uint_as_float(w[e] << 16), __uint_as_float(w[e] & 0xffff0000u)));
+  }
+  return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
 // Warp-uniform bounded wait (the tcgen05.ld that follows is warp-collective).
 __device__ __forceinline__ bool mbar_wait_warp(uint32_t bar, uint32_t parity) {
   return __all_sync(0xffffffffu, mbar_wait(bar, parity));
@@ -165,7 +223,8 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = *tmem_slot;
   bool ok = true;
-
+  if (warp < 4) {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(REG_CTRL));
   if (warp == 0) {
     if (lane == 0) {
       uint32_t rp = 0, nq = 0;
@@ -290,9 +349,11 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
       mma_commit(fin);
       if (!mbar_wait(fin, 0)) ok = false;
     }
+  }
   } else {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(REG_SOFTMAX));
     // Softmax warps: warp w reads TMEM lanes 32 (w % 4) .. +31; lane = row.
-    const int t = warp >= 6 ? 1 : 0;
+    const int t = warp >= 8 ? 1 : 0;
     const int quarter = warp & 3;
     const int row = quarter * 32 + lane;
     const uint32_t lanes = (uint32_t)(quarter * 32) << 16;
@@ -313,82 +374,53 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
       const int qt = t ? it.qb : it.qa, h = t ? it.hb : it.ha;
       if (h < 0) continue;
       const int n = qt + 1;
-      uint32_t sv[64];
+      uint32_t sv[BKEY];
       // pass 1: maximum of the raw accumulators over the causal keys
       float mx0 = -INFINITY, mx1 = -INFINITY;
       for (int j = 0; j < n; ++j) {
         if (!(ok = mbar_wait_warp(sfull, ns & 1u))) break;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        tmem_ld_cols<BKEY / 32>(tS, sv);
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        arrive(sfree);
+        ++ns;
+        if (j + 1 == n) causal_mask(sv, row);
 #pragma unroll
-        for (int hf = 0; hf < 2; ++hf) {
-          tmem_ld_cols<2>(tS + 64 * hf, sv);
-          if (hf == 1) {
-            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-            arrive(sfree);
-            ++ns;
-          }
-          if (j + 1 < n) {
-#pragma unroll
-            for (int c = 0; c < 64; c += 2) {
-              mx0 = fmaxf(mx0, __uint_as_float(sv[c]));
-              mx1 = fmaxf(mx1, __uint_as_float(sv[c + 1]));
-            }
-          } else {
-#pragma unroll
-            for (int c = 0; c < 64; c += 2) {
-              if (64 * hf + c <= row) mx0 = fmaxf(mx0, __uint_as_float(sv[c]));
-              if (64 * hf + c + 1 <= row) mx1 = fmaxf(mx1, __uint_as_float(sv[c + 1]));
-            }
-          }
+        for (int c = 0; c < BKEY; c += 4) {
+          mx0 = max3(mx0, __uint_as_float(sv[c]), __uint_as_float(sv[c + 1]));
+          mx1 = max3(mx1, __uint_as_float(sv[c + 2]), __uint_as_float(sv[c + 3]));
         }
       }
       if (!ok) break;
       const float m = __fmul_rn(fmaxf(mx0, mx1), scale);
+      const float2 sc2 = make_float2(scale, scale), m2 = make_float2(m, m);
       // pass 2: P = bf16(exp(fl(s) - m)), l = sum P, P -> shared memory
-      float l0 = 0.f, l1 = 0.f, l2 = 0.f, l3 = 0.f;
+      float2 la = make_float2(0.f, 0.f), lb = make_float2(0.f, 0.f);
       for (int j = 0; j < n; ++j) {
         if (!(ok = mbar_wait_warp(sfull, ns & 1u))) break;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        const bool diag = j + 1 == n;
-        uint32_t pk[BKEY / 2];
-#pragma unroll
-        for (int hf = 0; hf < 4; ++hf) {
-          tmem_ld_cols<1>(tS + 32 * hf, sv);
-          if (hf == 3) {
-            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-            arrive(sfree);
-            ++ns;
-          }
-#pragma unroll
-          for (int c = 0; c < 32; c += 4) {
-            float p[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const float x = __fsub_rn(__fmul_rn(__uint_as_float(sv[c + e]), scale), m);
-              p[e] = (!diag || 32 * hf + c + e <= row) ? expf(x) : 0.f;
-            }
-            const __nv_bfloat162 b01 = __floats2bfloat162_rn(p[0], p[1]), b23 = __floats2bfloat162_rn(p[2], p[3]);
-            const float2 f01 = __bfloat1622float2(b01), f23 = __bfloat1622float2(b23);
-            l0 = __fadd_rn(l0, f01.x);
-            l1 = __fadd_rn(l1, f01.y);
-            l2 = __fadd_rn(l2, f23.x);
-            l3 = __fadd_rn(l3, f23.y);
-            pk[16 * hf + c / 2] = *reinterpret_cast<const uint32_t*>(&b01);
-            pk[16 * hf + c / 2 + 1] = *reinterpret_cast<const uint32_t*>(&b23);
-          }
-        }
-        if (np >= 1 && !(ok = mbar_wait_warp(pfree, (np - 1) & 1u))) break;
+        tmem_ld_cols<BKEY / 32>(tS, sv);
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        arrive(sfree);
+        ++ns;
+        if (j + 1 == n) causal_mask(sv, row);
         // keys 8 ch .. 8 ch + 7 -> atom ch / 8, 16-byte chunk ch % 8, swizzled by row % 8
+        uint4 pk[8];
 #pragma unroll
-        for (int ch = 0; ch < BKEY / 8; ++ch)
-          *reinterpret_cast<uint4*>(prow + (ch >> 3) * ATOM + (((ch & 7) ^ (row & 7)) * 16)) =
-              make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2], pk[4 * ch + 3]);
+        for (int ch = 0; ch < 8; ++ch) pk[ch] = p_chunk(sv, 8 * ch, sc2, m2, (ch & 1) ? lb : la);
+        if (np >= 1 && !(ok = mbar_wait_warp(pfree, (np - 1) & 1u))) break;
+#pragma unroll
+        for (int ch = 0; ch < 8; ++ch) *reinterpret_cast<uint4*>(prow + (((ch & 7) ^ (row & 7)) * 16)) = pk[ch];
+#pragma unroll
+        for (int ch = 8; ch < 16; ++ch)
+          *reinterpret_cast<uint4*>(prow + ATOM + (((ch & 7) ^ (row & 7)) * 16)) =
+              p_chunk(sv, 8 * ch, sc2, m2, (ch & 1) ? lb : la);
         fence_async_smem();
         arrive(pfull);
         ++np;
       }
       if (!ok) break;
-      const float l = __fadd_rn(__fadd_rn(l0, l1), __fadd_rn(l2, l3));
+      const float l = __fadd_rn(__fadd_rn(la.x, la.y), __fadd_rn(lb.x, lb.y));
       if (!(ok = mbar_wait_warp(ofull, no & 1u))) break;
       ++no;
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
