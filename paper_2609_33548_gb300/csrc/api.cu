@@ -339,7 +339,7 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
     {
       ProfScope ps(c, 1, 4.0 * s.B * s.H * (double)s.hd * (0.5 * s.S * (s.S + 1.0)));
       if (c->att_tc) {
-        if (tmz::attention_tc_launch(c->att_plan, s.B, s.S, s.H, s.KV, s.hd, c->attn, c->ma.err, st) != cudaSuccess)
+        if (tmz::attention_tc_launch(c->att_plan, s.B, s.S, s.H, s.KV, s.hd, c->ma.err, st) != cudaSuccess)
           return TERMEZO_ECUDA;
       } else {
         tmz::launch_attention(c->qb, c->kb, c->vt, s.B, s.S, s.H, s.KV, s.hd, c->attn, st);
@@ -487,7 +487,7 @@ int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspa
       return TERMEZO_ECUDA;
     }
     c->att_tc = tmz::attention_tc_supported(s.S, s.hd) &&
-                tmz::attention_tc_plan(&c->att_plan, c->qb, c->kb, c->vt, s.B, s.S, s.H, s.KV, s.hd);
+                tmz::attention_tc_plan(&c->att_plan, c->qb, c->kb, c->vt, c->attn, s.B, s.S, s.H, s.KV, s.hd);
   }
   c->code_sw = c->ma.sw_cur;
   rc = sync_status(c);
@@ -814,8 +814,8 @@ int termezo_attention(const uint16_t* d_q, const uint16_t* d_k, const uint16_t* 
   if (hd != 64 && hd != 96 && hd != 128) return TERMEZO_EINVAL;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   tmz::AttnPlan plan;
-  if (tmz::attention_tc_supported(S, hd) && tmz::attention_tc_plan(&plan, d_q, d_k, d_vt, B, S, H, KV, hd))
-    return tmz::attention_tc_launch(plan, B, S, H, KV, hd, d_out, nullptr, st) == cudaSuccess ? TERMEZO_OK
+  if (tmz::attention_tc_supported(S, hd) && tmz::attention_tc_plan(&plan, d_q, d_k, d_vt, d_out, B, S, H, KV, hd))
+    return tmz::attention_tc_launch(plan, B, S, H, KV, hd, nullptr, st) == cudaSuccess ? TERMEZO_OK
                                                                                              : TERMEZO_ECUDA;
   tmz::launch_attention(d_q, d_k, d_vt, B, S, H, KV, hd, d_out, st);
   return cudaGetLastError() == cudaSuccess ? TERMEZO_OK : TERMEZO_ECUDA;

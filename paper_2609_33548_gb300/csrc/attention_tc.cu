@@ -150,6 +150,30 @@ __device__ __forceinline__ float2 add2(float2 a, float2 b) {
   return d;
 }
 
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
+  float2 d;
+  asm("{\n .reg .b64 x, y, z, w;\n mov.b64 x, {%2, %3};\n mov.b64 y, {%4, %5};\n mov.b64 z, {%6, %7};\n"
+      " fma.rn.f32x2 w, x, y, z;\n mov.b64 {%0, %1}, w;\n}\n"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+  return d;
+}
+
+// o / l rounded to nearest (Markstein, 1990): with y = RN(1/l), q = RN(o y)
+// and the exact residual r = o - l q (one FMA), RN(q + r y) is the correctly
+// rounded quotient.  Two lanes at a time.
+__device__ __forceinline__ float2 div2(float2 o, float2 l2, float2 y2) {
+  const float2 q = mul2(o, y2);
+  const float2 r = fma2(make_float2(-q.x, -q.y), l2, o);
+  return fma2(r, y2, q);
+}
+
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, uint32_t src, int x, int y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"((uint64_t)map),
+               "r"(src), "r"(x), "r"(y)
+               : "memory");
+}
+
 // Keys c > row of the diagonal block are outside the causal window: their
 // accumulator becomes -inf, which the maximum ignores and exp maps to 0.
 __device__ __forceinline__ void causal_mask(uint32_t* sv, int row) {
@@ -178,8 +202,8 @@ __device__ __forceinline__ bool mbar_wait_warp(uint32_t bar, uint32_t parity) {
 template <int HD>
 __global__ void __launch_bounds__(ATT_THREADS, 1)
     k_attention_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                   const __grid_constant__ CUtensorMap tmV, int B, int S, int H, int KV, float scale,
-                   float* __restrict__ out, unsigned* err) {
+                   const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmO, int B, int S,
+                   int H, int KV, float scale, unsigned* err) {
   using L = AttTc<HD>;
   constexpr int NS = L::NS;
   extern __shared__ uint8_t smem_raw[];
@@ -324,6 +348,7 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
         if (ok && (ok = take(slot))) {  // pass 2
           ok = mma_s(0, slot) && (nb < 1 || mma_s(1, slot));
           release(slot);
+          if (na == 1) mma_commit(q_empty);  // the last MMA that reads Q
         }
         for (int j = 0; j < na && ok; ++j) {
           if (j + 1 < na) {
@@ -331,6 +356,7 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
             ok = mma_s(0, slot) && (j + 1 >= nb || mma_s(1, slot));
             release(slot);
             if (!ok) break;
+            if (j + 2 == na) mma_commit(q_empty);
           }
           if (!(ok = take(slot))) break;
           ok = mma_pv(0, slot, j) && (j >= nb || mma_pv(1, slot, j));
@@ -343,7 +369,6 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
           mma_commit(o_full + 8);
           ++co[1];
         }
-        mma_commit(q_empty);
       }
       // every MMA issued has completed before TMEM is released
       mma_commit(fin);
@@ -424,20 +449,46 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
       if (!(ok = mbar_wait_warp(ofull, no & 1u))) break;
       ++no;
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-      float* orow = out + ((size_t)it.b * S + qt * BQ + row) * (size_t)(H * HD) + (size_t)h * HD;
+      // O / l staged through this tile's (now idle) P buffer in the 128-byte
+      // swizzled layout; each warp writes its own 32 rows with TMA stores of
+      // 32 x 32 fp32 boxes, so no warp waits on another
+      const float2 l2 = make_float2(l, l), y2 = make_float2(__frcp_rn(l), __frcp_rn(l));
+      const int orow = it.b * S + qt * BQ + quarter * 32, ocol0 = h * HD;
+      const uint32_t wbase = sb + L::P_OFF + t * 2 * ATOM + quarter * 32 * 128;
 #pragma unroll 1
-      for (int c = 0; c < HD / 32; ++c) {
-        uint32_t ov[32];
-        tmem_ld_cols<1>(tO + 32 * c, ov);
+      for (int rd = 0; rd < HD / 64; ++rd) {
+        if (rd > 0) {
+          if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+          __syncwarp();
+        }
 #pragma unroll
-        for (int q = 0; q < 32; q += 4)
-          *reinterpret_cast<float4*>(orow + 32 * c + q) =
-              make_float4(__fdiv_rn(__uint_as_float(ov[q]), l), __fdiv_rn(__uint_as_float(ov[q + 1]), l),
-                          __fdiv_rn(__uint_as_float(ov[q + 2]), l), __fdiv_rn(__uint_as_float(ov[q + 3]), l));
+        for (int cc = 0; cc < 2; ++cc) {
+          uint32_t ov[32];
+          tmem_ld_cols<1>(tO + 64 * rd + 32 * cc, ov);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const float2 a = div2(make_float2(__uint_as_float(ov[4 * k]), __uint_as_float(ov[4 * k + 1])), l2, y2);
+            const float2 b = div2(make_float2(__uint_as_float(ov[4 * k + 2]), __uint_as_float(ov[4 * k + 3])), l2, y2);
+            *reinterpret_cast<float4*>(prow + cc * ATOM + ((k ^ (row & 7)) * 16)) = make_float4(a.x, a.y, b.x, b.y);
+          }
+        }
+        if (rd + 1 == HD / 64) {
+          asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+          arrive(ofree);
+        }
+        fence_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_2d(&tmO, wbase, ocol0 + 64 * rd, orow);
+          tma_store_2d(&tmO, wbase + ATOM, ocol0 + 64 * rd + 32, orow);
+          asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+        }
       }
-      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-      arrive(ofree);
+      // this warp's P rows are written again only after the stores have read them
+      if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+      __syncwarp();
     }
+    if (lane == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
   }
   if (!ok && err) atomicOr(err, ERR_TIMEOUT);
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -462,16 +513,17 @@ PFN_cuTensorMapEncodeTiled_v12000 att_encode_fn() {
 }
 
 bool encode_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_cols,
-               uint32_t box_rows) {
+               uint32_t box_rows, bool fp32 = false) {
   auto fn = att_encode_fn();
-  if (!fn || (cols * 2) % 16 || ((uintptr_t)base & 15)) return false;
+  const uint64_t esz = fp32 ? 4 : 2;
+  if (!fn || (cols * esz) % 16 || ((uintptr_t)base & 15)) return false;
   cuuint64_t dims[2] = {cols, rows};
-  cuuint64_t strides[1] = {cols * 2};
+  cuuint64_t strides[1] = {cols * esz};
   cuuint32_t box[2] = {box_cols, box_rows};
   cuuint32_t estr[2] = {1, 1};
-  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  return fn(map, fp32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base),
+            dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 int sm_count() {
@@ -486,7 +538,7 @@ int sm_count() {
 }
 
 template <int HD>
-cudaError_t launch_tc(const AttnPlan& p, int B, int S, int H, int KV, float* out, unsigned* err, cudaStream_t s) {
+cudaError_t launch_tc(const AttnPlan& p, int B, int S, int H, int KV, unsigned* err, cudaStream_t s) {
   static bool attr = false;
   constexpr int smem = AttTc<HD>::BYTES;
   if (!attr) {
@@ -497,7 +549,7 @@ cudaError_t launch_tc(const AttnPlan& p, int B, int S, int H, int KV, float* out
   const int G = H / KV, NQ = S / BQ;
   const long long items = (long long)B * KV * ((G * NQ + 1) / 2);
   const int grid = (int)(items < sm_count() ? items : sm_count());
-  k_attention_tc<HD><<<grid, ATT_THREADS, smem, s>>>(p.q, p.k, p.v, B, S, H, KV, 1.0f / sqrtf((float)HD), out, err);
+  k_attention_tc<HD><<<grid, ATT_THREADS, smem, s>>>(p.q, p.k, p.v, p.o, B, S, H, KV, 1.0f / sqrtf((float)HD), err);
   return cudaGetLastError();
 }
 
@@ -505,17 +557,18 @@ cudaError_t launch_tc(const AttnPlan& p, int B, int S, int H, int KV, float* out
 
 bool attention_tc_supported(int S, int hd) { return (hd == 64 || hd == 128) && S % 128 == 0; }
 
-bool attention_tc_plan(AttnPlan* p, const uint16_t* q, const uint16_t* k, const uint16_t* vt, int B, int S, int H,
-                       int KV, int hd) {
+bool attention_tc_plan(AttnPlan* p, const uint16_t* q, const uint16_t* k, const uint16_t* vt, float* out, int B,
+                       int S, int H, int KV, int hd) {
   return encode_2d(&p->q, q, (uint64_t)B * H * S, hd, 64, BQ) &&
          encode_2d(&p->k, k, (uint64_t)B * KV * S, hd, 64, BKEY) &&
-         encode_2d(&p->v, vt, (uint64_t)B * KV * hd, S, 64, hd);
+         encode_2d(&p->v, vt, (uint64_t)B * KV * hd, S, 64, hd) &&
+         encode_2d(&p->o, out, (uint64_t)B * S, (uint64_t)H * hd, 32, 32, true);
 }
 
-cudaError_t attention_tc_launch(const AttnPlan& p, int B, int S, int H, int KV, int hd, float* out, unsigned* err,
+cudaError_t attention_tc_launch(const AttnPlan& p, int B, int S, int H, int KV, int hd, unsigned* err,
                                 cudaStream_t s) {
   kernel_launches() += 1;
-  return hd == 64 ? launch_tc<64>(p, B, S, H, KV, out, err, s) : launch_tc<128>(p, B, S, H, KV, out, err, s);
+  return hd == 64 ? launch_tc<64>(p, B, S, H, KV, err, s) : launch_tc<128>(p, B, S, H, KV, err, s);
 }
 
 }  // namespace tmz

@@ -81,15 +81,15 @@ void launch_final_norm_bf16(const float* x, const float* gain, int M, int D, uin
 void launch_ce_reduce(const float2* part, int ntiles, const float* tlogit, const int32_t* target, int B, int S,
                       int V, double* tok_loss, double* per_seq, double* total, unsigned* err, cudaStream_t s);
 // tcgen05 attention (hd 64 / 128, S % 128 == 0): tensor maps of Q
-// [B*H*S, hd], K [B*KV*S, hd] and V^T [B*KV*hd, S] (bf16).
+// [B*H*S, hd], K [B*KV*S, hd] and V^T [B*KV*hd, S] (bf16) and of the
+// output [B*S, H*hd] (fp32).
 struct AttnPlan {
-  CUtensorMap q, k, v;
+  CUtensorMap q, k, v, o;
 };
 bool attention_tc_supported(int S, int hd);
-bool attention_tc_plan(AttnPlan* p, const uint16_t* q, const uint16_t* k, const uint16_t* vt, int B, int S, int H,
-                       int KV, int hd);
-cudaError_t attention_tc_launch(const AttnPlan& p, int B, int S, int H, int KV, int hd, float* out, unsigned* err,
-                                cudaStream_t s);
+bool attention_tc_plan(AttnPlan* p, const uint16_t* q, const uint16_t* k, const uint16_t* vt, float* out, int B, int S,
+                       int H, int KV, int hd);
+cudaError_t attention_tc_launch(const AttnPlan& p, int B, int S, int H, int KV, int hd, unsigned* err, cudaStream_t s);
 // Final RMSNorm + LM head over the label tokens at the last position and
 // cross-entropy (loss mode 0): per_seq[b] (fp64), total = mean (fp64).
 void launch_head_ce_last(const float* x, const float* gain, const uint16_t* head, const int32_t* targets,
