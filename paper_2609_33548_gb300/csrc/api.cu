@@ -478,10 +478,10 @@ int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspa
   if (!s.op) {
     tmz::launch_rope_tables(s.S, s.hd, c->cosb, c->sinb, st);
     const int T = s.T, D = s.D, F = s.F, hq = s.H * s.hd, hkv = s.KV * s.hd;
-    bool ok = tmz::gemm_make_plan(&c->plan_qkv, c->xq, T, D, c->wexp, hq + 2 * hkv) &&
-              tmz::gemm_make_plan(&c->plan_o, c->xq, T, hq, c->wexp, D) &&
-              tmz::gemm_make_plan(&c->plan_gu, c->xq, T, D, c->wexp, 256 * ((F + 127) / 128)) &&
-              tmz::gemm_make_plan(&c->plan_down, c->xq, T, F, c->wexp, D);
+    bool ok = tmz::gemm_make_plan(&c->plan_qkv, c->xq, T, D, c->wexp, hq + 2 * hkv, true) &&
+              tmz::gemm_make_plan(&c->plan_o, c->xq, T, hq, c->wexp, D, true) &&
+              tmz::gemm_make_plan(&c->plan_gu, c->xq, T, D, c->wexp, 256 * ((F + 127) / 128), false) &&
+              tmz::gemm_make_plan(&c->plan_down, c->xq, T, F, c->wexp, D, true);
     if (!ok) {
       delete c;
       return TERMEZO_ECUDA;
@@ -509,7 +509,7 @@ int termezo_load_params(termezo_ctx* c, const float* d_latents, const float* d_e
   c->gains = d_gains;
   c->head = d_head;
   if (!c->sh.op && c->sh.mode == 1) {
-    c->head_plan_ok = tmz::gemm_make_plan(&c->plan_head, c->hfin, c->sh.T, c->sh.D, d_head, c->sh.V);
+    c->head_plan_ok = tmz::gemm_make_plan(&c->plan_head, c->hfin, c->sh.T, c->sh.D, d_head, c->sh.V, false);
     if (!c->head_plan_ok) return TERMEZO_EINVAL;  // head must be 16-byte aligned
   }
   return TERMEZO_OK;
@@ -712,7 +712,7 @@ int termezo_bitlinear(termezo_ctx* c, int32_t proj, const uint16_t* d_x, int32_t
   tmz::launch_norm_quant_bf16(d_x, M, K, c->xq, c->deq, st);
   tmz::launch_expand_codes(c->ma.packed + c->sh.base[proj] / 16, (uint64_t)N, K, c->wexp, st);
   GemmPlan plan;
-  if (!tmz::gemm_make_plan(&plan, c->xq, M, K, c->wexp, N)) return TERMEZO_ECUDA;
+  if (!tmz::gemm_make_plan(&plan, c->xq, M, K, c->wexp, N, true)) return TERMEZO_ECUDA;
   GemmArgs a{};
   a.out = d_y;
   a.ldo = N;

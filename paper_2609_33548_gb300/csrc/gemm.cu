@@ -9,7 +9,8 @@
 // 'sm_103a'"), so this exact-integer bf16 formulation is the tensor-core
 // path.
 //
-// Structure: a persistent grid (one CTA per SM) walks 128 x BN output tiles;
+// Structure: a persistent grid (one CTA per SM) walks 128 x BN output tiles
+// (BN 256, 192, 160 or 128, picked per shape to fill the last wave);
 // warp 0 issues TMA loads of 128 x 64 (A) and BN x 64 (B) bf16 tiles with
 // 128-byte swizzle into a STAGES-deep ring; one thread of warp 1 issues
 // tcgen05.mma (M = 128, N = BN, K = 16) into one of two fp32 accumulators in
@@ -29,7 +30,6 @@ namespace {
 
 constexpr int BM = 128;
 constexpr int BK = 64;
-constexpr int STAGES = 4;
 constexpr int GEMM_THREADS = 192;
 constexpr int A_BYTES = BM * BK * 2;
 
@@ -40,14 +40,23 @@ template <int BN>
 struct GemmSmem {
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  // as many ring stages as fit next to the epilogue staging (at most 6)
+  static constexpr int FIT = (232448 - 1280 - EPI_WARPS * 32 * (EPI_LD + 1) * 4) / STAGE_BYTES;
+  static constexpr int STAGES = FIT < 6 ? FIT : 6;
   static constexpr int EPI_OFF = STAGES * STAGE_BYTES;
   static constexpr int EPI_BYTES = EPI_WARPS * 32 * (EPI_LD + 1) * 4;
   static constexpr int BAR_OFF = EPI_OFF + EPI_BYTES;
   static constexpr int BYTES = BAR_OFF + 256 + 1024;  // barriers + alignment slack
+  // tensor memory: two accumulators of BN columns in a power-of-two allocation,
+  // the second at half of it
+  static constexpr uint32_t TMEM_COLS = 2 * BN <= 256 ? 256 : 512;
+  static constexpr uint32_t ACC_STRIDE = TMEM_COLS / 2;
 };
 
-// Persistent: CTA c processes tiles c, c + gridDim.x, ... (m fastest, so the
-// CTAs running together share the B tiles and sweep A through L2).  The
+// Persistent: CTA c processes tiles c, c + gridDim.x, ...  With m fastest the
+// CTAs running together share B tiles and sweep A through L2; with n fastest
+// (an A too large for L2, a B that fits) they share A tiles, so A streams from
+// HBM once.  The
 // accumulator is double-buffered in tensor memory (2 x BN columns) so that
 // the epilogue of one tile overlaps the main loop of the next.
 template <int BN>
@@ -55,6 +64,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     k_bitlinear_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                      GemmArgs p) {
   using L = GemmSmem<BN>;
+  constexpr int STAGES = L::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   const uint32_t sbase = smem_u32(smem);
@@ -82,7 +92,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
-                 "r"(2 * BN));
+                 "r"(L::TMEM_COLS));
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
   }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -97,7 +107,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmB) : "memory");
       uint32_t it = 0;
       for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
-        const int m0 = (tile % n_mt) * BM, n0 = (tile / n_mt) * BN;
+        const int m0 = (p.n_fast ? tile / n_nt : tile % n_mt) * BM;
+        const int n0 = (p.n_fast ? tile % n_nt : tile / n_mt) * BN;
         for (int kb = 0; kb < KB; ++kb, ++it) {
           const uint32_t s = it % STAGES, use = it / STAGES;
           if (it >= (uint32_t)STAGES && !(ok = mbar_wait(bar_empty + 8 * s, (use & 1u) ^ 1u))) break;
@@ -116,7 +127,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         const uint32_t b = local & 1u, j = local >> 1;
         if (j >= 1 && !(ok = mbar_wait(bar_tempty + 8 * b, (j & 1u) ^ 1u))) break;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        const uint32_t d = tmem + b * BN;
+        const uint32_t d = tmem + b * L::ACC_STRIDE;
         for (int kb = 0; kb < KB; ++kb, ++it) {
           const uint32_t s = it % STAGES;
           if (!(ok = mbar_wait(bar_full + 8 * s, (it / STAGES) & 1u))) break;
@@ -143,11 +154,22 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     const float s0 = p.sw[0], s1 = p.sw[1], s2 = p.sw[2];
     uint32_t local = 0;
     for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++local) {
-      const int m0 = (tile % n_mt) * BM, n0 = (tile / n_mt) * BN;
+      const int m0 = (p.n_fast ? tile / n_nt : tile % n_mt) * BM;
+      const int n0 = (p.n_fast ? tile % n_nt : tile / n_mt) * BN;
       const uint32_t b = local & 1u, j = local >> 1;
       const int row0 = m0 + quarter * 32;
       const int nrows = min(32, p.M - row0);
       dqs[lane] = (lane < nrows && p.deq) ? p.deq[row0 + lane] : 0.f;
+      // residual mode: the first chunk's residual rows are loaded before the
+      // accumulator is ready, and those of chunk c + 1 while chunk c is written
+      const bool resid = p.out && p.mode && !p.relu2 && !p.lse && nrows > 0;
+      float prev[32];
+      if (resid) {
+        const int col = n0 + lane;
+#pragma unroll
+        for (int rr = 0; rr < 32; ++rr)
+          prev[rr] = (rr < nrows && col < p.N) ? p.out[(size_t)(row0 + rr) * p.ldo + col] : 0.f;
+      }
       ok = mbar_wait(bar_tfull + 8 * b, j & 1u);
       if (!ok) break;
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
@@ -158,7 +180,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         float m = -INFINITY, se = 0.f;
         for (int c = 0; c < BN / 32; ++c) {
           uint32_t r[32];
-          tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + b * BN + (uint32_t)(c * 32), r);
+          tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + b * L::ACC_STRIDE + (uint32_t)(c * 32), r);
           const int col0 = n0 + c * 32;
           float cm = -INFINITY;
 #pragma unroll
@@ -190,7 +212,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         for (int c = 0; c < BN / 64; ++c) {
           {
             uint32_t g[32], u[32];
-            const uint32_t tb = tmem + ((uint32_t)(quarter * 32) << 16) + b * BN;
+            const uint32_t tb = tmem + ((uint32_t)(quarter * 32) << 16) + b * L::ACC_STRIDE;
             tmem_ld32(tb + (uint32_t)(c * 32), g);
             tmem_ld32(tb + (uint32_t)(BN / 2 + c * 32), u);
 #pragma unroll
@@ -214,7 +236,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       for (int c = 0; c < ((p.relu2 || p.lse) ? 0 : BN / 32); ++c) {
         {
           uint32_t r[32];
-          tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + b * BN + (uint32_t)(c * 32), r);
+          tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + b * L::ACC_STRIDE + (uint32_t)(c * 32), r);
 #pragma unroll
           for (int q = 0; q < 32; ++q) stage[lane * EPI_LD + q] = __uint_as_float(r[q]);
         }
@@ -231,14 +253,18 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
             const float sw = col < p.n1 ? s0 : (col < p.n2 ? s1 : s2);
             float* o = p.out + (size_t)row0 * p.ldo + col;
             if (p.mode) {
-              float prev[32];
+              float nxt[32];
+              const int ncol = col + 32;
+              const bool more = c + 1 < BN / 32 && ncol < p.N;
 #pragma unroll
-              for (int rr = 0; rr < 32; ++rr) prev[rr] = rr < nrows ? o[(size_t)rr * p.ldo] : 0.f;
+              for (int rr = 0; rr < 32; ++rr) nxt[rr] = (more && rr < nrows) ? o[(size_t)rr * p.ldo + 32] : 0.f;
 #pragma unroll
               for (int rr = 0; rr < 32; ++rr)
                 if (rr < nrows)
                   o[(size_t)rr * p.ldo] =
                       __fadd_rn(prev[rr], __fmul_rn(__fmul_rn(stage[rr * EPI_LD + lane], dqs[rr]), sw));
+#pragma unroll
+              for (int rr = 0; rr < 32; ++rr) prev[rr] = nxt[rr];
             } else {
 #pragma unroll 8
               for (int rr = 0; rr < 32; ++rr)
@@ -258,7 +284,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   __syncthreads();
   if (warp == 1) {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(2 * BN));
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(L::TMEM_COLS));
   }
 }
 
@@ -277,7 +303,7 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 
 }  // namespace
 
-constexpr int GEMM_BN = 256;
+constexpr int GEMM_BN = 256;  // fixed for the fused gate/up and LM-head modes
 
 bool encode_bf16_kmajor(CUtensorMap* map, const void* base, uint64_t rows, uint64_t k, uint32_t box_rows) {
   auto fn = encode_fn();
@@ -292,38 +318,90 @@ bool encode_bf16_kmajor(CUtensorMap* map, const void* base, uint64_t rows, uint6
   return r == CUDA_SUCCESS;
 }
 
-bool gemm_make_plan(GemmPlan* plan, const uint16_t* a, int M, int K, const uint16_t* b, int N) {
+namespace {
+
+int sm_count() {
+  static int sms = 0;
+  if (!sms) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) !=
+                                                   cudaSuccess || sms <= 0)
+      sms = 148;
+  }
+  return sms;
+}
+
+}  // namespace
+
+int gemm_pick_bn(int M, int N, int sms) {
+  // A persistent CTA's time is (tiles it walks) x (one tile's main loop, ~BN);
+  // smaller tiles fill the last wave better but re-read A more often.
+  static const int bns[4] = {256, 192, 160, 128};
+  static const double cost_per_col[4] = {1.0, 1.03, 1.05, 1.08};
+  const long long m_tiles = (M + BM - 1) / BM;
+  int best = 256;
+  double best_cost = 0;
+  for (int i = 0; i < 4; ++i) {
+    const long long tiles = m_tiles * ((N + bns[i] - 1) / bns[i]);
+    const long long waves = (tiles + sms - 1) / sms;
+    const double cost = (double)waves * bns[i] * cost_per_col[i];
+    if (i == 0 || cost < best_cost * 0.999) {
+      best = bns[i];
+      best_cost = cost;
+    }
+  }
+  return best;
+}
+
+bool gemm_make_plan(GemmPlan* plan, const uint16_t* a, int M, int K, const uint16_t* b, int N, bool any_bn) {
   plan->M = M;
   plan->N = N;
   plan->K = K;
+  plan->bn = any_bn ? gemm_pick_bn(M, N, sm_count()) : GEMM_BN;
+  // n fastest when A (M x K bf16) is too large to stay in L2 and B is not
+  const double a_bytes = 2.0 * M * K, b_bytes = 2.0 * N * K;
+  plan->n_fast = (a_bytes > 64e6 && b_bytes < a_bytes) ? 1 : 0;
   return encode_bf16_kmajor(&plan->a, a, (uint64_t)M, (uint64_t)K, BM) &&
-         encode_bf16_kmajor(&plan->b, b, (uint64_t)N, (uint64_t)K, GEMM_BN);
+         encode_bf16_kmajor(&plan->b, b, (uint64_t)N, (uint64_t)K, (uint32_t)plan->bn);
 }
 
 int gemm_col_tiles(int N) { return (N + GEMM_BN - 1) / GEMM_BN; }
 
-cudaError_t gemm_launch(const GemmPlan& plan, GemmArgs args, cudaStream_t stream) {
+namespace {
+
+template <int BN>
+cudaError_t launch_bn(const GemmPlan& plan, const GemmArgs& args, cudaStream_t stream) {
   static bool attr_set = false;
-  constexpr int smem = GemmSmem<GEMM_BN>::BYTES;
+  constexpr int smem = GemmSmem<BN>::BYTES;
+  static_assert(smem <= 232448, "shared memory");
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(k_bitlinear_gemm<GEMM_BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaError_t e = cudaFuncSetAttribute(k_bitlinear_gemm<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  static int sms = 0;
-  if (!sms) {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) sms = 148;
-  }
+  const int sms = sm_count();
+  const int tiles = ((plan.N + BN - 1) / BN) * ((plan.M + BM - 1) / BM);
+  dim3 grid(tiles < sms ? tiles : sms);
+  k_bitlinear_gemm<BN><<<grid, GEMM_THREADS, smem, stream>>>(plan.a, plan.b, args);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t gemm_launch(const GemmPlan& plan, GemmArgs args, cudaStream_t stream) {
   args.M = plan.M;
   args.N = plan.N;
   args.K = plan.K;
-  const int tiles = ((plan.N + GEMM_BN - 1) / GEMM_BN) * ((plan.M + BM - 1) / BM);
-  dim3 grid(tiles < sms ? tiles : sms);
+  args.n_fast = plan.n_fast;
+  if ((args.relu2 || args.lse) && plan.bn != GEMM_BN) return cudaErrorInvalidValue;
   ++kernel_launches();
-  k_bitlinear_gemm<GEMM_BN><<<grid, GEMM_THREADS, smem, stream>>>(plan.a, plan.b, args);
-  return cudaGetLastError();
+  switch (plan.bn) {
+    case 256: return launch_bn<256>(plan, args, stream);
+    case 192: return launch_bn<192>(plan, args, stream);
+    case 160: return launch_bn<160>(plan, args, stream);
+    case 128: return launch_bn<128>(plan, args, stream);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 }  // namespace tmz

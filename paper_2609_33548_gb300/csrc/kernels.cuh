@@ -34,6 +34,7 @@ struct GemmArgs {
   float* tlogit;
   const int32_t* target;
   unsigned* err;        // device error word
+  int n_fast;           // filled from the plan: tile order walks n fastest
 };
 
 // Column tiles of the GEMM (the stride of GemmArgs::part).
@@ -41,10 +42,14 @@ int gemm_col_tiles(int N);
 
 struct GemmPlan {
   CUtensorMap a, b;
-  int M, N, K;
+  int M, N, K, bn;  // bn: output tile width (columns of B per tile)
+  int n_fast;       // tile order: n fastest (A streamed once, B kept in L2)
 };
 
-bool gemm_make_plan(GemmPlan* plan, const uint16_t* a, int M, int K, const uint16_t* b, int N);
+// any_bn: the plan may use any tile width (store / residual-add epilogues);
+// otherwise 256 (fused gate/up and LM-head epilogues).
+bool gemm_make_plan(GemmPlan* plan, const uint16_t* a, int M, int K, const uint16_t* b, int N, bool any_bn);
+int gemm_pick_bn(int M, int N, int sms);
 cudaError_t gemm_launch(const GemmPlan& plan, GemmArgs args, cudaStream_t stream);
 
 // ------------------------------------------------------------ forward ----
