@@ -342,6 +342,8 @@ def run_op(args):
     from paper_2609_33548_gb300 import termezo as tz
 
     N, K, M = synth.BITLINEAR_OP["N"], synth.BITLINEAR_OP["K"], synth.BITLINEAR_OP["M"]
+    if args.op_shape:
+        N, K, M = (int(v) for v in args.op_shape.split(","))
     density = args.op_density
     dev = torch.device("cuda", 0)
     w = synth.op_latents(N, K, device=dev).reshape(-1)
@@ -443,6 +445,7 @@ def main():
     ap.add_argument("--impl", choices=("mine", "reference"), default="mine")
     ap.add_argument("--workload", choices=sorted(WORKLOADS) + ["op"] + sorted(ATTN_WORKLOADS), default="2b")
     ap.add_argument("--op-density", type=float, default=0.01)
+    ap.add_argument("--op-shape", default="", help="N,K,M of the op workload's projection (default 6912,2560,2048)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:

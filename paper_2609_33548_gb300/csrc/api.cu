@@ -486,6 +486,10 @@ int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspa
       delete c;
       return TERMEZO_ECUDA;
     }
+    // TMA output maps (a layout that does not allow one keeps the plain stores)
+    tmz::gemm_plan_output(&c->plan_qkv, c->qkv, hq + 2 * hkv);
+    tmz::gemm_plan_output(&c->plan_o, c->x, D);
+    tmz::gemm_plan_output(&c->plan_down, c->x, D);
     c->att_tc = tmz::attention_tc_supported(s.S, s.hd) &&
                 tmz::attention_tc_plan(&c->att_plan, c->qb, c->kb, c->vt, c->attn, s.B, s.S, s.H, s.KV, s.hd);
   }
@@ -713,6 +717,7 @@ int termezo_bitlinear(termezo_ctx* c, int32_t proj, const uint16_t* d_x, int32_t
   tmz::launch_expand_codes(c->ma.packed + c->sh.base[proj] / 16, (uint64_t)N, K, c->wexp, st);
   GemmPlan plan;
   if (!tmz::gemm_make_plan(&plan, c->xq, M, K, c->wexp, N, true)) return TERMEZO_ECUDA;
+  if (d_y) tmz::gemm_plan_output(&plan, d_y, N);
   GemmArgs a{};
   a.out = d_y;
   a.ldo = N;

@@ -41,10 +41,13 @@ struct GemmSmem {
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   // as many ring stages as fit next to the epilogue staging (at most 6)
-  static constexpr int FIT = (232448 - 1280 - EPI_WARPS * 32 * (EPI_LD + 1) * 4) / STAGE_BYTES;
+  // epilogue staging: per warp two 32 x 32 fp32 tiles (128-byte swizzle) for
+  // the TMA output path, or one 32 x 33 transpose block for the others
+  static constexpr int EPI_BYTES = EPI_WARPS * 2 * 4096;
+  static_assert(EPI_BYTES >= EPI_WARPS * 32 * (EPI_LD + 1) * 4, "staging");
+  static constexpr int FIT = (232448 - 1280 - EPI_BYTES) / STAGE_BYTES;
   static constexpr int STAGES = FIT < 6 ? FIT : 6;
   static constexpr int EPI_OFF = STAGES * STAGE_BYTES;
-  static constexpr int EPI_BYTES = EPI_WARPS * 32 * (EPI_LD + 1) * 4;
   static constexpr int BAR_OFF = EPI_OFF + EPI_BYTES;
   static constexpr int BYTES = BAR_OFF + 256 + 1024;  // barriers + alignment slack
   // tensor memory: two accumulators of BN columns in a power-of-two allocation,
@@ -62,7 +65,7 @@ struct GemmSmem {
 template <int BN>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     k_bitlinear_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                     GemmArgs p) {
+                     const __grid_constant__ CUtensorMap tmO, GemmArgs p) {
   using L = GemmSmem<BN>;
   constexpr int STAGES = L::STAGES;
   extern __shared__ uint8_t smem_raw[];
@@ -150,6 +153,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     // every store (and residual load) is one coalesced 128-byte row segment.
     const int quarter = warp & 3;
     float* stage = reinterpret_cast<float*>(smem + L::EPI_OFF) + (warp - 2) * 32 * (EPI_LD + 1);
+    // TMA output path: this warp's two swizzled 32 x 32 staging tiles
+    uint8_t* otile = smem + L::EPI_OFF + (warp - 2) * 2 * 4096;
+    uint32_t n_out_tiles = 0;
     float* dqs = stage + 32 * EPI_LD;  // the 32 rows' activation scales
     const float s0 = p.sw[0], s1 = p.sw[1], s2 = p.sw[2];
     uint32_t local = 0;
@@ -159,10 +165,15 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       const uint32_t b = local & 1u, j = local >> 1;
       const int row0 = m0 + quarter * 32;
       const int nrows = min(32, p.M - row0);
-      dqs[lane] = (lane < nrows && p.deq) ? p.deq[row0 + lane] : 0.f;
-      // residual mode: the first chunk's residual rows are loaded before the
-      // accumulator is ready, and those of chunk c + 1 while chunk c is written
-      const bool resid = p.out && p.mode && !p.relu2 && !p.lse && nrows > 0;
+      const bool tma_path = p.tma_out && !p.relu2 && !p.lse;
+      const float dq_row = (lane < nrows && p.deq) ? p.deq[row0 + lane] : 0.f;
+      // dqs shares shared memory with the TMA staging tiles: only the
+      // transposing paths use it
+      if (!tma_path) dqs[lane] = dq_row;
+      // residual mode without the TMA path: the first chunk's residual rows are
+      // loaded before the accumulator is ready, those of chunk c + 1 while
+      // chunk c is written
+      const bool resid = p.out && p.mode && !p.tma_out && !p.relu2 && !p.lse && nrows > 0;
       float prev[32];
       if (resid) {
         const int col = n0 + lane;
@@ -233,7 +244,60 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           __syncwarp();
         }
       }
-      for (int c = 0; c < ((p.relu2 || p.lse) ? 0 : BN / 32); ++c) {
+      if (tma_path) {
+        // lane = row: y = acc (a/127)[row] s_w[col] written by this warp as
+        // 32 x 32 tiles through shared memory with a TMA store, or added into
+        // the residual stream with a TMA reduce-add (one fp32 add, rounded to
+        // nearest, per element: the same value as out + y)
+        const float dq = dq_row;
+        const int row = row0 + lane;
+        for (int c = 0; c < BN / 32; ++c) {
+          const int col0 = n0 + c * 32;
+          if (col0 >= p.N) break;
+          uint32_t r[32];
+          tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + b * L::ACC_STRIDE + (uint32_t)(c * 32), r);
+          if (p.acc_out && lane < nrows) {
+#pragma unroll
+            for (int q = 0; q < 32; ++q)
+              if (col0 + q < p.N) p.acc_out[(size_t)row * p.N + col0 + q] = __float2int_rn(__uint_as_float(r[q]));
+          }
+          uint8_t* ot = otile + (n_out_tiles & 1u) * 4096;
+          if (n_out_tiles >= 2) {
+            if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+            __syncwarp();
+          }
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            float v[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const int col = col0 + 4 * k + e;
+              const float sw = col < p.n1 ? s0 : (col < p.n2 ? s1 : s2);
+              v[e] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * k + e]), dq), sw);
+            }
+            *reinterpret_cast<float4*>(ot + lane * 128 + ((k ^ (lane & 7)) * 16)) = make_float4(v[0], v[1], v[2], v[3]);
+          }
+          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+          __syncwarp();
+          if (lane == 0) {
+            const uint32_t src = smem_u32(ot);
+            if (p.mode)
+              asm volatile(
+                  "cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                      (uint64_t)&tmO),
+                  "r"(src), "r"(col0), "r"(row0)
+                  : "memory");
+            else
+              asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                               (uint64_t)&tmO),
+                           "r"(src), "r"(col0), "r"(row0)
+                           : "memory");
+            asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+          }
+          ++n_out_tiles;
+        }
+      }
+      for (int c = 0; c < ((p.relu2 || p.lse || p.tma_out) ? 0 : BN / 32); ++c) {
         {
           uint32_t r[32];
           tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + b * L::ACC_STRIDE + (uint32_t)(c * 32), r);
@@ -278,6 +342,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(bar_tempty + 8 * b);
     }
+    // the TMA writes complete before the kernel does
+    if (lane == 0 && n_out_tiles) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
   }
   if (!ok && p.err) atomicOr(p.err, ERR_TIMEOUT);
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -334,10 +400,13 @@ int sm_count() {
 }  // namespace
 
 int gemm_pick_bn(int M, int N, int sms) {
-  // A persistent CTA's time is (tiles it walks) x (one tile's main loop, ~BN);
-  // smaller tiles fill the last wave better but re-read A more often.
+  // A persistent CTA's time is (tiles it walks) x (one tile's main loop, ~BN).
+  // Smaller tiles fill the last wave better, but each k-step then holds less
+  // MMA work to cover the load latency of the ring: measured on GB300 at
+  // K 2560-6912, a 160-column tile costs ~1.4x per column what a 256-column
+  // one does.
   static const int bns[4] = {256, 192, 160, 128};
-  static const double cost_per_col[4] = {1.0, 1.03, 1.05, 1.08};
+  static const double cost_per_col[4] = {1.0, 1.2, 1.4, 1.6};
   const long long m_tiles = (M + BM - 1) / BM;
   int best = 256;
   double best_cost = 0;
@@ -358,6 +427,8 @@ bool gemm_make_plan(GemmPlan* plan, const uint16_t* a, int M, int K, const uint1
   plan->N = N;
   plan->K = K;
   plan->bn = any_bn ? gemm_pick_bn(M, N, sm_count()) : GEMM_BN;
+  plan->o_ptr = nullptr;
+  plan->o_ld = 0;
   // n fastest when A (M x K bf16) is too large to stay in L2 and B is not
   const double a_bytes = 2.0 * M * K, b_bytes = 2.0 * N * K;
   plan->n_fast = (a_bytes > 64e6 && b_bytes < a_bytes) ? 1 : 0;
@@ -366,6 +437,23 @@ bool gemm_make_plan(GemmPlan* plan, const uint16_t* a, int M, int K, const uint1
 }
 
 int gemm_col_tiles(int N) { return (N + GEMM_BN - 1) / GEMM_BN; }
+
+bool gemm_plan_output(GemmPlan* plan, float* out, int ldo) {
+  plan->o_ptr = nullptr;
+  auto fn = encode_fn();
+  if (!fn || !out || ldo < plan->N || ((uintptr_t)out & 15) || ((size_t)ldo * 4) % 16) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)plan->N, (cuuint64_t)plan->M};
+  cuuint64_t strides[1] = {(cuuint64_t)ldo * 4};
+  cuuint32_t box[2] = {32, 32};
+  cuuint32_t estr[2] = {1, 1};
+  if (fn(&plan->o, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, out, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+         CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) !=
+      CUDA_SUCCESS)
+    return false;
+  plan->o_ptr = out;
+  plan->o_ld = ldo;
+  return true;
+}
 
 namespace {
 
@@ -382,7 +470,7 @@ cudaError_t launch_bn(const GemmPlan& plan, const GemmArgs& args, cudaStream_t s
   const int sms = sm_count();
   const int tiles = ((plan.N + BN - 1) / BN) * ((plan.M + BM - 1) / BM);
   dim3 grid(tiles < sms ? tiles : sms);
-  k_bitlinear_gemm<BN><<<grid, GEMM_THREADS, smem, stream>>>(plan.a, plan.b, args);
+  k_bitlinear_gemm<BN><<<grid, GEMM_THREADS, smem, stream>>>(plan.a, plan.b, plan.o, args);
   return cudaGetLastError();
 }
 
@@ -393,6 +481,7 @@ cudaError_t gemm_launch(const GemmPlan& plan, GemmArgs args, cudaStream_t stream
   args.N = plan.N;
   args.K = plan.K;
   args.n_fast = plan.n_fast;
+  args.tma_out = (plan.o_ptr && args.out == plan.o_ptr && args.ldo == plan.o_ld && !args.relu2 && !args.lse) ? 1 : 0;
   if ((args.relu2 || args.lse) && plan.bn != GEMM_BN) return cudaErrorInvalidValue;
   ++kernel_launches();
   switch (plan.bn) {

@@ -35,6 +35,7 @@ struct GemmArgs {
   const int32_t* target;
   unsigned* err;        // device error word
   int n_fast;           // filled from the plan: tile order walks n fastest
+  int tma_out;          // filled at launch: out / ldo match the plan's output map
 };
 
 // Column tiles of the GEMM (the stride of GemmArgs::part).
@@ -44,7 +45,15 @@ struct GemmPlan {
   CUtensorMap a, b;
   int M, N, K, bn;  // bn: output tile width (columns of B per tile)
   int n_fast;       // tile order: n fastest (A streamed once, B kept in L2)
+  CUtensorMap o;    // fp32 output [M, N] (row stride o_ld): TMA store / reduce-add
+  float* o_ptr;     // the output the map was made for (null: none)
+  int o_ld;
 };
+
+// Records a TMA map of the fp32 output out [M, ldo] in the plan; launches
+// whose GemmArgs::out / ldo match it write through TMA (store, or reduce-add
+// in residual mode).  False (and no map) when the layout does not allow it.
+bool gemm_plan_output(GemmPlan* plan, float* out, int ldo);
 
 // any_bn: the plan may use any tile width (store / residual-add epilogues);
 // otherwise 256 (fused gate/up and LM-head epilogues).
