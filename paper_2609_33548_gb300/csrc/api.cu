@@ -331,11 +331,23 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
     a.n1 = hq;
     a.n2 = hq + hkv;
     a.err = c->ma.err;
+    if (c->plan_qkv.rope) {
+      a.rope = 1;
+      a.cosb = c->cosb;
+      a.sinb = c->sinb;
+      a.vt = c->vt;
+      a.S = s.S;
+      a.H = s.H;
+      a.KV = s.KV;
+      a.hd = s.hd;
+    }
     {
       ProfScope ps(c, 0, gemm_flops(c->plan_qkv));
       if (tmz::gemm_launch(c->plan_qkv, a, st) != cudaSuccess) return TERMEZO_ECUDA;
     }
-    tmz::launch_rope_pack(c->qkv, c->cosb, c->sinb, s.B, s.S, s.H, s.KV, s.hd, c->qb, c->kb, c->vt, st);
+    if (!c->plan_qkv.rope)
+      tmz::launch_rope_pack(c->qkv, c->cosb, c->sinb, s.B, s.S, s.H, s.KV, s.hd, c->qb, c->kb, c->vt, st);
+    a.rope = 0;  // the remaining projections of the layer reuse a
     {
       ProfScope ps(c, 1, 4.0 * s.B * s.H * (double)s.hd * (0.5 * s.S * (s.S + 1.0)));
       if (c->att_tc) {
@@ -478,7 +490,8 @@ int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspa
   if (!s.op) {
     tmz::launch_rope_tables(s.S, s.hd, c->cosb, c->sinb, st);
     const int T = s.T, D = s.D, F = s.F, hq = s.H * s.hd, hkv = s.KV * s.hd;
-    bool ok = tmz::gemm_make_plan(&c->plan_qkv, c->xq, T, D, c->wexp, hq + 2 * hkv, true) &&
+    const bool rope_fused = (s.hd == 64 || s.hd == 128) && s.S % 32 == 0;
+    bool ok = tmz::gemm_make_plan(&c->plan_qkv, c->xq, T, D, c->wexp, hq + 2 * hkv, !rope_fused) &&
               tmz::gemm_make_plan(&c->plan_o, c->xq, T, hq, c->wexp, D, true) &&
               tmz::gemm_make_plan(&c->plan_gu, c->xq, T, D, c->wexp, 256 * ((F + 127) / 128), false) &&
               tmz::gemm_make_plan(&c->plan_down, c->xq, T, F, c->wexp, D, true);
@@ -487,7 +500,10 @@ int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspa
       return TERMEZO_ECUDA;
     }
     // TMA output maps (a layout that does not allow one keeps the plain stores)
-    tmz::gemm_plan_output(&c->plan_qkv, c->qkv, hq + 2 * hkv);
+    // q, k, v written by the QKV GEMM's epilogue (RoPE fused) where the head
+    // layout allows it
+    if (!(rope_fused && tmz::gemm_plan_rope(&c->plan_qkv, c->qb, c->kb, s.B, s.S, s.H, s.KV, s.hd)))
+      tmz::gemm_plan_output(&c->plan_qkv, c->qkv, hq + 2 * hkv);
     tmz::gemm_plan_output(&c->plan_o, c->x, D);
     tmz::gemm_plan_output(&c->plan_down, c->x, D);
     c->att_tc = tmz::attention_tc_supported(s.S, s.hd) &&

@@ -18,6 +18,7 @@
 // transpose it through shared memory and store coalesced rows of
 // y = acc * (a/127)[m] * s_w[n] (or add them into the residual stream).
 #include <cuda.h>
+#include <cuda_bf16.h>
 #include <cudaTypedefs.h>
 
 #include "common.cuh"
@@ -65,7 +66,8 @@ struct GemmSmem {
 template <int BN>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     k_bitlinear_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                     const __grid_constant__ CUtensorMap tmO, GemmArgs p) {
+                     const __grid_constant__ CUtensorMap tmO, const __grid_constant__ CUtensorMap tmQ,
+                     const __grid_constant__ CUtensorMap tmK, GemmArgs p) {
   using L = GemmSmem<BN>;
   constexpr int STAGES = L::STAGES;
   extern __shared__ uint8_t smem_raw[];
@@ -165,11 +167,11 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       const uint32_t b = local & 1u, j = local >> 1;
       const int row0 = m0 + quarter * 32;
       const int nrows = min(32, p.M - row0);
-      const bool tma_path = p.tma_out && !p.relu2 && !p.lse;
+      const bool tma_path = p.tma_out && !p.relu2 && !p.lse && !p.rope;
       const float dq_row = (lane < nrows && p.deq) ? p.deq[row0 + lane] : 0.f;
       // dqs shares shared memory with the TMA staging tiles: only the
       // transposing paths use it
-      if (!tma_path) dqs[lane] = dq_row;
+      if (!tma_path && !p.rope) dqs[lane] = dq_row;
       // residual mode without the TMA path: the first chunk's residual rows are
       // loaded before the accumulator is ready, those of chunk c + 1 while
       // chunk c is written
@@ -244,6 +246,92 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           __syncwarp();
         }
       }
+      if (p.rope) {
+        // lane = row = token at position pos of sequence sb; the tile's
+        // columns are whole heads of hd (q heads, then k, then v)
+        const float dq = dq_row;
+        const int sb = row0 / p.S, pos0 = row0 - sb * p.S, pos = pos0 + lane;
+        const int half = p.hd >> 1;
+        for (int hb = 0; hb < BN / p.hd; ++hb) {
+          const int col0 = n0 + hb * p.hd;
+          if (col0 >= p.N) break;
+          const int head = col0 / p.hd;
+          const uint32_t tb = tmem + ((uint32_t)(quarter * 32) << 16) + b * L::ACC_STRIDE + (uint32_t)(hb * p.hd);
+          if (head >= p.H + p.KV) {
+            // v: bf16 into vt[b, kvh, d, pos]; the warp's 32 positions of
+            // one d are 64 contiguous bytes
+            uint16_t* vcol = p.vt + ((size_t)(sb * p.KV + head - p.H - p.KV) * p.hd) * p.S + pos;
+            for (int c = 0; c < p.hd / 32; ++c) {
+              uint32_t r[32];
+              tmem_ld32(tb + (uint32_t)(c * 32), r);
+#pragma unroll
+              for (int q = 0; q < 32; ++q) {
+                const __nv_bfloat16 v = __float2bfloat16_rn(__fmul_rn(__fmul_rn(__uint_as_float(r[q]), dq), s2));
+                vcol[(size_t)(c * 32 + q) * p.S] = *reinterpret_cast<const uint16_t*>(&v);
+              }
+            }
+            continue;
+          }
+          const bool isq = head < p.H;
+          const float sw = isq ? s0 : s1;
+          // both staging tiles are rewritten: the previous head's stores must
+          // have read them
+          if (n_out_tiles) {
+            if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+            __syncwarp();
+          }
+          for (int c = 0; c < half / 32; ++c) {
+            uint32_t r1[32], r2[32];
+            tmem_ld32(tb + (uint32_t)(c * 32), r1);
+            tmem_ld32(tb + (uint32_t)(half + c * 32), r2);
+            const float4* cr = reinterpret_cast<const float4*>(p.cosb + (size_t)pos * half + c * 32);
+            const float4* sr = reinterpret_cast<const float4*>(p.sinb + (size_t)pos * half + c * 32);
+            uint32_t w1[16], w2[16];
+#pragma unroll
+            for (int g = 0; g < 8; ++g) {
+              const float4 cv = cr[g], sv = sr[g];
+              const float cs[4] = {cv.x, cv.y, cv.z, cv.w}, sn[4] = {sv.x, sv.y, sv.z, sv.w};
+              float o1[4], o2[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const float x1 = __fmul_rn(__fmul_rn(__uint_as_float(r1[4 * g + e]), dq), sw);
+                const float x2 = __fmul_rn(__fmul_rn(__uint_as_float(r2[4 * g + e]), dq), sw);
+                o1[e] = __fsub_rn(__fmul_rn(x1, cs[e]), __fmul_rn(x2, sn[e]));
+                o2[e] = __fadd_rn(__fmul_rn(x2, cs[e]), __fmul_rn(x1, sn[e]));
+              }
+              __nv_bfloat162 a0 = __floats2bfloat162_rn(o1[0], o1[1]), a1 = __floats2bfloat162_rn(o1[2], o1[3]);
+              __nv_bfloat162 c0 = __floats2bfloat162_rn(o2[0], o2[1]), c1 = __floats2bfloat162_rn(o2[2], o2[3]);
+              w1[2 * g] = *reinterpret_cast<uint32_t*>(&a0);
+              w1[2 * g + 1] = *reinterpret_cast<uint32_t*>(&a1);
+              w2[2 * g] = *reinterpret_cast<uint32_t*>(&c0);
+              w2[2 * g + 1] = *reinterpret_cast<uint32_t*>(&c1);
+            }
+            // bf16 columns 32c.. (first half) and half + 32c.. (second half)
+            // of the head -> 64-column swizzled tiles
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+              const int c1c = c * 32 + 8 * t, c2c = half + c * 32 + 8 * t;
+              *reinterpret_cast<uint4*>(otile + (c1c >> 6) * 4096 + lane * 128 + ((((c1c & 63) >> 3) ^ (lane & 7)) * 16)) =
+                  make_uint4(w1[4 * t], w1[4 * t + 1], w1[4 * t + 2], w1[4 * t + 3]);
+              *reinterpret_cast<uint4*>(otile + (c2c >> 6) * 4096 + lane * 128 + ((((c2c & 63) >> 3) ^ (lane & 7)) * 16)) =
+                  make_uint4(w2[4 * t], w2[4 * t + 1], w2[4 * t + 2], w2[4 * t + 3]);
+            }
+          }
+          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+          __syncwarp();
+          if (lane == 0) {
+            const int hidx = isq ? head : head - p.H;
+            const int yrow = (sb * (isq ? p.H : p.KV) + hidx) * p.S + pos0;
+            for (int bx = 0; bx < p.hd / 64; ++bx)
+              asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                               (uint64_t)(isq ? &tmQ : &tmK)),
+                           "r"(smem_u32(otile + bx * 4096)), "r"(bx * 64), "r"(yrow)
+                           : "memory");
+            asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+          }
+          ++n_out_tiles;
+        }
+      }
       if (tma_path) {
         // lane = row: y = acc (a/127)[row] s_w[col] written by this warp as
         // 32 x 32 tiles through shared memory with a TMA store, or added into
@@ -297,7 +385,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           ++n_out_tiles;
         }
       }
-      for (int c = 0; c < ((p.relu2 || p.lse || p.tma_out) ? 0 : BN / 32); ++c) {
+      for (int c = 0; c < ((p.relu2 || p.lse || p.tma_out || p.rope) ? 0 : BN / 32); ++c) {
         {
           uint32_t r[32];
           tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + b * L::ACC_STRIDE + (uint32_t)(c * 32), r);
@@ -429,6 +517,7 @@ bool gemm_make_plan(GemmPlan* plan, const uint16_t* a, int M, int K, const uint1
   plan->bn = any_bn ? gemm_pick_bn(M, N, sm_count()) : GEMM_BN;
   plan->o_ptr = nullptr;
   plan->o_ld = 0;
+  plan->rope = 0;
   // n fastest when A (M x K bf16) is too large to stay in L2 and B is not
   const double a_bytes = 2.0 * M * K, b_bytes = 2.0 * N * K;
   plan->n_fast = (a_bytes > 64e6 && b_bytes < a_bytes) ? 1 : 0;
@@ -437,6 +526,29 @@ bool gemm_make_plan(GemmPlan* plan, const uint16_t* a, int M, int K, const uint1
 }
 
 int gemm_col_tiles(int N) { return (N + GEMM_BN - 1) / GEMM_BN; }
+
+bool gemm_plan_rope(GemmPlan* plan, uint16_t* q, uint16_t* k, int B, int S, int H, int KV, int hd) {
+  if ((hd != 64 && hd != 128) || S % 32 || plan->bn % hd || (long long)B * S != plan->M ||
+      plan->N != (H + 2 * KV) * hd)
+    return false;
+  CUtensorMap mq, mk;
+  auto enc = [&](CUtensorMap* m, uint16_t* base, uint64_t rows) {
+    auto fn = encode_fn();
+    if (!fn || ((uintptr_t)base & 15)) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)hd, rows};
+    cuuint64_t strides[1] = {(cuuint64_t)hd * 2};
+    cuuint32_t box[2] = {64, 32};
+    cuuint32_t estr[2] = {1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+              CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  };
+  if (!enc(&mq, q, (uint64_t)B * H * S) || !enc(&mk, k, (uint64_t)B * KV * S)) return false;
+  plan->q = mq;
+  plan->k = mk;
+  plan->rope = 1;
+  return true;
+}
 
 bool gemm_plan_output(GemmPlan* plan, float* out, int ldo) {
   plan->o_ptr = nullptr;
@@ -470,7 +582,7 @@ cudaError_t launch_bn(const GemmPlan& plan, const GemmArgs& args, cudaStream_t s
   const int sms = sm_count();
   const int tiles = ((plan.N + BN - 1) / BN) * ((plan.M + BM - 1) / BM);
   dim3 grid(tiles < sms ? tiles : sms);
-  k_bitlinear_gemm<BN><<<grid, GEMM_THREADS, smem, stream>>>(plan.a, plan.b, plan.o, args);
+  k_bitlinear_gemm<BN><<<grid, GEMM_THREADS, smem, stream>>>(plan.a, plan.b, plan.o, plan.q, plan.k, args);
   return cudaGetLastError();
 }
 
@@ -481,6 +593,7 @@ cudaError_t gemm_launch(const GemmPlan& plan, GemmArgs args, cudaStream_t stream
   args.N = plan.N;
   args.K = plan.K;
   args.n_fast = plan.n_fast;
+  if (args.rope && (!plan.rope || plan.bn % args.hd)) return cudaErrorInvalidValue;
   args.tma_out = (plan.o_ptr && args.out == plan.o_ptr && args.ldo == plan.o_ld && !args.relu2 && !args.lse) ? 1 : 0;
   if ((args.relu2 || args.lse) && plan.bn != GEMM_BN) return cudaErrorInvalidValue;
   ++kernel_launches();

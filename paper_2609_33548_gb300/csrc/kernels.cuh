@@ -36,6 +36,16 @@ struct GemmArgs {
   unsigned* err;        // device error word
   int n_fast;           // filled from the plan: tile order walks n fastest
   int tma_out;          // filled at launch: out / ldo match the plan's output map
+  // fused RoPE + pack of the attention projections (q, k, v heads of hd
+  // columns, the plan made by gemm_plan_rope): q, k rotated at position
+  // (row mod S) with the cos / sin tables [S, hd/2], rounded to bf16 and
+  // stored as [B, H, S, hd] / [B, KV, S, hd]; v rounded to bf16 into vt
+  // [B, KV, hd, S].  out is not written.
+  int rope;
+  const float* cosb;
+  const float* sinb;
+  uint16_t* vt;
+  int S, H, KV, hd;
 };
 
 // Column tiles of the GEMM (the stride of GemmArgs::part).
@@ -48,7 +58,14 @@ struct GemmPlan {
   CUtensorMap o;    // fp32 output [M, N] (row stride o_ld): TMA store / reduce-add
   float* o_ptr;     // the output the map was made for (null: none)
   int o_ld;
+  CUtensorMap q, k;  // fused RoPE outputs (gemm_plan_rope)
+  int rope;
 };
+
+// Tensor maps of the bf16 Q [B*H*S, hd] and K [B*KV*S, hd] for the fused
+// RoPE epilogue.  Needs a plan with 256-column tiles, hd 64 or 128, S a
+// multiple of 32 and M = B*S; false (plan unchanged) otherwise.
+bool gemm_plan_rope(GemmPlan* plan, uint16_t* q, uint16_t* k, int B, int S, int H, int KV, int hd);
 
 // Records a TMA map of the fp32 output out [M, ldo] in the plan; launches
 // whose GemmArgs::out / ldo match it write through TMA (store, or reduce-add
