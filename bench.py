@@ -45,6 +45,22 @@ WORKLOADS = {
     "tiny": (synth.TINY, 0.01),
 }
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+# DRAM bytes (read + write) per k_bitlinear_gemm launch, the mean over the 240
+# GEMM launches of one 2B-shaped step, from the one-pass ncu launch list in
+# profiles/step_2b_launch_list.md.  It describes the kernel source with this
+# SHA-1 only; any other source, or another workload, reports null.
+GEMM_TRAFFIC = {"workload": "2b", "source": "paper_2609_33548_gb300/csrc/gemm.cu",
+                "sha1": "f1f8230b074097b4cba674b0d28eb081f660aa9c", "bytes_per_launch": 251.9e6}
+
+
+def gemm_traffic(workload):
+    import hashlib
+    try:
+        with open(os.path.join(ROOT, GEMM_TRAFFIC["source"]), "rb") as f:
+            same = hashlib.sha1(f.read()).hexdigest() == GEMM_TRAFFIC["sha1"]
+    except OSError:
+        same = False
+    return GEMM_TRAFFIC["bytes_per_launch"] if (same and workload == GEMM_TRAFFIC["workload"]) else None
 
 
 def peaks():
@@ -309,7 +325,7 @@ def run_mine(args):
         "steps_per_s": world * args.steps / (ms_max / 1e3),
         "roofline": {"bound": "tensor", "kernel": "k_bitlinear_gemm (tcgen05 kind::f16, exact int8 x ternary)",
                      "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                     "frac": achieved / peak if achieved else None, "traffic": None,
+                     "frac": achieved / peak if achieved else None, "traffic": gemm_traffic(args.workload),
                      "peak_source": f"{how} bf16_tflops_sustained",
                      "launches": prof["gemm_launches"], "avg_launch_ms": prof["gemm_ms"] / max(1, prof["gemm_launches"]),
                      "share_of_step": prof["gemm_ms"] / ms},
