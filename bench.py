@@ -137,6 +137,12 @@ def dist_setup(n_gpus):
     return None, 0, 1, 0
 
 
+def job_value(world: int, steps: int, tokens_per_step: int, ms_max: float) -> float:
+    """Whole-job tokens/s of N independent replicas: the tokens every rank
+    processed over the slowest rank's time (weak scaling)."""
+    return world * steps * tokens_per_step / (ms_max / 1e3)
+
+
 def barrier(dist):
     if dist is not None:
         dist.barrier()
@@ -306,7 +312,7 @@ def run_mine(args):
 
     pk, how = peaks()
     tokens = world * args.steps * B * S
-    value = tokens / (ms_max / 1e3)
+    value = job_value(world, args.steps, B * S, ms_max)
     gemm_s = prof["gemm_ms"] / 1e3
     achieved = prof["gemm_flops"] / gemm_s / 1e12 if gemm_s > 0 else None
     peak = float(pk.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
