@@ -88,7 +88,7 @@ int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspa
 int termezo_load_params(termezo_ctx* ctx, const float* d_latents, const float* d_embed,
                         const float* d_gains, const uint16_t* d_head);
 
-/* Algorithm 1, lines 1-2 (Eqs. 2-4): per projection gamma = mean |w|
+/* The initial mask of Algorithm 1 (Eqs. 2-4): per projection gamma = mean |w|
  * (exact sum), tau_0 = (gamma + 1e-5) / 2, distances d_i = min(|w_i - tau|,
  * |w_i + tau|) of all weights of all projections, xi_0 the lower
  * rho_0-quantile: exactly k0 = floor(rho_0 d) weights with the smallest
