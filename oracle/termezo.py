@@ -148,6 +148,42 @@ def masked_spsa(w: np.ndarray, active: np.ndarray, z: np.ndarray, eps, lr, objec
     return w_next, f_plus, f_minus, g, w_plus, w_minus, w_rest
 
 
+def masked_spsa_k(w: np.ndarray, active: np.ndarray, zs, eps, lr, objective):
+    """Algorithm 1's two inner loops with K = len(zs) directions.
+
+    Loop 1, for each direction k in order: w+ = w + e_k, F+; w- = w+ - 2 e_k,
+    F-; restore w = w- + e_k (the next direction starts from this restored
+    w); g_k = (F+ - F-) / (2 eps).  Loop 2, for each k in order with z_k
+    drawn again: w = w - (lr / K) g_k z_k, the coefficient (lr / K) g_k
+    formed in float64 and rounded to float32, every latent operation in
+    float32.  With K = 1 this is ``masked_spsa``.
+
+    Returns (w_next, [F+], [F-], [g], [w_restored after direction k])."""
+    eps = np.float32(eps)
+    K = len(zs)
+    w = w.copy()
+    fps, fms, gs, rests = [], [], [], []
+    for z in zs:
+        e = (eps * np.asarray(z, dtype=np.float32)).astype(np.float32)
+        w_plus = w.copy()
+        w_plus[active] = (w[active] + e).astype(np.float32)
+        fp = float(objective(w_plus))
+        w_minus = w_plus.copy()
+        w_minus[active] = (w_plus[active] - (np.float32(2.0) * e)).astype(np.float32)
+        fm = float(objective(w_minus))
+        w = w_minus.copy()
+        w[active] = (w_minus[active] + e).astype(np.float32)
+        fps.append(fp)
+        fms.append(fm)
+        gs.append((fp - fm) / (2.0 * float(eps)))
+        rests.append(w[active].copy())
+    lr_k = float(np.float32(lr)) / K
+    for z, g in zip(zs, gs):
+        c = np.float32(lr_k * g)
+        w[active] = (w[active] - (c * np.asarray(z, dtype=np.float32)).astype(np.float32)).astype(np.float32)
+    return w, fps, fms, gs, rests
+
+
 @dataclass
 class State:
     """Dense oracle state of a TerMeZO run."""
@@ -218,6 +254,47 @@ def step(state: State, loss_fn, seed: int, eps, lr):
                codes_minus=passes["minus"]["codes"],
                near_plus=passes["plus"]["near"], near_minus=passes["minus"]["near"],
                w_restored=w_rest[active].copy())
+    state.w = w_next
+    state.t += 1
+    state.log.append(rec)
+    return rec
+
+
+def step_k(state: State, loss_fn, seeds, eps, lr):
+    """One TerMeZO iteration of Algorithm 1 with K = len(seeds) directions:
+    the mask shrinks once (Eq. 5), then ``masked_spsa_k`` with z_k drawn
+    from seeds[k] at the active indices.  Returns per-direction losses,
+    g and counters (codes compared between the + and - pass of each
+    direction)."""
+    reg = state.reg
+    if state.t >= 1:
+        kept, tau_t = shrink(state.w, reg, state.active, state.xi0)
+        dropped = np.setdiff1d(state.active, kept)
+        if dropped.size:
+            tj = _tensor_of(reg, dropped)
+            state.frozen_code[dropped] = ternary.quantize(state.w[dropped], tau_t[tj])
+        state.active = kept
+    active = state.active
+    zs = [philox.normal(s, active) if active.size else np.zeros(0, np.float32) for s in seeds]
+    passes = []
+
+    def objective(wp):
+        codes, tau, sw = requantize(wp, reg)
+        frozen = np.ones(wp.size, dtype=bool)
+        frozen[active] = False
+        mism = int(np.count_nonzero(codes[frozen] != state.frozen_code[frozen]))
+        split = [codes[p.base:p.base + p.n].reshape(p.N, p.K) for p in reg]
+        passes.append(dict(codes=codes[active].astype(np.int64), tau=tau, sw=sw, frozen_mismatch=mism))
+        return loss_fn(split, sw)
+
+    w_next, fps, fms, gs, rests = masked_spsa_k(state.w, active, zs, eps, lr, objective)
+    flips = sum(int(np.count_nonzero(passes[2 * k]["codes"] != passes[2 * k + 1]["codes"])) for k in range(len(seeds)))
+    jumps = sum(int(np.count_nonzero(np.abs(passes[2 * k]["codes"] - passes[2 * k + 1]["codes"]) == 2))
+                for k in range(len(seeds)))
+    rec = dict(t=state.t, seeds=list(seeds), loss_plus=fps, loss_minus=fms, g=gs, k=int(active.size),
+               n_flipped=flips, n_jumps=jumps, frozen_mismatch=sum(p["frozen_mismatch"] for p in passes),
+               tau_plus=[passes[2 * k]["tau"] for k in range(len(seeds))],
+               tau_minus=[passes[2 * k + 1]["tau"] for k in range(len(seeds))], w_restored=rests)
     state.w = w_next
     state.t += 1
     state.log.append(rec)

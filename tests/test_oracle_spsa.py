@@ -106,3 +106,59 @@ def test_restore_and_update_arithmetic():
     c = np.float32(float(lr) * g)
     assert np.array_equal(w_next[active], (w_rest[active] - (c * z).astype(np.float32)).astype(np.float32))
     assert g == (fp - fm) / (2 * float(eps))
+
+
+def test_k_directions_reduce_to_one_and_apply_every_term():
+    """Algorithm 1 with K directions: K = 1 is the single-direction pass bit
+    for bit; for K = 3 each g_k is the exact two-point quotient at the
+    restored point of direction k, and the update applies the K terms
+    (lr / K) g_k z_k in order."""
+    n = 48
+    A, b, F = _quadratic(n, seed=3)
+    rng = np.random.default_rng(4)
+    w = (rng.standard_normal(n) * 0.1).astype(np.float32)
+    active = np.sort(rng.choice(n, 16, replace=False)).astype(np.int64)
+    eps, lr = 1e-3, 5e-3
+    z1 = philox.normal(7, active)
+    one = termezo.masked_spsa(w, active, z1, eps, lr, F)
+    many = termezo.masked_spsa_k(w, active, [z1], eps, lr, F)
+    assert np.array_equal(one[0], many[0]) and one[3] == many[3][0]
+    zs = [philox.normal(s, active) for s in (11, 12, 13)]
+    w_next, fps, fms, gs, rests = termezo.masked_spsa_k(w, active, zs, eps, lr, F)
+    e32 = np.float32(eps)
+    start = w.copy()
+    for k, z in enumerate(zs):
+        e = (e32 * z).astype(np.float32)
+        wp = start.copy()
+        wp[active] = (start[active] + e).astype(np.float32)
+        wm = wp.copy()
+        wm[active] = (wp[active] - np.float32(2) * e).astype(np.float32)
+        dp = wp.astype(np.float64) - wm.astype(np.float64)
+        mid = (wp.astype(np.float64) + wm.astype(np.float64)) / 2
+        assert abs(gs[k] - dp @ (A @ mid + b) / (2 * float(e32))) <= 1e-9 * max(1.0, abs(gs[k]))
+        start = wm.copy()
+        start[active] = (wm[active] + e).astype(np.float32)
+        assert np.array_equal(start[active], rests[k])
+    expect = start.copy()
+    for z, g in zip(zs, gs):
+        c = np.float32(float(np.float32(lr)) / 3 * g)
+        expect[active] = (expect[active] - (c * z).astype(np.float32)).astype(np.float32)
+    assert np.array_equal(w_next, expect)
+    frozen = np.setdiff1d(np.arange(n), active)
+    assert np.array_equal(w_next[frozen], w[frozen])
+
+
+def test_k_direction_update_averages_to_the_masked_gradient():
+    """E[z z^T] = I: over K directions the update -(lr / K) sum_k g_k z_k
+    tends to -lr (m * grad F) (App. E), which pins the 1 / K factor."""
+    n = 8
+    A, b, F = _quadratic(n, seed=5)
+    w = np.linspace(-0.5, 0.5, n).astype(np.float32)
+    active = np.array([0, 2, 3, 6], dtype=np.int64)
+    K, eps, lr = 4000, 1e-2, 1e-3
+    zs = [philox.normal(100 + k, active) for k in range(K)]
+    w_next, *_ = termezo.masked_spsa_k(w, active, zs, eps, lr, F)
+    step = (w_next.astype(np.float64) - w.astype(np.float64)) / -lr
+    grad = A @ w.astype(np.float64) + b
+    assert np.allclose(step[active], grad[active], atol=6 * np.abs(grad).max() / math.sqrt(K) + 0.05)
+    assert np.all(step[np.setdiff1d(np.arange(n), active)] == 0)
