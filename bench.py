@@ -1,5 +1,6 @@
 #!/usr/bin/env python
-"""Throughput of the TerMeZO training step (Algorithm 1, K = 1) on GB300.
+"""Throughput of the TerMeZO training step (Algorithm 1; K = 1 direction by
+default, --k-dirs K for more) on GB300.
 
 Prints ONE JSON line.  A step is one whole TerMeZO iteration: shrink (Eq. 5),
 perturb + requantise to 2-bit codes, BitNet forward at +eps z, perturb,
@@ -9,6 +10,7 @@ of synthetic tokens.  Default workload: the BitNet-b1.58-2B-shaped model
 last-token loss over 4 label tokens) at mask density 1%.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl mine|reference]
+                  [--workload NAME] [--k-dirs K]
 
 With N > 1 (torchrun) every rank runs an independent replica (the step has
 no cross-GPU exchange in this build); value = tokens of all ranks / max
@@ -265,6 +267,15 @@ def run_mine(args):
     ctx.termezo_load_params(w, emb, gains, head)
     stream = torch.cuda.current_stream()
 
+    K = args.k_dirs
+
+    def do_step(i, tok, tgt):
+        # one iteration of Algorithm 1 with K directions (seeds distinct per
+        # direction and step)
+        if K == 1:
+            return ctx.termezo_step(synth.step_seed(i), EPS, LR, density, tok, tgt)
+        return ctx.termezo_step_k([synth.step_seed(i * K + k) for k in range(K)], EPS, LR, density, tok, tgt)
+
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     k0, xi0 = ctx.termezo_build_mask(density)
@@ -276,7 +287,7 @@ def run_mine(args):
 
     for i in range(args.warmup):
         tok, tgt = batches[i]
-        ctx.termezo_step(synth.step_seed(i), EPS, LR, density, tok, tgt)
+        do_step(i, tok, tgt)
 
     with Clocks(local) as clk:
         barrier(dist)
@@ -286,7 +297,7 @@ def run_mine(args):
         outs = []
         for i in range(args.warmup, nb):
             tok, tgt = batches[i]
-            outs.append(ctx.termezo_step(synth.step_seed(i), EPS, LR, density, tok, tgt))
+            outs.append(do_step(i, tok, tgt))
         e1.record(stream)
         torch.cuda.synchronize()
         barrier(dist)
@@ -306,7 +317,7 @@ def run_mine(args):
     for i in range(args.warmup, nb):
         tok_d.copy_(tok_h[i], non_blocking=True)
         tgt_d.copy_(tgt_h[i], non_blocking=True)
-        ctx.termezo_step(synth.step_seed(nb + i), EPS, LR, density, tok_d, tgt_d)
+        do_step(nb + i, tok_d, tgt_d)
     torch.cuda.synchronize()
     e2e_s = max_over_ranks(dist, time.perf_counter() - t0)
 
@@ -327,6 +338,7 @@ def run_mine(args):
         "config": {"workload": f"{cfg.name} density {density}", "global_batch": B * world, "seq_len": S,
                    "parallelism": f"replicas{world}", "layers": cfg.layers, "hidden": cfg.hidden,
                    "density": density, "k_active": int(outs[-1]["k_active"]), "eps": EPS, "lr": LR,
+                   "directions": K,
                    "l2": "no flush: per-step working set (521 MB packed codes, >1 GB activations) exceeds L2"},
         "steps_per_s": world * args.steps / (ms_max / 1e3),
         "roofline": {"bound": "tensor", "kernel": "k_bitlinear_gemm (tcgen05 kind::f16, exact int8 x ternary)",
@@ -467,6 +479,8 @@ def main():
     ap.add_argument("--impl", choices=("mine", "reference"), default="mine")
     ap.add_argument("--workload", choices=sorted(WORKLOADS) + ["op"] + sorted(ATTN_WORKLOADS), default="2b")
     ap.add_argument("--op-density", type=float, default=0.01)
+    ap.add_argument("--k-dirs", type=int, default=1,
+                    help="perturbation directions per step (Algorithm 1's K, 1..8)")
     ap.add_argument("--op-shape", default="", help="N,K,M of the op workload's projection (default 6912,2560,2048)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()

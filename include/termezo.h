@@ -119,6 +119,23 @@ int termezo_step(termezo_ctx* ctx, uint64_t seed, float eps, float lr, double de
                  const int32_t* d_tokens, const int32_t* d_targets, termezo_step_out* out,
                  double* per_seq_plus, double* per_seq_minus);
 
+/* One TerMeZO iteration of Algorithm 1 with K directions (1 <= K <= 8; the
+ * paper's experiments use K = 5):
+ *   t >= 1: the mask shrinks once (Eq. 5), as in termezo_step;
+ *   for k = 0..K-1 with z_k regenerated from seeds[k]:
+ *     w += eps m.z_k -> F+_k;  w -= 2 eps m.z_k -> F-_k;  w += eps m.z_k
+ *     (restore: the next direction starts from the restored latents);
+ *     g_k = (F+_k - F-_k) / (2 eps);
+ *   then for k = 0..K-1: w -= (lr / K) g_k m.z_k, with (lr / K) g_k formed in
+ *   float64 and rounded to float32.
+ * seeds: host [K].  out: host report (required; loss_plus, loss_minus and g
+ * are those of the last direction, the counters are summed over the
+ * directions); losses: host [2K] F+_0, F-_0, F+_1, ... (nullable); g: host
+ * [K] (nullable).  K = 1 is termezo_step.  Synchronises once. */
+int termezo_step_k(termezo_ctx* ctx, const uint64_t* seeds, int32_t K, float eps, float lr, double density,
+                   const int32_t* d_tokens, const int32_t* d_targets, termezo_step_out* out, double* losses,
+                   double* g);
+
 /* Pieces of the step, for the single-projection context and for tests.
  * termezo_shrink: Eq. 5 at the current latents (no-op before the first
  *   update); host output n_dropped (nullable).

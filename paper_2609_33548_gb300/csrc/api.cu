@@ -125,7 +125,8 @@ struct termezo_ctx {
   float *cosb = nullptr, *sinb = nullptr;
   double* per_seq = nullptr;  // [2B]
   double* loss = nullptr;     // [2]
-  double* g = nullptr;        // [1]
+  double* g = nullptr;        // [KMAX]: g of each direction of a step
+  double* lossk = nullptr;    // [2 KMAX]: F+, F- of each direction
   GemmPlan plan_qkv{}, plan_o{}, plan_gu{}, plan_down{}, plan_head{};
   tmz::AttnPlan att_plan{};
   bool att_tc = false;
@@ -235,7 +236,8 @@ void carve(termezo_ctx* c, Carver& cv) {
   }
   c->per_seq = cv.take<double>(2 * (size_t)s.B);
   c->loss = cv.take<double>(2);
-  c->g = cv.take<double>(1);
+  c->g = cv.take<double>(tmz::KMAX);
+  c->lossk = cv.take<double>(2 * tmz::KMAX);
 }
 
 void plan_sizes(termezo_ctx* c, double density) {
@@ -609,9 +611,17 @@ int termezo_forward_loss(termezo_ctx* c, const int32_t* d_tokens, const int32_t*
   return TERMEZO_OK;
 }
 
-int termezo_step(termezo_ctx* c, uint64_t seed, float eps, float lr, double density, const int32_t* d_tokens,
-                 const int32_t* d_targets, termezo_step_out* out, double* per_seq_plus, double* per_seq_minus) {
-  if (!c || !d_tokens || !d_targets || !out) return TERMEZO_EINVAL;
+namespace {
+
+// Algorithm 1's loop body with K directions: shrink (t >= 1); for each
+// direction k: pm taus, requantise at +eps z_k, forward, requantise at
+// -eps z_k, forward, g_k, and (k < K-1) restore; then the last restore and
+// the K-term update in one pass.
+int step_impl(termezo_ctx* c, const uint64_t* seeds, int K, float eps, float lr, double density,
+              const int32_t* d_tokens, const int32_t* d_targets, termezo_step_out* out, double* losses, double* gs,
+              double* per_seq_plus, double* per_seq_minus) {
+  if (!c || !seeds || !d_tokens || !d_targets || !out) return TERMEZO_EINVAL;
+  if (K < 1 || K > tmz::KMAX) return TERMEZO_EINVAL;
   if (c->sh.op || !c->built) return TERMEZO_ESTATE;
   if (!(eps > 0.f) || !std::isfinite(lr)) return TERMEZO_EINVAL;
   const int warn = (density != c->density) ? TERMEZO_WMASKFIXED : TERMEZO_OK;
@@ -624,37 +634,50 @@ int termezo_step(termezo_ctx* c, uint64_t seed, float eps, float lr, double dens
   }
   c->pm_valid = false;
   const double k8 = 8.0 * (double)c->k_active;
-  {
-    ProfScope ps(c, 2, k8);
-    ensure_pm(c, seed, eps);
+  tmz::UpdateDirs dirs{};
+  dirs.K = K;
+  for (int k = 0; k < K; ++k) {
+    const uint64_t seed = seeds[k];
+    dirs.seed[k] = seed;
+    {
+      ProfScope ps(c, 2, k8);
+      ensure_pm(c, seed, eps);
+    }
+    {
+      ProfScope ps(c, 2, k8);
+      tmz::sparse_requant(c->ma, c->cur, seed, eps, +1, st);
+    }
+    rc = run_forward(c, d_tokens, d_targets, c->ma.sw_plus, 0);
+    if (rc) return rc;
+    {
+      ProfScope ps(c, 2, k8);
+      tmz::sparse_requant(c->ma, c->cur, seed, eps, -1, st);
+    }
+    rc = run_forward(c, d_tokens, d_targets, c->ma.sw_minus, 1);
+    if (rc) return rc;
+    c->code_sw = c->ma.sw_minus;
+    tmz::launch_grad(c->loss, eps, c->g + k, st);
+    if (K > 1) cudaMemcpyAsync(c->lossk + 2 * k, c->loss, 2 * sizeof(double), cudaMemcpyDeviceToDevice, st);
+    if (k + 1 < K) {
+      ProfScope ps(c, 2, 1.5 * k8);
+      tmz::sparse_restore(c->ma, c->cur, seed, eps, st);
+      c->pm_valid = false;
+    }
   }
-  {
-    ProfScope ps(c, 2, k8);
-    tmz::sparse_requant(c->ma, c->cur, seed, eps, +1, st);
-  }
-  rc = run_forward(c, d_tokens, d_targets, c->ma.sw_plus, 0);
-  if (rc) return rc;
-  {
-    ProfScope ps(c, 2, k8);
-    tmz::sparse_requant(c->ma, c->cur, seed, eps, -1, st);
-  }
-  rc = run_forward(c, d_tokens, d_targets, c->ma.sw_minus, 1);
-  if (rc) return rc;
-  c->code_sw = c->ma.sw_minus;
-  tmz::launch_grad(c->loss, eps, c->g, st);
+  dirs.last = seeds[K - 1];
   {
     ProfScope ps(c, 2, 1.5 * k8);
-    tmz::sparse_update(c->ma, c->cur, seed, eps, lr, c->g, 0.0, 0, st);
+    tmz::sparse_update_dirs(c->ma, c->cur, dirs, eps, lr, c->g, st);
   }
   c->pm_valid = false;
   struct {
-    double loss[2];
-    double g;
+    double loss[2 * tmz::KMAX];
+    double g[tmz::KMAX];
     unsigned long long cnt[4];
     uint32_t k;
   } h{};
-  cudaMemcpyAsync(h.loss, c->loss, 2 * sizeof(double), cudaMemcpyDeviceToHost, st);
-  cudaMemcpyAsync(&h.g, c->g, sizeof(double), cudaMemcpyDeviceToHost, st);
+  cudaMemcpyAsync(h.loss, K > 1 ? c->lossk : c->loss, 2 * K * sizeof(double), cudaMemcpyDeviceToHost, st);
+  cudaMemcpyAsync(h.g, c->g, K * sizeof(double), cudaMemcpyDeviceToHost, st);
   cudaMemcpyAsync(h.cnt, c->ma.counters, 4 * sizeof(unsigned long long), cudaMemcpyDeviceToHost, st);
   cudaMemcpyAsync(&h.k, c->ma.off[c->cur] + c->sh.P, sizeof(uint32_t), cudaMemcpyDeviceToHost, st);
   if (per_seq_plus)
@@ -666,14 +689,32 @@ int termezo_step(termezo_ctx* c, uint64_t seed, float eps, float lr, double dens
   c->updated = true;
   c->t += 1;
   c->k_active = h.k;
-  out->loss_plus = h.loss[0];
-  out->loss_minus = h.loss[1];
-  out->g = h.g;
+  out->loss_plus = h.loss[2 * (K - 1)];
+  out->loss_minus = h.loss[2 * (K - 1) + 1];
+  out->g = h.g[K - 1];
   out->k_active = h.k;
   out->n_flipped = h.cnt[0];
   out->n_jumps = h.cnt[1];
   out->n_dropped = h.cnt[2];
+  if (losses)
+    for (int i = 0; i < 2 * K; ++i) losses[i] = h.loss[i];
+  if (gs)
+    for (int k = 0; k < K; ++k) gs[k] = h.g[k];
   return warn;
+}
+
+}  // namespace
+
+int termezo_step(termezo_ctx* c, uint64_t seed, float eps, float lr, double density, const int32_t* d_tokens,
+                 const int32_t* d_targets, termezo_step_out* out, double* per_seq_plus, double* per_seq_minus) {
+  return step_impl(c, &seed, 1, eps, lr, density, d_tokens, d_targets, out, nullptr, nullptr, per_seq_plus,
+                   per_seq_minus);
+}
+
+int termezo_step_k(termezo_ctx* c, const uint64_t* seeds, int32_t K, float eps, float lr, double density,
+                   const int32_t* d_tokens, const int32_t* d_targets, termezo_step_out* out, double* losses,
+                   double* g) {
+  return step_impl(c, seeds, K, eps, lr, density, d_tokens, d_targets, out, losses, g, nullptr, nullptr);
 }
 
 int termezo_shrink(termezo_ctx* c, uint64_t* n_dropped) {

@@ -465,26 +465,50 @@ __global__ void __launch_bounds__(TPB) k_sparse_requant(MaskArgs a, int cur, uin
 
 // Restore and update: w' = ((w + e) - 2e) + e; w <- w' - fl32(c z) with
 // c = (float)(lr * g); accumulates the exact sum of the new |w|.
-__global__ void __launch_bounds__(TPB) k_sparse_update(MaskArgs a, int cur, uint64_t seed, float eps, float lr,
+// Algorithm 1's restore of the last direction followed by its update loop:
+// w' = fl(w- + e) with the last direction's z, then for each direction k in
+// order w = fl(w - fl(c_k z_k)), z_k regenerated from its seed.  Also the
+// exact per-block sums of |w| of the result (the next tau).
+template <int KM>
+__global__ void __launch_bounds__(TPB) k_sparse_update(MaskArgs a, int cur, UpdateDirs d, float eps, float lr,
                                                        const double* g_dev, double g_host, int use_host) {
   __shared__ ExactSum red[TPB / 32];
   const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
-  const double g = use_host ? g_host : *g_dev;
-  const float c = (float)((double)lr * g);
+  const double lr_k = (double)lr / (double)d.K;
+  float c[KM];
+#pragma unroll
+  for (int k = 0; k < KM; ++k) c[k] = k < d.K ? (float)(lr_k * (use_host ? g_host : g_dev[k])) : 0.f;
+  const uint64_t last = KM == 1 ? d.seed[0] : d.last;
   ExactAcc acc;
   ea_zero(acc);
   for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) {
-    const float z = normal_at(seed, a.idx[cur][e]);
+    const uint32_t i = a.idx[cur][e];
+    const float zl = normal_at(last, i);
     float wp, wm, ee;
-    perturbed(a.lat[cur][e], z, eps, &wp, &wm, &ee);
-    const float wr = __fadd_rn(wm, ee);
-    const float wn = __fsub_rn(wr, __fmul_rn(c, z));
+    perturbed(a.lat[cur][e], zl, eps, &wp, &wm, &ee);
+    float wn = __fadd_rn(wm, ee);
+#pragma unroll
+    for (int k = 0; k < KM; ++k)
+      if (k < d.K) {
+        const float z = (KM == 1 || k == d.K - 1) ? zl : normal_at(d.seed[k], i);
+        wn = __fsub_rn(wn, __fmul_rn(c[k], z));
+      }
     a.lat[cur][e] = wn;
     ea_add_abs(acc, wn);
   }
   ExactSum s = ea_result(acc);
   es_block_reduce(s, red);
   if (threadIdx.x == 0) a.partials[blockIdx.x] = s;
+}
+
+// Algorithm 1's restore after a direction that is not the last one.
+__global__ void __launch_bounds__(TPB) k_sparse_restore(MaskArgs a, int cur, uint64_t seed, float eps) {
+  const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
+  for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) {
+    float wp, wm, ee;
+    perturbed(a.lat[cur][e], normal_at(seed, a.idx[cur][e]), eps, &wp, &wm, &ee);
+    a.lat[cur][e] = __fadd_rn(wm, ee);
+  }
 }
 
 // Eq. 5 at tau_cur: marks dropped weights, writes their code at tau_cur,
@@ -641,9 +665,28 @@ void sparse_requant(const MaskArgs& a, int cur, uint64_t seed, float eps, int si
 void sparse_update(const MaskArgs& a, int cur, uint64_t seed, float eps, float lr, const double* g_dev, double g_host,
                    int use_host, cudaStream_t s) {
   kernel_launches() += 2;
-  k_sparse_update<<<a.NBS, TPB, 0, s>>>(a, cur, seed, eps, lr, g_dev, g_host, use_host);
+  UpdateDirs d{};
+  d.seed[0] = d.last = seed;
+  d.K = 1;
+  k_sparse_update<1><<<a.NBS, TPB, 0, s>>>(a, cur, d, eps, lr, g_dev, g_host, use_host);
   k_reduce_proj<<<a.P, TPB, 0, s>>>(a.partials, a.spre, 1, 0, a.A_frozen, a.base, nullptr, a.gamma_cur, a.tau_cur,
                                     a.sw_cur);
+}
+
+void sparse_update_dirs(const MaskArgs& a, int cur, const UpdateDirs& d, float eps, float lr, const double* g_dev,
+                        cudaStream_t s) {
+  kernel_launches() += 2;
+  if (d.K == 1)
+    k_sparse_update<1><<<a.NBS, TPB, 0, s>>>(a, cur, d, eps, lr, g_dev, 0.0, 0);
+  else
+    k_sparse_update<KMAX><<<a.NBS, TPB, 0, s>>>(a, cur, d, eps, lr, g_dev, 0.0, 0);
+  k_reduce_proj<<<a.P, TPB, 0, s>>>(a.partials, a.spre, 1, 0, a.A_frozen, a.base, nullptr, a.gamma_cur, a.tau_cur,
+                                    a.sw_cur);
+}
+
+void sparse_restore(const MaskArgs& a, int cur, uint64_t seed, float eps, cudaStream_t s) {
+  kernel_launches() += 1;
+  k_sparse_restore<<<a.NBS, TPB, 0, s>>>(a, cur, seed, eps);
 }
 
 void sparse_shrink(const MaskArgs& a, int cur, float xi0, uint32_t* d_total, cudaStream_t s) {

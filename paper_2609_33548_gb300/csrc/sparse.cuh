@@ -46,6 +46,19 @@ void mask_build(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_t s);
 void mask_finish(const MaskArgs& a, cudaStream_t s);
 void sparse_pm_taus(const MaskArgs& a, int cur, uint64_t seed, float eps, cudaStream_t s);
 void sparse_requant(const MaskArgs& a, int cur, uint64_t seed, float eps, int sign, cudaStream_t s);
+// Directions of one step (Algorithm 1 with K <= KMAX perturbations).
+constexpr int KMAX = 8;
+struct UpdateDirs {
+  uint64_t seed[KMAX];
+  uint64_t last;  // seed[K - 1]
+  int K;
+};
+// Restore after direction seed: w = fl(fl(fl(w + e) - 2 e) + e), e = fl(eps z).
+void sparse_restore(const MaskArgs& a, int cur, uint64_t seed, float eps, cudaStream_t s);
+// Restore after the last direction, then w = fl(w - fl(c_k z_k)) for k = 0..K-1
+// with c_k = (float)((lr / K) g_k), g_k = g_dev[k]; exact sums of the result.
+void sparse_update_dirs(const MaskArgs& a, int cur, const UpdateDirs& d, float eps, float lr, const double* g_dev,
+                        cudaStream_t s);
 void sparse_update(const MaskArgs& a, int cur, uint64_t seed, float eps, float lr, const double* g_dev,
                    double g_host, int use_host, cudaStream_t s);
 void sparse_shrink(const MaskArgs& a, int cur, float xi0, uint32_t* d_total, cudaStream_t s);

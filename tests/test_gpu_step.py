@@ -163,3 +163,69 @@ def test_mask_and_update_replay_many_steps(inputs):
         sizes.append(act.size)
     assert sizes[-1] < sizes[0]
     assert all(a >= b for a, b in zip(sizes, sizes[1:]))
+
+
+def test_k_directions_step_matches_oracle(inputs):
+    """Algorithm 1 with K = 3 directions: per-direction F+-, g_k against the
+    oracle's ensembles; the latents after the K restores and the K-term
+    update (the oracle's update recomputed with the GPU's g_k, so that only
+    the rounding of the restores and of z remains); and the index list."""
+    K = 3
+    ctx, dev = _gpu_ctx(inputs)
+    ctx.termezo_build_mask(DENSITY)
+    cfg, th = _cfg(inputs), _theta_np(inputs)
+    reg = otz.registry(cfg)
+    state = otz.build(inputs[0].numpy(), reg, DENSITY)
+    fn = otz.bitnet_loss_fn(cfg, *th)
+    w_before = state.w.copy()
+    act = state.active.copy()
+    seeds = [synth.step_seed(10 + k) for k in range(K)]
+    out = ctx.termezo_step_k(seeds, EPS, LR, DENSITY, dev[4], dev[5])
+    rec = otz.step_k(state, fn, seeds, EPS, LR)
+    eps32 = np.float32(EPS)
+    w = w_before.copy()
+    zs = []
+    for k, seed in enumerate(seeds):
+        z = philox.normal(seed, act)
+        zs.append(z)
+        e = (eps32 * z).astype(np.float32)
+        wp = w.copy(); wp[act] = (w[act] + e).astype(np.float32)
+        wm = wp.copy(); wm[act] = (wp[act] - np.float32(2) * e).astype(np.float32)
+        cp, _, swp = otz.requantize(wp, reg)
+        cm, _, swm = otz.requantize(wm, reg)
+        lp = rounding.loss_ensemble(cfg, (_split(cp, reg), swp), th, n=4).mean(axis=1)
+        lm = rounding.loss_ensemble(cfg, (_split(cm, reg), swm), th, n=4).mean(axis=1)
+        fp, fm = out["losses"][k]
+        assert rounding.within(fp, rec["loss_plus"][k], lp), (k, fp, rec["loss_plus"][k], lp)
+        assert rounding.within(fm, rec["loss_minus"][k], lm), (k, fm, rec["loss_minus"][k], lm)
+        ens = (lp - lm) / (2 * float(eps32))
+        assert rounding.g_within_ensemble(out["g_k"][k], rec["g"][k], ens), (k, out["g_k"][k], rec["g"][k], ens)
+        w = wm.copy(); w[act] = (wm[act] + e).astype(np.float32)
+        np.testing.assert_array_equal(w[act], rec["w_restored"][k])
+    assert out["g"] == out["g_k"][-1] and out["loss_plus"] == out["losses"][-1][0]
+    assert out["k_active"] == rec["k"] == act.size and out["n_jumps"] == rec["n_jumps"]
+    # the update with the GPU's g_k
+    lr_k = float(np.float32(LR)) / K
+    expect = w.copy()
+    for z, g in zip(zs, out["g_k"]):
+        c = np.float32(lr_k * g)
+        expect[act] = (expect[act] - (c * z).astype(np.float32)).astype(np.float32)
+    st = ctx.termezo_export_state(packed=False)
+    np.testing.assert_array_equal(st["idx"], act.astype(np.uint32))
+    scale = np.abs(w_before[act]) + 2 * max(float(np.abs(eps32 * z).max()) for z in zs)
+    assert np.all(np.abs(st["latents"].astype(np.float64) - expect[act]) <= K * 1e-5 * scale)
+
+
+def test_single_direction_step_k_is_step(inputs):
+    """termezo_step_k with one seed runs the same kernels as termezo_step:
+    losses, g and the latents after the step are identical."""
+    a, dev = _gpu_ctx(inputs)
+    b, _ = _gpu_ctx(inputs)
+    a.termezo_build_mask(DENSITY)
+    b.termezo_build_mask(DENSITY)
+    seed = synth.step_seed(3)
+    oa = a.termezo_step(seed, EPS, LR, DENSITY, dev[4], dev[5])
+    ob = b.termezo_step_k([seed], EPS, LR, DENSITY, dev[4], dev[5])
+    assert (oa["loss_plus"], oa["loss_minus"], oa["g"]) == (ob["loss_plus"], ob["loss_minus"], ob["g"])
+    sa, sb = a.termezo_export_state(packed=False), b.termezo_export_state(packed=False)
+    np.testing.assert_array_equal(sa["latents"].view(np.uint32), sb["latents"].view(np.uint32))
