@@ -21,6 +21,7 @@ from __future__ import annotations
 
 import argparse
 import json
+import math
 import os
 import statistics
 import subprocess
@@ -210,6 +211,26 @@ class OracleSample:
         return est, t_rq, t_fw
 
 
+def memory_report(cfg, density, peak_bytes):
+    """Device bytes by part (termezo_memory) next to the memory equation of
+    Sec. 5 evaluated with this build's precisions (B = 4 fp32 latents,
+    B_Q = 1/4, 32-bit active indices), and the peak torch allocation over the
+    timed steps (workspace + theta + batches)."""
+    from paper_2609_33548_gb300 import termezo as tz
+    m = tz.termezo_memory(tz.make_cfg(cfg), density)
+    d, k0 = m["d"], m["k_cap"]
+    B, BQ = 4, 0.25
+    eq_latent = d * B - math.ceil(d * (1 - density) * (B - BQ)) + math.ceil(density * d * BQ) + math.ceil(k0 * 4)
+    gb = 1e9
+    return {"workspace_gb": m["workspace"] / gb, "packed_codes_gb": m["packed"] / gb,
+            "sparse_store_gb": (m["sparse_index"] + m["sparse_latents"]) / gb, "forward_gb": m["forward"] / gb,
+            "theta_gb": m["theta"] / gb, "peak_allocated_gb": peak_bytes / gb,
+            "latents": {"mezo_fp32_gb": d * B / gb, "equation_gb": eq_latent / gb,
+                        "build_gb": (m["packed"] + m["sparse_index"] + m["sparse_latents"]) / gb,
+                        "note": "build = equation + the second sparse-store buffer of the shrink"},
+            "mask_options_gb": {"bitmask": m["mask_bitmask"] / gb, "index_list": m["mask_index_list"] / gb}}
+
+
 def cores():
     try:
         return len(os.sched_getaffinity(0))
@@ -284,6 +305,11 @@ def run_mine(args):
     build_ms = e0.elapsed_time(e1)
     d = cfg.d_lat
     build_bytes = 6 * 4 * d + d / 4 + 8 * k0          # 6 reads of w_0, packed codes and S_0 written
+    # the dense latents are read only by the mask build: released here, so the
+    # footprint measured over the timed steps is the method's (Sec. 5)
+    del w
+    torch.cuda.empty_cache()
+    torch.cuda.reset_peak_memory_stats(dev)
 
     for i in range(args.warmup):
         tok, tgt = batches[i]
@@ -353,6 +379,7 @@ def run_mine(args):
                     "sparse_share": prof["sparse_ms"] / ms,
                     "mask_build_ms": build_ms, "mask_build_gbs": build_bytes / (build_ms / 1e3) / 1e9},
         "e2e": {"value": tokens / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "memory": memory_report(cfg, density, torch.cuda.max_memory_allocated(dev)),
         "gpu_launches": int(prof["launches"]),
         "clocks": clocks,
         "last_step": {k: outs[-1][k] for k in ("loss_plus", "loss_minus", "g", "n_flipped", "n_jumps")},

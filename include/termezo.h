@@ -70,6 +70,29 @@ typedef struct {
  * rho_0 (the sparse store holds floor(rho_0 * d) weights).  Host only. */
 int termezo_workspace_bytes(const termezo_model_cfg* cfg, double density, size_t* bytes);
 
+/* Device memory of a context, by part (Sec. 5's memory equation): the
+ * paper gives the TerMeZO footprint as the MeZO footprint minus
+ * d (1 - rho_0)(B - B_Q) plus rho_0 d B_Q plus the mask, M_mask =
+ * min(ceil(d / 8), ceil(rho_0 d ceil(log2 d) / 8)).  This build stores the
+ * active latents in float32 (B = 4) with 32-bit indices, both in two buffers
+ * (the order-preserving shrink writes the second), and every code packed at
+ * B_Q = 2/8.  All sizes in bytes; host only, no device call. */
+typedef struct {
+  uint64_t d;               /* ternary latents */
+  uint64_t k_cap;           /* active latents the store holds (k0) */
+  uint64_t packed;          /* 2-bit codes of all d latents */
+  uint64_t sparse_index;    /* active index lists (two buffers) */
+  uint64_t sparse_latents;  /* fp32 active latents (two buffers) */
+  uint64_t mask_state;      /* exact sums, partials, histograms, counters, losses */
+  uint64_t forward;         /* forward activations and GEMM operands */
+  uint64_t workspace;       /* all of the above: termezo_workspace_bytes */
+  uint64_t theta;           /* the caller's embeddings (fp32), norm gains (fp32), LM head (bf16) */
+  uint64_t mask_bitmask;    /* the paper's dense bit-mask option, ceil(d / 8) */
+  uint64_t mask_index_list; /* the paper's index-list option, ceil(rho_0 d ceil(log2 d) / 8) */
+} termezo_memory_out;
+
+int termezo_memory(const termezo_model_cfg* cfg, double density, termezo_memory_out* out);
+
 /* Creates a context over a caller-owned device workspace of `bytes` bytes
  * (>= termezo_workspace_bytes(cfg, density)); 256-byte aligned.  `stream`
  * is a cudaStream_t.  The workspace must outlive the context. */
@@ -78,7 +101,10 @@ int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspa
 
 /* Registers the parameters (device pointers, read by later calls; they
  * must stay valid until termezo_build_mask returns, and d_embed, d_gains,
- * d_head for the life of the context):
+ * d_head for the life of the context).  d_latents is read by
+ * termezo_build_mask only: once it returns successfully the context forgets
+ * the pointer (the caller may release the dense latents; another build
+ * needs another termezo_load_params, else it returns TERMEZO_ESTATE):
  *   d_latents fp32 [d]       dense latent weights w_0, global order;
  *   d_embed   fp32 [V, D]    token embeddings (theta);
  *   d_gains   fp32 [2L+1, D] RMSNorm gains: 2l = attention input of layer l,

@@ -80,17 +80,28 @@ int make_shape(const termezo_model_cfg* c, Shape* s) {
 uint64_t keep_count(double density, uint64_t d) { return (uint64_t)std::floor(density * (double)d); }
 
 // Bump allocator over the workspace; with base == nullptr it only measures.
+// Workspace sections, for the memory report.
+enum Section { SEC_PACKED, SEC_INDEX, SEC_LATENTS, SEC_MASK, SEC_FORWARD, SEC_COUNT };
+
 struct Carver {
   uint8_t* base;
   size_t off = 0;
+  int sec = SEC_MASK;
+  size_t bytes[SEC_COUNT] = {};
   template <typename T>
   T* take(size_t count) {
-    off = (off + 255) & ~(size_t)255;
-    T* p = base ? reinterpret_cast<T*>(base + off) : nullptr;
-    off += count * sizeof(T);
+    const size_t start = (off + 255) & ~(size_t)255;
+    T* p = base ? reinterpret_cast<T*>(base + start) : nullptr;
+    bytes[sec] += start + count * sizeof(T) - off;
+    off = start + count * sizeof(T);
     return p;
   }
 };
+
+// The QKV projection writes RoPE-rotated bf16 Q, K and V^T directly (fused
+// epilogue) for head dims 64 / 128 and S a multiple of 32; other shapes go
+// through an fp32 QKV buffer and a separate RoPE pass.
+bool rope_fused_shape(const Shape& s) { return !s.op && (s.hd == 64 || s.hd == 128) && s.S % 32 == 0; }
 
 }  // namespace
 
@@ -189,10 +200,14 @@ void carve(termezo_ctx* c, Carver& cv) {
   a.spre = cv.take<uint32_t>(P + 1);
   a.dproj = cv.take<uint16_t>(c->dpre.empty() ? 1 : c->dpre.back());
   a.sproj = cv.take<uint16_t>(c->NBS_max);
+  cv.sec = SEC_PACKED;
   a.packed = cv.take<uint32_t>(s.d / 16);
   for (int i = 0; i < 2; ++i) {
+    cv.sec = SEC_INDEX;
     a.idx[i] = cv.take<uint32_t>(c->k_cap);
+    cv.sec = SEC_LATENTS;
     a.lat[i] = cv.take<float>(c->k_cap);
+    cv.sec = SEC_MASK;
     a.off[i] = cv.take<uint32_t>(P + 1);
   }
   a.S_total = cv.take<ExactSum>(P);
@@ -213,18 +228,19 @@ void carve(termezo_ctx* c, Carver& cv) {
   a.err = cv.take<unsigned>(1);
   c->d_total = cv.take<uint32_t>(1);
   const size_t T = s.T;
+  cv.sec = SEC_FORWARD;
   c->xq = cv.take<uint16_t>(T * xq_cols(s));
   c->deq = cv.take<float>(T);
   c->wexp = cv.take<uint16_t>(wexp_elems(s));
   if (!s.op) {
     const size_t hq = (size_t)s.H * s.hd, hkv = (size_t)s.KV * s.hd;
     c->x = cv.take<float>(T * s.D);
-    c->qkv = cv.take<float>(T * (hq + 2 * hkv));
+    c->qkv = rope_fused_shape(s) ? nullptr : cv.take<float>(T * (hq + 2 * hkv));
     c->qb = cv.take<uint16_t>(T * hq);
     c->kb = cv.take<uint16_t>(T * hkv);
     c->vt = cv.take<uint16_t>(T * hkv);
     c->attn = cv.take<float>(T * hq);
-    c->gu = cv.take<float>(T * 2 * (size_t)s.F);
+    c->gu = cv.take<float>(T * (size_t)s.F);  // hid = relu(gate)^2 up
     c->cosb = cv.take<float>((size_t)s.S * s.hd / 2);
     c->sinb = cv.take<float>((size_t)s.S * s.hd / 2);
     if (s.mode == 1) {
@@ -234,6 +250,7 @@ void carve(termezo_ctx* c, Carver& cv) {
       c->tok_loss = cv.take<double>(T);
     }
   }
+  cv.sec = SEC_MASK;
   c->per_seq = cv.take<double>(2 * (size_t)s.B);
   c->loss = cv.take<double>(2);
   c->g = cv.take<double>(tmz::KMAX);
@@ -453,6 +470,33 @@ int termezo_workspace_bytes(const termezo_model_cfg* cfg, double density, size_t
   return TERMEZO_OK;
 }
 
+int termezo_memory(const termezo_model_cfg* cfg, double density, termezo_memory_out* out) {
+  if (!out || !(density > 0.0 && density <= 1.0)) return TERMEZO_EINVAL;
+  termezo_ctx tmp;
+  int rc = make_shape(cfg, &tmp.sh);
+  if (rc) return rc;
+  plan_sizes(&tmp, density);
+  Carver cv{nullptr};
+  carve(&tmp, cv);
+  const Shape& s = tmp.sh;
+  out->d = s.d;
+  out->k_cap = tmp.k_cap;
+  out->packed = cv.bytes[SEC_PACKED];
+  out->sparse_index = cv.bytes[SEC_INDEX];
+  out->sparse_latents = cv.bytes[SEC_LATENTS];
+  out->mask_state = cv.bytes[SEC_MASK];
+  out->forward = cv.bytes[SEC_FORWARD];
+  out->workspace = cv.off + 256;
+  out->theta = s.op ? 0
+                    : (uint64_t)s.V * s.D * 4 + (uint64_t)(2 * s.L + 1) * s.D * 4 + (uint64_t)s.V * s.D * 2;
+  uint64_t lg = 0;
+  while ((1ull << lg) < s.d) ++lg;
+  const uint64_t k0 = keep_count(density, s.d);
+  out->mask_bitmask = (s.d + 7) / 8;
+  out->mask_index_list = (k0 * lg + 7) / 8;
+  return TERMEZO_OK;
+}
+
 int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspace, size_t bytes, void* stream,
                    termezo_ctx** out) {
   if (!out || !d_workspace || !(density > 0.0 && density <= 1.0)) return TERMEZO_EINVAL;
@@ -492,7 +536,7 @@ int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspa
   if (!s.op) {
     tmz::launch_rope_tables(s.S, s.hd, c->cosb, c->sinb, st);
     const int T = s.T, D = s.D, F = s.F, hq = s.H * s.hd, hkv = s.KV * s.hd;
-    const bool rope_fused = (s.hd == 64 || s.hd == 128) && s.S % 32 == 0;
+    const bool rope_fused = rope_fused_shape(s);
     bool ok = tmz::gemm_make_plan(&c->plan_qkv, c->xq, T, D, c->wexp, hq + 2 * hkv, !rope_fused) &&
               tmz::gemm_make_plan(&c->plan_o, c->xq, T, hq, c->wexp, D, true) &&
               tmz::gemm_make_plan(&c->plan_gu, c->xq, T, D, c->wexp, 256 * ((F + 127) / 128), false) &&
@@ -504,8 +548,15 @@ int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspa
     // TMA output maps (a layout that does not allow one keeps the plain stores)
     // q, k, v written by the QKV GEMM's epilogue (RoPE fused) where the head
     // layout allows it
-    if (!(rope_fused && tmz::gemm_plan_rope(&c->plan_qkv, c->qb, c->kb, s.B, s.S, s.H, s.KV, s.hd)))
+    if (rope_fused) {
+      // the workspace has no fp32 QKV buffer for these shapes
+      if (!tmz::gemm_plan_rope(&c->plan_qkv, c->qb, c->kb, s.B, s.S, s.H, s.KV, s.hd)) {
+        delete c;
+        return TERMEZO_ECUDA;
+      }
+    } else {
       tmz::gemm_plan_output(&c->plan_qkv, c->qkv, hq + 2 * hkv);
+    }
     tmz::gemm_plan_output(&c->plan_o, c->x, D);
     tmz::gemm_plan_output(&c->plan_down, c->x, D);
     c->att_tc = tmz::attention_tc_supported(s.S, s.hd) &&
@@ -588,6 +639,8 @@ int termezo_build_mask(termezo_ctx* c, double density, uint64_t* k0_out, float* 
   rc = sync_status(c);
   if (rc) return rc;
   c->built = true;
+  // the dense latents are not read again: the caller may release them
+  c->latents = nullptr;
   if (k0_out) *k0_out = k0;
   if (xi0_out) *xi0_out = xi0;
   return TERMEZO_OK;

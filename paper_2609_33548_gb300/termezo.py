@@ -19,7 +19,7 @@ OK, WMASKFIXED, EINVAL, ESTATE, ENOMEM, ECUDA, ETIMEOUT = 0, 1, -1, -2, -3, -4, 
 
 # Every function declared in include/termezo.h.
 EXPORTS = (
-    "termezo_workspace_bytes", "termezo_create", "termezo_load_params", "termezo_build_mask",
+    "termezo_workspace_bytes", "termezo_memory", "termezo_create", "termezo_load_params", "termezo_build_mask",
     "termezo_forward_loss", "termezo_step", "termezo_step_k", "termezo_shrink", "termezo_requantize", "termezo_update",
     "termezo_bitlinear", "termezo_state_sizes", "termezo_export_state", "termezo_normal",
     "termezo_absmean_noalloc", "termezo_attention", "termezo_profile", "termezo_destroy", "termezo_strerror",
@@ -37,6 +37,15 @@ class StepOut(ctypes.Structure):
                 ("g", ctypes.c_double), ("k_active", ctypes.c_uint64),
                 ("n_flipped", ctypes.c_uint64), ("n_jumps", ctypes.c_uint64),
                 ("n_dropped", ctypes.c_uint64)]
+
+    def as_dict(self):
+        return {n: getattr(self, n) for n, _ in self._fields_}
+
+
+class MemoryOut(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_uint64) for n in
+                ("d", "k_cap", "packed", "sparse_index", "sparse_latents", "mask_state", "forward", "workspace",
+                 "theta", "mask_bitmask", "mask_index_list")]
 
     def as_dict(self):
         return {n: getattr(self, n) for n, _ in self._fields_}
@@ -80,6 +89,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
     P, I32, U64, F32, F64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_uint64, ctypes.c_float, ctypes.c_double
     sig = {
         "termezo_workspace_bytes": (I32, [ctypes.POINTER(ModelCfg), F64, ctypes.POINTER(ctypes.c_size_t)]),
+        "termezo_memory": (I32, [ctypes.POINTER(ModelCfg), F64, ctypes.POINTER(MemoryOut)]),
         "termezo_create": (I32, [ctypes.POINTER(ModelCfg), F64, P, ctypes.c_size_t, P, ctypes.POINTER(P)]),
         "termezo_load_params": (I32, [P, P, P, P, P]),
         "termezo_build_mask": (I32, [P, F64, ctypes.POINTER(U64), ctypes.POINTER(F32)]),
@@ -140,6 +150,13 @@ def termezo_workspace_bytes(cfg: ModelCfg, density: float) -> int:
     return n.value
 
 
+def termezo_memory(cfg: ModelCfg, density: float) -> dict:
+    """Device bytes of a context by part (host only)."""
+    out = MemoryOut()
+    _check("termezo_memory", load().termezo_memory(ctypes.byref(cfg), density, ctypes.byref(out)))
+    return out.as_dict()
+
+
 class Context:
     """Owns the device workspace (a torch tensor) and the library context."""
 
@@ -179,6 +196,7 @@ class Context:
         xi0 = ctypes.c_float(0)
         _check("termezo_build_mask", load().termezo_build_mask(self.handle, density, ctypes.byref(k0),
                                                                ctypes.byref(xi0)))
+        self._keep[0] = None  # the library no longer reads the dense latents
         return k0.value, np.float32(xi0.value)
 
     def termezo_forward_loss(self, tokens, targets):
