@@ -184,6 +184,63 @@ def masked_spsa_k(w: np.ndarray, active: np.ndarray, zs, eps, lr, objective):
     return w, fps, fms, gs, rests
 
 
+def _stored(x, bf16: bool) -> np.ndarray:
+    """x rounded to a part's stored precision: float32, then bfloat16 for a
+    bf16 part (round to nearest even)."""
+    x = np.asarray(x, dtype=np.float32)
+    return bitnet.bf16_round(x) if bf16 else x
+
+
+def joint_spsa_k(w: np.ndarray, active: np.ndarray, theta, bf16, zs_w, zs_t, eps, lr, objective):
+    """Algorithm 1's two inner loops over the masked latents w[active] and
+    the full-precision parameters theta together (both perturbed with the
+    seed of each direction).
+
+    theta: list of float32 arrays (embeddings, norm gains, LM head); bf16[i]
+    marks a part stored in bfloat16.  zs_t[k]: z of theta for direction k,
+    the parts concatenated in order.  Every assignment of Algorithm 1 is
+    rounded to the stored precision of what it assigns (float32; bfloat16
+    after the float32 operation for a bf16 part).  objective(w, theta) ->
+    float.  Returns (w, theta, [F+], [F-], [g])."""
+    eps = np.float32(eps)
+    K = len(zs_w)
+    w = w.copy()
+    th = [np.asarray(t, dtype=np.float32).copy() for t in theta]
+    offs = np.cumsum([0] + [t.size for t in th])
+
+    def split(z):
+        return [np.asarray(z[offs[i]:offs[i + 1]], dtype=np.float32).reshape(th[i].shape) for i in range(len(th))]
+
+    fps, fms, gs = [], [], []
+    for zw, zt in zip(zs_w, zs_t):
+        ew = (eps * np.asarray(zw, dtype=np.float32)).astype(np.float32)
+        et = [(eps * z).astype(np.float32) for z in split(zt)]
+        w[active] = (w[active] + ew).astype(np.float32)
+        th = [_stored(t + e, b) for t, e, b in zip(th, et, bf16)]
+        fp = float(objective(w, th))
+        w[active] = (w[active] - np.float32(2.0) * ew).astype(np.float32)
+        th = [_stored(t - np.float32(2.0) * e, b) for t, e, b in zip(th, et, bf16)]
+        fm = float(objective(w, th))
+        w[active] = (w[active] + ew).astype(np.float32)
+        th = [_stored(t + e, b) for t, e, b in zip(th, et, bf16)]
+        fps.append(fp)
+        fms.append(fm)
+        gs.append((fp - fm) / (2.0 * float(eps)))
+    lr_k = float(np.float32(lr)) / K
+    for zw, zt, g in zip(zs_w, zs_t, gs):
+        c = np.float32(lr_k * g)
+        w[active] = (w[active] - (c * np.asarray(zw, dtype=np.float32)).astype(np.float32)).astype(np.float32)
+        th = [_stored(t - (c * z).astype(np.float32), b) for t, z, b in zip(th, split(zt), bf16)]
+    return w, th, fps, fms, gs
+
+
+def theta_normals(seed: int, d: int, p: int) -> np.ndarray:
+    """z of the full-precision parameters for one direction: the Philox
+    stream of the seed at global indices d .. d + p - 1 (after the d
+    latents), so that it never shares a value with the latents' z."""
+    return philox.normal(seed, np.arange(d, d + p, dtype=np.uint64))
+
+
 @dataclass
 class State:
     """Dense oracle state of a TerMeZO run."""
@@ -299,6 +356,51 @@ def step_k(state: State, loss_fn, seeds, eps, lr):
     state.t += 1
     state.log.append(rec)
     return rec
+
+
+def step_joint(state: State, theta, loss_fn, seeds, eps, lr):
+    """One iteration of Algorithm 1 as written: K = len(seeds) directions
+    over the masked latents and theta = [embeddings fp32, norm gains fp32,
+    LM head bf16] together.  loss_fn(codes, s_w, theta) -> float.  Returns
+    the record and the new theta."""
+    reg = state.reg
+    if state.t >= 1:
+        kept, tau_t = shrink(state.w, reg, state.active, state.xi0)
+        dropped = np.setdiff1d(state.active, kept)
+        if dropped.size:
+            tj = _tensor_of(reg, dropped)
+            state.frozen_code[dropped] = ternary.quantize(state.w[dropped], tau_t[tj])
+        state.active = kept
+    active = state.active
+    d = state.w.size
+    p = sum(np.asarray(t).size for t in theta)
+    zs_w = [philox.normal(s, active) if active.size else np.zeros(0, np.float32) for s in seeds]
+    zs_t = [theta_normals(s, d, p) for s in seeds]
+
+    def objective(wp, th):
+        codes, tau, sw = requantize(wp, reg)
+        split = [codes[q.base:q.base + q.n].reshape(q.N, q.K) for q in reg]
+        return loss_fn(split, sw, th)
+
+    w_next, th_next, fps, fms, gs = joint_spsa_k(state.w, active, theta, [False, False, True], zs_w, zs_t, eps,
+                                                 lr, objective)
+    rec = dict(t=state.t, seeds=list(seeds), loss_plus=fps, loss_minus=fms, g=gs, k=int(active.size))
+    state.w = w_next
+    state.t += 1
+    state.log.append(rec)
+    return rec, th_next
+
+
+def bitnet_theta_loss_fn(cfg, tokens, targets, rows=None):
+    """loss_fn for ``step_joint``: minibatch loss of Eq. 7 with theta =
+    [embeddings, norm gains, LM head] passed per call."""
+    def fn(codes, sw, th):
+        per, mean = bitnet.batch_loss(cfg, codes, sw, th[0], th[1], th[2], tokens, targets, rows)
+        fn.per_sequence.append(per)
+        return mean
+
+    fn.per_sequence = []
+    return fn
 
 
 def bitnet_loss_fn(cfg, embed, gains, head, tokens, targets, rows=None):

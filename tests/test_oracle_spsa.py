@@ -162,3 +162,94 @@ def test_k_direction_update_averages_to_the_masked_gradient():
     grad = A @ w.astype(np.float64) + b
     assert np.allclose(step[active], grad[active], atol=6 * np.abs(grad).max() / math.sqrt(K) + 0.05)
     assert np.all(step[np.setdiff1d(np.arange(n), active)] == 0)
+
+
+def test_joint_theta_loops_reduce_and_are_exact_two_point_quotients():
+    """Algorithm 1 over (w, theta): with no theta it is the latent-only
+    loops; on a quadratic over the concatenated vector each g_k is the exact
+    two-point quotient of that direction's perturbed pair, and theta's
+    entries follow the same fp32 arithmetic as the latents."""
+    n_w, n_t = 24, 10
+    A, b, F = _quadratic(n_w + n_t, seed=8)
+    rng = np.random.default_rng(9)
+    w = (rng.standard_normal(n_w) * 0.1).astype(np.float32)
+    th = [(rng.standard_normal(n_t) * 0.1).astype(np.float32)]
+    active = np.sort(rng.choice(n_w, 9, replace=False)).astype(np.int64)
+    eps, lr = 1e-3, 5e-3
+    zs_w = [philox.normal(s, active) for s in (21, 22)]
+    zs_t = [termezo.theta_normals(s, n_w, n_t) for s in (21, 22)]
+    # no theta: the latent-only loops bit for bit
+    a = termezo.masked_spsa_k(w, active, zs_w, eps, lr, lambda v: F(np.concatenate([v, th[0]])))
+    j = termezo.joint_spsa_k(w, active, [], [], zs_w, [np.zeros(0, np.float32)] * 2, eps, lr,
+                             lambda v, t: F(np.concatenate([v, th[0]])))
+    assert np.array_equal(a[0], j[0]) and a[3] == j[4]
+    # joint: exact quotients on the quadratic
+    Fj = lambda v, t: F(np.concatenate([v, t[0]]))
+    w1, th1, fps, fms, gs = termezo.joint_spsa_k(w, active, th, [False], zs_w, zs_t, eps, lr, Fj)
+    e32 = np.float32(eps)
+    cw, ct = w.copy(), th[0].copy()
+    for k in range(2):
+        ew = (e32 * zs_w[k]).astype(np.float32)
+        et = (e32 * zs_t[k]).astype(np.float32)
+        wp, tp = cw.copy(), (ct + et).astype(np.float32)
+        wp[active] = (cw[active] + ew).astype(np.float32)
+        wm, tm = wp.copy(), (tp - np.float32(2) * et).astype(np.float32)
+        wm[active] = (wp[active] - np.float32(2) * ew).astype(np.float32)
+        xp = np.concatenate([wp, tp]).astype(np.float64)
+        xm = np.concatenate([wm, tm]).astype(np.float64)
+        g = (xp - xm) @ (A @ ((xp + xm) / 2) + b) / (2 * float(e32))
+        assert abs(gs[k] - g) <= 1e-9 * max(1.0, abs(g))
+        cw = wm.copy()
+        cw[active] = (wm[active] + ew).astype(np.float32)
+        ct = (tm + et).astype(np.float32)
+    lr_k = float(np.float32(lr)) / 2
+    for k in range(2):
+        c = np.float32(lr_k * gs[k])
+        cw[active] = (cw[active] - (c * zs_w[k]).astype(np.float32)).astype(np.float32)
+        ct = (ct - (c * zs_t[k]).astype(np.float32)).astype(np.float32)
+    assert np.array_equal(w1, cw) and np.array_equal(th1[0], ct)
+    assert np.array_equal(w1[np.setdiff1d(np.arange(n_w), active)], w[np.setdiff1d(np.arange(n_w), active)])
+
+
+def test_joint_theta_update_averages_to_both_gradient_blocks():
+    """Over K directions the joint update tends to -lr (m * grad_w F,
+    grad_theta F): theta is perturbed densely, the latents on the mask."""
+    n_w, n_t = 6, 3
+    A, b, F = _quadratic(n_w + n_t, seed=10)
+    w = np.linspace(-0.4, 0.4, n_w).astype(np.float32)
+    th = [np.array([0.3, -0.2, 0.1], dtype=np.float32)]
+    active = np.array([1, 4], dtype=np.int64)
+    K, eps, lr = 4000, 1e-2, 1e-3
+    seeds = range(300, 300 + K)
+    zs_w = [philox.normal(s, active) for s in seeds]
+    zs_t = [termezo.theta_normals(s, n_w, n_t) for s in seeds]
+    w1, th1, *_ = termezo.joint_spsa_k(w, active, th, [False], zs_w, zs_t, eps, lr,
+                                       lambda v, t: F(np.concatenate([v, t[0]])))
+    grad = A @ np.concatenate([w, th[0]]).astype(np.float64) + b
+    tol = 6 * np.abs(grad).max() / math.sqrt(K) + 0.05
+    step_w = (w1.astype(np.float64) - w) / -lr
+    step_t = (th1[0].astype(np.float64) - th[0]) / -lr
+    assert np.allclose(step_w[active], grad[active], atol=tol)
+    assert np.allclose(step_t, grad[n_w:], atol=tol)
+    assert np.all(step_w[np.setdiff1d(np.arange(n_w), active)] == 0)
+
+
+def test_bf16_theta_part_is_rounded_at_every_assignment():
+    """A part stored in bfloat16 (the LM head) is rounded to bfloat16 after
+    each float32 operation of Algorithm 1, so its restore need not return
+    the starting value; each step is checked by hand."""
+    from oracle import bitnet
+    th = [bitnet.bf16_round(np.array([0.0213, -0.0117, 0.5], dtype=np.float32))]
+    zt = [termezo.theta_normals(77, 4, 3)]
+    eps, lr, g = np.float32(1e-3), 1e-3, None
+    seen = []
+    w1, th1, fps, fms, gs = termezo.joint_spsa_k(np.zeros(4, np.float32), np.zeros(0, np.int64), th, [True],
+                                                 [np.zeros(0, np.float32)], zt, eps, lr,
+                                                 lambda v, t: (seen.append(t[0].copy()), float(t[0].sum()))[1])
+    e = (eps * zt[0]).astype(np.float32)
+    tp = bitnet.bf16_round((th[0] + e).astype(np.float32))
+    tm = bitnet.bf16_round((tp - np.float32(2) * e).astype(np.float32))
+    tr = bitnet.bf16_round((tm + e).astype(np.float32))
+    assert np.array_equal(seen[0], tp) and np.array_equal(seen[1], tm)
+    c = np.float32(float(np.float32(lr)) * gs[0])
+    assert np.array_equal(th1[0], bitnet.bf16_round((tr - (c * zt[0]).astype(np.float32)).astype(np.float32)))
