@@ -292,10 +292,11 @@ def run_mine(args):
 
     def do_step(i, tok, tgt):
         # one iteration of Algorithm 1 with K directions (seeds distinct per
-        # direction and step)
-        if K == 1:
+        # direction and step); --theta also trains embeddings, gains and head
+        if K == 1 and not args.theta:
             return ctx.termezo_step(synth.step_seed(i), EPS, LR, density, tok, tgt)
-        return ctx.termezo_step_k([synth.step_seed(i * K + k) for k in range(K)], EPS, LR, density, tok, tgt)
+        return ctx.termezo_step_k([synth.step_seed(i * K + k) for k in range(K)], EPS, LR, density, tok, tgt,
+                                  theta=args.theta)
 
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
@@ -364,7 +365,7 @@ def run_mine(args):
         "config": {"workload": f"{cfg.name} density {density}", "global_batch": B * world, "seq_len": S,
                    "parallelism": f"replicas{world}", "layers": cfg.layers, "hidden": cfg.hidden,
                    "density": density, "k_active": int(outs[-1]["k_active"]), "eps": EPS, "lr": LR,
-                   "directions": K,
+                   "directions": K, "theta_trained": bool(args.theta),
                    "l2": "no flush: per-step working set (521 MB packed codes, >1 GB activations) exceeds L2"},
         "steps_per_s": world * args.steps / (ms_max / 1e3),
         "roofline": {"bound": "tensor", "kernel": "k_bitlinear_gemm (tcgen05 kind::f16, exact int8 x ternary)",
@@ -508,6 +509,8 @@ def main():
     ap.add_argument("--op-density", type=float, default=0.01)
     ap.add_argument("--k-dirs", type=int, default=1,
                     help="perturbation directions per step (Algorithm 1's K, 1..8)")
+    ap.add_argument("--theta", action="store_true",
+                    help="Algorithm 1 as written: also perturb and update embeddings, norm gains and LM head")
     ap.add_argument("--op-shape", default="", help="N,K,M of the op workload's projection (default 6912,2560,2048)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()

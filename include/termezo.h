@@ -162,6 +162,22 @@ int termezo_step_k(termezo_ctx* ctx, const uint64_t* seeds, int32_t K, float eps
                    const int32_t* d_tokens, const int32_t* d_targets, termezo_step_out* out, double* losses,
                    double* g);
 
+/* Algorithm 1 as written: termezo_step_k over the masked latents and the
+ * full-precision parameters theta together.  Each direction perturbs theta
+ * densely with the same seed (+eps z, -2 eps z, restore +eps z, each pass
+ * next to the latents' requantisation), and the update applies
+ * theta -= (lr / K) g_k z_k.  theta is the embeddings (fp32), norm gains
+ * (fp32) and LM head (bf16) given to termezo_load_params, which must be
+ * writable: they are updated in place, every assignment rounded to the
+ * stored precision (the head: the float32 result rounded to bfloat16).
+ * theta's z is the Philox stream of the seed at global indices d + j, j over
+ * the embeddings, then the gains, then the head.  Needs D % 4 == 0,
+ * 16-byte aligned embeddings and gains and an 8-byte aligned head, else
+ * TERMEZO_EINVAL.  Arguments and report as termezo_step_k. */
+int termezo_step_joint(termezo_ctx* ctx, const uint64_t* seeds, int32_t K, float eps, float lr, double density,
+                       const int32_t* d_tokens, const int32_t* d_targets, termezo_step_out* out, double* losses,
+                       double* g);
+
 /* Pieces of the step, for the single-projection context and for tests.
  * termezo_shrink: Eq. 5 at the current latents (no-op before the first
  *   update); host output n_dropped (nullable).

@@ -672,10 +672,26 @@ namespace {
 // the K-term update in one pass.
 int step_impl(termezo_ctx* c, const uint64_t* seeds, int K, float eps, float lr, double density,
               const int32_t* d_tokens, const int32_t* d_targets, termezo_step_out* out, double* losses, double* gs,
-              double* per_seq_plus, double* per_seq_minus) {
+              double* per_seq_plus, double* per_seq_minus, bool theta) {
   if (!c || !seeds || !d_tokens || !d_targets || !out) return TERMEZO_EINVAL;
   if (K < 1 || K > tmz::KMAX) return TERMEZO_EINVAL;
   if (c->sh.op || !c->built) return TERMEZO_ESTATE;
+  tmz::ThetaArgs th{};
+  if (theta) {
+    // theta is updated in place in the caller's buffers of termezo_load_params
+    const Shape& s = c->sh;
+    if (!c->embed || !c->gains || !c->head || s.D % 4 || ((uintptr_t)c->embed & 15) || ((uintptr_t)c->gains & 15) ||
+        ((uintptr_t)c->head & 7) || s.d % 4)
+      return TERMEZO_EINVAL;
+    th.emb = const_cast<float*>(c->embed);
+    th.n_emb = (uint64_t)s.V * s.D;
+    th.gains = const_cast<float*>(c->gains);
+    th.n_gains = (uint64_t)(2 * s.L + 1) * s.D;
+    th.head = const_cast<uint16_t*>(c->head);
+    th.n_head = (uint64_t)s.V * s.D;
+    th.d = s.d;
+  }
+  const double theta8 = theta ? 2.0 * (4.0 * (th.n_emb + th.n_gains) + 2.0 * th.n_head) : 0.0;
   if (!(eps > 0.f) || !std::isfinite(lr)) return TERMEZO_EINVAL;
   const int warn = (density != c->density) ? TERMEZO_WMASKFIXED : TERMEZO_OK;
   cudaStream_t st = c->stream;
@@ -700,11 +716,19 @@ int step_impl(termezo_ctx* c, const uint64_t* seeds, int K, float eps, float lr,
       ProfScope ps(c, 2, k8);
       tmz::sparse_requant(c->ma, c->cur, seed, eps, +1, st);
     }
+    if (theta) {
+      ProfScope ps(c, 2, theta8);
+      tmz::theta_pm(th, seed, eps, 0, st);
+    }
     rc = run_forward(c, d_tokens, d_targets, c->ma.sw_plus, 0);
     if (rc) return rc;
     {
       ProfScope ps(c, 2, k8);
       tmz::sparse_requant(c->ma, c->cur, seed, eps, -1, st);
+    }
+    if (theta) {
+      ProfScope ps(c, 2, theta8);
+      tmz::theta_pm(th, seed, eps, 1, st);
     }
     rc = run_forward(c, d_tokens, d_targets, c->ma.sw_minus, 1);
     if (rc) return rc;
@@ -715,12 +739,17 @@ int step_impl(termezo_ctx* c, const uint64_t* seeds, int K, float eps, float lr,
       ProfScope ps(c, 2, 1.5 * k8);
       tmz::sparse_restore(c->ma, c->cur, seed, eps, st);
       c->pm_valid = false;
+      if (theta) tmz::theta_pm(th, seed, eps, 0, st);
     }
   }
   dirs.last = seeds[K - 1];
   {
     ProfScope ps(c, 2, 1.5 * k8);
     tmz::sparse_update_dirs(c->ma, c->cur, dirs, eps, lr, c->g, st);
+  }
+  if (theta) {
+    ProfScope ps(c, 2, theta8);
+    tmz::theta_update(th, dirs, eps, lr, c->g, st);
   }
   c->pm_valid = false;
   struct {
@@ -761,13 +790,19 @@ int step_impl(termezo_ctx* c, const uint64_t* seeds, int K, float eps, float lr,
 int termezo_step(termezo_ctx* c, uint64_t seed, float eps, float lr, double density, const int32_t* d_tokens,
                  const int32_t* d_targets, termezo_step_out* out, double* per_seq_plus, double* per_seq_minus) {
   return step_impl(c, &seed, 1, eps, lr, density, d_tokens, d_targets, out, nullptr, nullptr, per_seq_plus,
-                   per_seq_minus);
+                   per_seq_minus, false);
 }
 
 int termezo_step_k(termezo_ctx* c, const uint64_t* seeds, int32_t K, float eps, float lr, double density,
                    const int32_t* d_tokens, const int32_t* d_targets, termezo_step_out* out, double* losses,
                    double* g) {
-  return step_impl(c, seeds, K, eps, lr, density, d_tokens, d_targets, out, losses, g, nullptr, nullptr);
+  return step_impl(c, seeds, K, eps, lr, density, d_tokens, d_targets, out, losses, g, nullptr, nullptr, false);
+}
+
+int termezo_step_joint(termezo_ctx* c, const uint64_t* seeds, int32_t K, float eps, float lr, double density,
+                       const int32_t* d_tokens, const int32_t* d_targets, termezo_step_out* out, double* losses,
+                       double* g) {
+  return step_impl(c, seeds, K, eps, lr, density, d_tokens, d_targets, out, losses, g, nullptr, nullptr, true);
 }
 
 int termezo_shrink(termezo_ctx* c, uint64_t* n_dropped) {

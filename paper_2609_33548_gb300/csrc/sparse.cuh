@@ -53,6 +53,24 @@ struct UpdateDirs {
   uint64_t last;  // seed[K - 1]
   int K;
 };
+// The full-precision parameters theta (device pointers the caller owns):
+// embeddings fp32 [n_emb], norm gains fp32 [n_gains], LM head bf16 [n_head];
+// all sizes and d multiples of 4, fp32 parts 16-byte and the head 8-byte
+// aligned.
+struct ThetaArgs {
+  float* emb;
+  uint64_t n_emb;
+  float* gains;
+  uint64_t n_gains;
+  uint16_t* head;
+  uint64_t n_head;
+  uint64_t d;  // latents: theta's z is the Philox stream at indices d + j
+};
+// theta += e (mode 0: the + pass and the restore) or theta -= 2 e (mode 1).
+void theta_pm(const ThetaArgs& t, uint64_t seed, float eps, int mode, cudaStream_t s);
+// The last direction's restore, then theta -= (lr / K) g_k z_k for each k.
+void theta_update(const ThetaArgs& t, const UpdateDirs& d, float eps, float lr, const double* g_dev, cudaStream_t s);
+
 // Restore after direction seed: w = fl(fl(fl(w + e) - 2 e) + e), e = fl(eps z).
 void sparse_restore(const MaskArgs& a, int cur, uint64_t seed, float eps, cudaStream_t s);
 // Restore after the last direction, then w = fl(w - fl(c_k z_k)) for k = 0..K-1

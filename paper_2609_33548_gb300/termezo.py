@@ -20,7 +20,7 @@ OK, WMASKFIXED, EINVAL, ESTATE, ENOMEM, ECUDA, ETIMEOUT = 0, 1, -1, -2, -3, -4, 
 # Every function declared in include/termezo.h.
 EXPORTS = (
     "termezo_workspace_bytes", "termezo_memory", "termezo_create", "termezo_load_params", "termezo_build_mask",
-    "termezo_forward_loss", "termezo_step", "termezo_step_k", "termezo_shrink", "termezo_requantize", "termezo_update",
+    "termezo_forward_loss", "termezo_step", "termezo_step_k", "termezo_step_joint", "termezo_shrink", "termezo_requantize", "termezo_update",
     "termezo_bitlinear", "termezo_state_sizes", "termezo_export_state", "termezo_normal",
     "termezo_absmean_noalloc", "termezo_attention", "termezo_profile", "termezo_destroy", "termezo_strerror",
 )
@@ -96,6 +96,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         "termezo_forward_loss": (I32, [P, P, P, ctypes.POINTER(F64), P]),
         "termezo_step": (I32, [P, U64, F32, F32, F64, P, P, ctypes.POINTER(StepOut), P, P]),
         "termezo_step_k": (I32, [P, P, I32, F32, F32, F64, P, P, ctypes.POINTER(StepOut), P, P]),
+        "termezo_step_joint": (I32, [P, P, I32, F32, F32, F64, P, P, ctypes.POINTER(StepOut), P, P]),
         "termezo_shrink": (I32, [P, ctypes.POINTER(U64)]),
         "termezo_requantize": (I32, [P, U64, F32, I32]),
         "termezo_update": (I32, [P, U64, F32, F32, F64]),
@@ -219,18 +220,21 @@ class Context:
         d["per_seq_plus"], d["per_seq_minus"], d["status"] = pp, pm, st
         return d
 
-    def termezo_step_k(self, seeds, eps: float, lr: float, density: float, tokens, targets):
+    def termezo_step_k(self, seeds, eps: float, lr: float, density: float, tokens, targets, theta=False):
         """Algorithm 1 with K = len(seeds) directions; adds per-direction
-        losses [K, 2] (F+, F-) and g [K] to the report."""
+        losses [K, 2] (F+, F-) and g [K] to the report.  theta=True also
+        perturbs and updates the embeddings, norm gains and LM head in place
+        (termezo_step_joint)."""
         K = len(seeds)
         sd = np.asarray(seeds, dtype=np.uint64)
         out = StepOut()
         losses = np.zeros(2 * K, dtype=np.float64)
         g = np.zeros(K, dtype=np.float64)
-        st = load().termezo_step_k(self.handle, sd.ctypes.data_as(ctypes.c_void_p), K, eps, lr, density,
-                                   _ptr(tokens), _ptr(targets), ctypes.byref(out),
-                                   losses.ctypes.data_as(ctypes.c_void_p), g.ctypes.data_as(ctypes.c_void_p))
-        _check("termezo_step_k", st, allow=(OK, WMASKFIXED))
+        fn = "termezo_step_joint" if theta else "termezo_step_k"
+        st = getattr(load(), fn)(self.handle, sd.ctypes.data_as(ctypes.c_void_p), K, eps, lr, density,
+                                 _ptr(tokens), _ptr(targets), ctypes.byref(out),
+                                 losses.ctypes.data_as(ctypes.c_void_p), g.ctypes.data_as(ctypes.c_void_p))
+        _check(fn, st, allow=(OK, WMASKFIXED))
         d = out.as_dict()
         d["losses"], d["g_k"], d["status"] = losses.reshape(K, 2), g, st
         return d

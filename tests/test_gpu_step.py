@@ -229,3 +229,75 @@ def test_single_direction_step_k_is_step(inputs):
     assert (oa["loss_plus"], oa["loss_minus"], oa["g"]) == (ob["loss_plus"], ob["loss_minus"], ob["g"])
     sa, sb = a.termezo_export_state(packed=False), b.termezo_export_state(packed=False)
     np.testing.assert_array_equal(sa["latents"].view(np.uint32), sb["latents"].view(np.uint32))
+
+
+def test_joint_theta_step_matches_oracle(inputs):
+    """Algorithm 1 as written (termezo_step_joint, K = 2): the masked
+    latents and theta (embeddings, norm gains fp32, LM head bf16) perturbed
+    together.  Per-direction F+- and g_k against the oracle's ensembles at
+    the oracle's own (codes, theta+-); latents and theta after the update
+    against the oracle's arithmetic with the GPU's g_k.  theta's z differs
+    from the oracle's by a few ulp, so fp32 parts agree within the restore
+    rounding and the bf16 head in all but a rare element that rounds to a
+    neighbouring bf16 value."""
+    K = 2
+    w0, emb0, gains0, head0, tok, tgt, cfg = inputs
+    ctx, dev = _gpu_ctx(inputs)
+    ctx.termezo_build_mask(DENSITY)
+    reg = otz.registry(cfg)
+    state = otz.build(w0.numpy(), reg, DENSITY)
+    act = state.active.copy()
+    seeds = [synth.step_seed(40 + k) for k in range(K)]
+    out = ctx.termezo_step_k(seeds, EPS, LR, DENSITY, dev[4], dev[5], theta=True)
+    th0 = [emb0.numpy(), gains0.numpy(), head0.float().numpy()]
+    fn = otz.bitnet_theta_loss_fn(cfg, tok.numpy(), tgt.numpy())
+    rec, th_oracle = otz.step_joint(state, th0, fn, seeds, EPS, LR)
+    eps32 = np.float32(EPS)
+    d, p = w0.numel(), sum(t.size for t in th0)
+    bf = [False, False, True]
+    offs = np.cumsum([0] + [t.size for t in th0])
+    split = lambda z: [z[offs[i]:offs[i + 1]].reshape(th0[i].shape) for i in range(3)]
+    w, th = w0.numpy().copy(), [t.copy() for t in th0]
+    zs_w, zs_t = [], []
+    for k, seed in enumerate(seeds):
+        zw, zt = philox.normal(seed, act), otz.theta_normals(seed, d, p)
+        zs_w.append(zw)
+        zs_t.append(zt)
+        ew = (eps32 * zw).astype(np.float32)
+        et = [(eps32 * z).astype(np.float32) for z in split(zt)]
+        wp = w.copy(); wp[act] = (w[act] + ew).astype(np.float32)
+        thp = [otz._stored(t + e, b) for t, e, b in zip(th, et, bf)]
+        wm = wp.copy(); wm[act] = (wp[act] - np.float32(2) * ew).astype(np.float32)
+        thm = [otz._stored(t - np.float32(2) * e, b) for t, e, b in zip(thp, et, bf)]
+        cp, _, swp = otz.requantize(wp, reg)
+        cm, _, swm = otz.requantize(wm, reg)
+        tt = (tok.numpy(), tgt.numpy())
+        lp = rounding.loss_ensemble(cfg, (_split(cp, reg), swp), (*thp, *tt), n=4).mean(axis=1)
+        lm = rounding.loss_ensemble(cfg, (_split(cm, reg), swm), (*thm, *tt), n=4).mean(axis=1)
+        fp, fm = out["losses"][k]
+        assert rounding.within(fp, rec["loss_plus"][k], lp), (k, fp, rec["loss_plus"][k], lp)
+        assert rounding.within(fm, rec["loss_minus"][k], lm), (k, fm, rec["loss_minus"][k], lm)
+        ens = (lp - lm) / (2 * float(eps32))
+        assert rounding.g_within_ensemble(out["g_k"][k], rec["g"][k], ens), (k, out["g_k"][k], rec["g"][k], ens)
+        w = wm.copy(); w[act] = (wm[act] + ew).astype(np.float32)
+        th = [otz._stored(t + e, b) for t, e, b in zip(thm, et, bf)]
+    # the update with the GPU's g_k
+    lr_k = float(np.float32(LR)) / K
+    for zw, zt, g in zip(zs_w, zs_t, out["g_k"]):
+        c = np.float32(lr_k * g)
+        w[act] = (w[act] - (c * zw).astype(np.float32)).astype(np.float32)
+        th = [otz._stored(t - (c * z).astype(np.float32), b) for t, z, b in zip(th, split(zt), bf)]
+    st = ctx.termezo_export_state(packed=False)
+    np.testing.assert_array_equal(st["idx"], act.astype(np.uint32))
+    emax = float(np.abs(eps32 * np.concatenate(zs_w)).max())
+    assert np.all(np.abs(st["latents"].astype(np.float64) - w[act]) <= K * 1e-5 * (np.abs(w0.numpy()[act]) + 2 * emax))
+    got = [dev[1].cpu().numpy(), dev[2].cpu().numpy(), dev[3].cpu().float().numpy()]
+    for i in range(2):
+        emax_t = 2 * float(np.abs(eps32 * np.concatenate([split(z)[i].ravel() for z in zs_t])).max())
+        assert np.all(np.abs(got[i].astype(np.float64) - th[i]) <= K * 1e-5 * (np.abs(th0[i]) + emax_t)), i
+        assert not np.array_equal(got[i], th0[i])          # theta did move
+    diff = np.abs(got[2].astype(np.float64) - th[2])
+    ulp = np.abs(th[2]).astype(np.float64) * 2.0 ** -7 + 1e-30
+    assert np.count_nonzero(diff) <= max(3, int(1e-4 * diff.size)), np.count_nonzero(diff)
+    assert np.all(diff <= 2 * ulp)
+    assert not np.array_equal(got[2], th0[2])
