@@ -119,11 +119,30 @@ def initial_mask(w: np.ndarray, reg, rho0: float):
     return sel, xi0, k0, tau
 
 
-def shrink(w: np.ndarray, reg, active: np.ndarray, xi0):
-    """Eq. 5: members of S_{t-1} whose distance at tau_t is <= xi_0."""
+def initial_mask_per_tensor(w: np.ndarray, reg, rho0: float):
+    """The per-tensor variant of Eq. 4: every projection l keeps its own
+    floor(rho_0 n_l) smallest (d_i, i) pairs (ties to the lower index), and
+    xi_0^l is that projection's quantile.  Returns (S_0 sorted, xi_0 [P]
+    float32, k0 = sum of the k_l, tau_0)."""
     _, tau, _ = thresholds(w, reg)
     d = all_distances(w, reg, tau)
-    keep = d[active] <= np.float32(xi0)
+    sels, xis = [], []
+    for p in reg:
+        sel, xi = select_smallest(d[p.base:p.base + p.n], keep_count(rho0, p.n))
+        sels.append(sel + p.base)
+        xis.append(xi)
+    sel = np.concatenate(sels).astype(np.int64) if sels else np.zeros(0, np.int64)
+    return sel, np.array(xis, dtype=np.float32), int(sel.size), tau
+
+
+def shrink(w: np.ndarray, reg, active: np.ndarray, xi0):
+    """Eq. 5: members of S_{t-1} whose distance at tau_t is <= xi_0 (a
+    scalar, or one xi_0^l per projection for the per-tensor mask)."""
+    _, tau, _ = thresholds(w, reg)
+    d = all_distances(w, reg, tau)
+    xi = np.asarray(xi0, dtype=np.float32)
+    thr = xi[_tensor_of(reg, active)] if xi.ndim else xi
+    keep = d[active] <= thr
     return active[keep], tau
 
 
@@ -254,8 +273,10 @@ class State:
     log: list = field(default_factory=list)
 
 
-def build(w0: np.ndarray, reg, rho0: float) -> State:
-    active, xi0, k0, tau0 = initial_mask(w0, reg, rho0)
+def build(w0: np.ndarray, reg, rho0: float, per_tensor: bool = False) -> State:
+    """Oracle state after the initial mask: the global quantile of Eq. 4, or
+    its per-tensor variant (xi_0 then holds one value per projection)."""
+    active, xi0, k0, tau0 = (initial_mask_per_tensor if per_tensor else initial_mask)(w0, reg, rho0)
     codes0 = np.concatenate([ternary.quantize(v, tau0[j]) for j, v in enumerate(views(w0, reg))])
     return State(w=w0.astype(np.float32).copy(), reg=reg, active=active, xi0=xi0,
                  k0=k0, frozen_code=codes0)

@@ -1,10 +1,13 @@
 """Pins of the oracle's mask rules (Eqs. 4-5, Algorithm 1): cardinality,
 quantile order, index tie-break, global selection across projections,
 nesting S_t within S_{t-1}, frozen weights keeping their code.  CPU only."""
+import math
+
 import numpy as np
 import pytest
 
 from oracle import ternary, termezo
+from paper_2609_33548_gb300 import synth
 
 
 def _reg(sizes):
@@ -113,3 +116,50 @@ def test_step_keeps_frozen_weights_and_codes():
         assert rec["n_jumps"] == 0
         assert rec["k"] == st.active.size <= prev.size
         prev = st.active
+
+
+def test_per_tensor_mask_cardinality_and_order_within_each_projection():
+    """Per-tensor variant of Eq. 4: projection l keeps floor(rho_0 n_l) of its
+    own smallest (d, i); within it every kept distance <= xi_0^l <= every
+    dropped one, ties to the lower index; one projection is the global rule."""
+    cfg = synth.TINY
+    reg = termezo.registry(cfg)
+    w = synth.latents(cfg).numpy()
+    rho = 0.013
+    sel, xi, k0, tau = termezo.initial_mask_per_tensor(w, reg, rho)
+    d = termezo.all_distances(w, reg, tau)
+    assert xi.shape == (len(reg),) and np.all(np.diff(sel) > 0)
+    total = 0
+    for j, p in enumerate(reg):
+        inside = sel[(sel >= p.base) & (sel < p.base + p.n)]
+        assert inside.size == math.floor(rho * p.n)
+        total += inside.size
+        dp = d[p.base:p.base + p.n]
+        mask = np.zeros(p.n, bool)
+        mask[inside - p.base] = True
+        assert dp[mask].max() == xi[j] and np.all(dp[~mask] >= xi[j])
+        ties = np.flatnonzero(dp == xi[j])
+        assert np.all(np.flatnonzero(mask & (dp == xi[j])) == ties[:np.count_nonzero(mask & (dp == xi[j]))])
+    assert total == k0
+    one = termezo.single_registry(688, 256)
+    w1 = w[:688 * 256]
+    a = termezo.initial_mask(w1, one, rho)
+    b = termezo.initial_mask_per_tensor(w1, one, rho)
+    assert np.array_equal(a[0], b[0]) and a[1] == b[1][0] and a[2] == b[2]
+
+
+def test_per_tensor_shrink_uses_each_projections_xi():
+    """Eq. 5 with the per-tensor xi_0^l: a weight is kept iff its distance is
+    within its own projection's xi_0^l; the sets nest."""
+    cfg = synth.TINY
+    reg = termezo.registry(cfg)
+    w = synth.latents(cfg).numpy()
+    state = termezo.build(w, reg, 0.02, per_tensor=True)
+    rng = np.random.default_rng(3)
+    w2 = (w + rng.standard_normal(w.size).astype(np.float32) * np.float32(2e-4)).astype(np.float32)
+    kept, tau = termezo.shrink(w2, reg, state.active, state.xi0)
+    d = termezo.all_distances(w2, reg, tau)
+    tj = termezo._tensor_of(reg, state.active)
+    expect = state.active[d[state.active] <= state.xi0[tj]]
+    assert np.array_equal(kept, expect) and kept.size < state.active.size
+    assert np.all(np.isin(kept, state.active))
