@@ -124,6 +124,18 @@ int termezo_load_params(termezo_ctx* ctx, const float* d_latents, const float* d
  * density must not exceed the one given to termezo_create.  Synchronises. */
 int termezo_build_mask(termezo_ctx* ctx, double density, uint64_t* k0, float* xi0);
 
+/* Mask rules: the global quantile of Eq. 4 (termezo_build_mask), or its
+ * per-tensor variant, in which every projection l keeps its own
+ * floor(rho_0 n_l) smallest (d_i, i) pairs (ties to the lower index) and has
+ * its own xi_0^l, used by its shrink (Eq. 5). */
+enum { TERMEZO_MASK_GLOBAL = 0, TERMEZO_MASK_PER_TENSOR = 1 };
+
+/* termezo_build_mask with a mask rule.  Host outputs: k0 (the total kept),
+ * xi0: one float for TERMEZO_MASK_GLOBAL, [n_proj] floats (xi_0 of every
+ * projection, 0 where a projection keeps none) for TERMEZO_MASK_PER_TENSOR;
+ * nullable.  Synchronises. */
+int termezo_build_mask_rule(termezo_ctx* ctx, double density, int32_t rule, uint64_t* k0, float* xi0);
+
 /* Minibatch loss F(Q(w_t), theta; B) (Eqs. 6-7) at the current latents:
  * requantises the active weights, runs the BitNet forward.  d_tokens int32
  * [batch, seq]; d_targets int32 (see loss_mode).  Host outputs: loss, and

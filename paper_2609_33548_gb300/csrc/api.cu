@@ -218,8 +218,10 @@ void carve(termezo_ctx* c, Carver& cv) {
   float** fl[9] = {&a.gamma_cur, &a.tau_cur, &a.sw_cur, &a.gamma_plus, &a.tau_plus,
                    &a.sw_plus,   &a.gamma_minus, &a.tau_minus, &a.sw_minus};
   for (auto f : fl) *f = cv.take<float>(P + 2);
-  a.hist = cv.take<unsigned long long>(2048);
-  a.sel = cv.take<tmz::SelectState>(1);
+  a.hist = cv.take<unsigned long long>(2048 * (size_t)P);
+  a.sel = cv.take<tmz::SelectState>(P);
+  a.grp_tie0 = cv.take<unsigned long long>(P);
+  a.xi0p = cv.take<float>(P);
   a.blk_a = cv.take<uint32_t>(nblk);
   a.blk_b = cv.take<uint32_t>(nblk);
   a.blk_c = cv.take<uint32_t>(nblk);
@@ -448,7 +450,7 @@ void ensure_pm(termezo_ctx* c, uint64_t seed, float eps) {
 
 int do_shrink(termezo_ctx* c) {
   ProfScope ps(c, 2, 3.0 * 8.0 * (double)c->k_active);
-  tmz::sparse_shrink(c->ma, c->cur, c->xi0, c->d_total, c->stream);
+  tmz::sparse_shrink(c->ma, c->cur, c->d_total, c->stream);
   c->cur ^= 1;
   c->pm_valid = false;
   return cuda_status(c);
@@ -589,22 +591,41 @@ int termezo_load_params(termezo_ctx* c, const float* d_latents, const float* d_e
 }
 
 int termezo_build_mask(termezo_ctx* c, double density, uint64_t* k0_out, float* xi0_out) {
+  return termezo_build_mask_rule(c, density, TERMEZO_MASK_GLOBAL, k0_out, xi0_out);
+}
+
+int termezo_build_mask_rule(termezo_ctx* c, double density, int32_t rule, uint64_t* k0_out, float* xi0_out) {
   if (!c) return TERMEZO_EINVAL;
   if (!c->latents) return TERMEZO_ESTATE;
   if (!(density > 0.0 && density <= 1.0)) return TERMEZO_EINVAL;
-  const uint64_t k0 = keep_count(density, c->sh.d);
-  if (k0 > keep_count(c->density, c->sh.d)) return TERMEZO_EINVAL;
+  if (rule != TERMEZO_MASK_GLOBAL && rule != TERMEZO_MASK_PER_TENSOR) return TERMEZO_EINVAL;
   const Shape& s = c->sh;
+  // one selection group for the global quantile, one per projection else
+  std::vector<tmz::SelectState> groups;
+  uint64_t k0 = 0;
+  if (rule == TERMEZO_MASK_GLOBAL) {
+    k0 = keep_count(density, s.d);
+    groups.push_back(tmz::SelectState{k0, 0u, 0u});
+  } else {
+    for (int p = 0; p < s.P; ++p) {
+      const uint64_t kp = keep_count(density, s.base[p + 1] - s.base[p]);
+      groups.push_back(tmz::SelectState{kp, 0u, 0u});
+      k0 += kp;
+    }
+  }
+  if (k0 > keep_count(c->density, s.d)) return TERMEZO_EINVAL;
   cudaStream_t st = c->stream;
-  tmz::SelectState sel{k0, 0u, 0u};
-  cudaMemcpyAsync(c->ma.sel, &sel, sizeof(sel), cudaMemcpyHostToDevice, st);
-  cudaMemsetAsync(c->ma.hist, 0, 2048 * sizeof(unsigned long long), st);
+  c->ma.groups = (int)groups.size();
+  std::vector<tmz::SelectState> sel_h = groups;
+  cudaMemcpyAsync(c->ma.sel, sel_h.data(), groups.size() * sizeof(tmz::SelectState), cudaMemcpyHostToDevice, st);
+  cudaMemsetAsync(c->ma.hist, 0, groups.size() * 2048 * sizeof(unsigned long long), st);
   tmz::mask_build(c->ma, c->latents, k0, st);
   int rc = cuda_status(c);
   if (rc) return rc;
   std::vector<uint32_t> off(s.P + 1);
+  std::vector<float> xi0p(s.P);
   cudaMemcpyAsync(off.data(), c->ma.off[0], (s.P + 1) * sizeof(uint32_t), cudaMemcpyDeviceToHost, st);
-  cudaMemcpyAsync(&sel, c->ma.sel, sizeof(sel), cudaMemcpyDeviceToHost, st);
+  cudaMemcpyAsync(xi0p.data(), c->ma.xi0p, s.P * sizeof(float), cudaMemcpyDeviceToHost, st);
   rc = sync_status(c);
   if (rc) return rc;
   if (off[s.P] != k0) {
@@ -628,10 +649,7 @@ int termezo_build_mask(termezo_ctx* c, double density, uint64_t* k0_out, float* 
   c->cur = 0;
   c->k0 = k0;
   c->k_active = k0;
-  uint32_t key = sel.prefix;
-  float xi0 = 0.f;
-  if (k0) memcpy(&xi0, &key, 4);
-  c->xi0 = xi0;
+  c->xi0 = rule == TERMEZO_MASK_GLOBAL ? xi0p[0] : 0.f;
   c->t = 0;
   c->updated = false;
   c->pm_valid = false;
@@ -642,7 +660,12 @@ int termezo_build_mask(termezo_ctx* c, double density, uint64_t* k0_out, float* 
   // the dense latents are not read again: the caller may release them
   c->latents = nullptr;
   if (k0_out) *k0_out = k0;
-  if (xi0_out) *xi0_out = xi0;
+  if (xi0_out) {
+    if (rule == TERMEZO_MASK_GLOBAL)
+      *xi0_out = xi0p[0];
+    else
+      for (int p = 0; p < s.P; ++p) xi0_out[p] = xi0p[p];
+  }
   return TERMEZO_OK;
 }
 

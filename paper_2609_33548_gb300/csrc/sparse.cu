@@ -155,7 +155,9 @@ __global__ void __launch_bounds__(TPB) k_hist(MaskArgs a, const float* __restric
   __syncthreads();
   const DenseRange r = dense_range(a, blockIdx.x);
   const float tau = a.tau_cur[r.proj];
-  const uint32_t prefix = a.sel->prefix;
+  const int grp = a.groups > 1 ? r.proj : 0;
+  const uint32_t prefix = a.sel[grp].prefix;
+  unsigned long long* hist = a.hist + (size_t)grp * 2048;
   float v[16];
   const uint64_t i0 = r.start + 16ull * threadIdx.x;
   const int n = i0 < r.end ? 16 : 0;
@@ -172,37 +174,45 @@ __global__ void __launch_bounds__(TPB) k_hist(MaskArgs a, const float* __restric
     for (int i = threadIdx.x; i < NB0; i += TPB) {
       uint32_t t = 0;
       for (int ww = 0; ww < TPB / 32; ++ww) t += h[ww * NB0 + i];
-      if (t) atomicAdd(&a.hist[i], (unsigned long long)t);
+      if (t) atomicAdd(&hist[i], (unsigned long long)t);
     }
   } else {
     for (int i = threadIdx.x; i < 2048; i += TPB)
-      if (h[i]) atomicAdd(&a.hist[i], (unsigned long long)h[i]);
+      if (h[i]) atomicAdd(&hist[i], (unsigned long long)h[i]);
   }
 }
 
 // Picks the radix bin that holds the krem-th smallest key (1-based).
+// One block per selection group: the radix bin holding the group's rank.
 __global__ void k_select(MaskArgs a, int pass) {
+  SelectState* sel = a.sel + blockIdx.x;
+  unsigned long long* hist = a.hist + (size_t)blockIdx.x * 2048;
   if (threadIdx.x == 0) {
     const int bins = pass < 2 ? 2048 : 1024;
     const int bits = pass < 2 ? 11 : 10;
-    unsigned long long cum = 0, krem = a.sel->krem;
+    unsigned long long cum = 0, krem = sel->krem;
     int B = bins - 1;
     for (int i = 0; i < bins; ++i) {
-      if (cum + a.hist[i] >= krem) { B = i; break; }
-      cum += a.hist[i];
+      if (cum + hist[i] >= krem) { B = i; break; }
+      cum += hist[i];
     }
-    a.sel->krem = krem - cum;
-    a.sel->prefix = pass == 0 ? (uint32_t)B : ((a.sel->prefix << bits) | (uint32_t)B);
+    sel->krem = krem - cum;
+    sel->prefix = pass == 0 ? (uint32_t)B : ((sel->prefix << bits) | (uint32_t)B);
   }
   __syncthreads();
-  for (int i = threadIdx.x; i < 2048; i += blockDim.x) a.hist[i] = 0;
+  for (int i = threadIdx.x; i < 2048; i += blockDim.x) hist[i] = 0;
+}
+
+// xi_0 of every projection: the key its group's selection ended on.
+__global__ void k_xi0(MaskArgs a) {
+  for (int p = threadIdx.x; p < a.P; p += blockDim.x) a.xi0p[p] = __uint_as_float(a.sel[a.groups > 1 ? p : 0].prefix);
 }
 
 __global__ void __launch_bounds__(TPB) k_count(MaskArgs a, const float* __restrict__ w) {
   __shared__ uint32_t sh[TPB / 32];
   const DenseRange r = dense_range(a, blockIdx.x);
   const float tau = a.tau_cur[r.proj];
-  const uint32_t key_p = a.sel->prefix;
+  const uint32_t key_p = a.sel[a.groups > 1 ? r.proj : 0].prefix;
   uint32_t less = 0, eq = 0;
   float v[16];
   const uint64_t i0 = r.start + 16ull * threadIdx.x;
@@ -240,32 +250,48 @@ __device__ __forceinline__ unsigned long long scan1024(unsigned long long v, uns
   return sh[threadIdx.x] - v;  // exclusive
 }
 
+// Single block over the dense blocks in order: per block b, the selected
+// weights before it (blk_c, a position in the sorted store) and the ties of
+// its group before it (blk_d); group g selects the first sel[g].krem ties in
+// index order.  Groups are runs of consecutive blocks (one projection each,
+// or all of them).
 __global__ void __launch_bounds__(1024) k_scan_dense(MaskArgs a, uint32_t nblk) {
   __shared__ unsigned long long sh[1024];
-  const unsigned long long ties = a.sel->krem;
   const uint32_t per = (nblk + 1023) / 1024;
   const uint32_t b0 = min(nblk, threadIdx.x * per), b1 = min(nblk, b0 + per);
+  auto group = [&](uint32_t b) { return a.groups > 1 ? (int)a.dproj[b] : 0; };
   unsigned long long eq = 0;
   for (uint32_t b = b0; b < b1; ++b) eq += a.blk_b[b];
   const unsigned long long tie_start = scan1024(eq, sh);
-  unsigned long long tie_before = tie_start, sel = 0;
+  // ties before the first block of each group
+  unsigned long long tb = tie_start;
   for (uint32_t b = b0; b < b1; ++b) {
-    const unsigned long long e = a.blk_b[b];
-    unsigned long long take = tie_before >= ties ? 0 : (ties - tie_before);
+    const int g = group(b);
+    if (b == (a.groups > 1 ? a.dpre[g] : 0u)) a.grp_tie0[g] = tb;
+    tb += a.blk_b[b];
+  }
+  __syncthreads();
+  unsigned long long sel = 0;
+  tb = tie_start;
+  for (uint32_t b = b0; b < b1; ++b) {
+    const int g = group(b);
+    const unsigned long long in = tb - a.grp_tie0[g], ties = a.sel[g].krem, e = a.blk_b[b];
+    unsigned long long take = in >= ties ? 0 : (ties - in);
     if (take > e) take = e;
     sel += a.blk_a[b] + take;
-    tie_before += e;
+    tb += e;
   }
   unsigned long long sel_before = scan1024(sel, sh);
-  tie_before = tie_start;
+  tb = tie_start;
   for (uint32_t b = b0; b < b1; ++b) {
+    const int g = group(b);
+    const unsigned long long in = tb - a.grp_tie0[g], ties = a.sel[g].krem, e = a.blk_b[b];
     a.blk_c[b] = (uint32_t)sel_before;
-    a.blk_d[b] = (uint32_t)tie_before;
-    const unsigned long long e = a.blk_b[b];
-    unsigned long long take = tie_before >= ties ? 0 : (ties - tie_before);
+    a.blk_d[b] = (uint32_t)in;
+    unsigned long long take = in >= ties ? 0 : (ties - in);
     if (take > e) take = e;
     sel_before += a.blk_a[b] + take;
-    tie_before += e;
+    tb += e;
   }
 }
 
@@ -274,8 +300,9 @@ __global__ void __launch_bounds__(TPB) k_compact(MaskArgs a, const float* __rest
   __shared__ uint32_t sh[TPB / 32];
   const DenseRange r = dense_range(a, blockIdx.x);
   const float tau = a.tau_cur[r.proj];
-  const uint32_t key_p = a.sel->prefix;
-  const unsigned long long ties = a.sel->krem;
+  const SelectState sg = a.sel[a.groups > 1 ? r.proj : 0];
+  const uint32_t key_p = sg.prefix;
+  const unsigned long long ties = sg.krem;
   const uint64_t i0 = r.start + 16ull * threadIdx.x;
   const bool live = i0 < r.end;
   float v[16];
@@ -513,13 +540,14 @@ __global__ void __launch_bounds__(TPB) k_sparse_restore(MaskArgs a, int cur, uin
 
 // Eq. 5 at tau_cur: marks dropped weights, writes their code at tau_cur,
 // sums their |w| and counts the kept ones per block.
-__global__ void __launch_bounds__(TPB) k_shrink_mark(MaskArgs a, int cur, float xi0) {
+__global__ void __launch_bounds__(TPB) k_shrink_mark(MaskArgs a, int cur) {
   __shared__ ExactSum red[TPB / 32];
   __shared__ uint32_t sh[TPB / 32];
   const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
   const uint32_t* idx = a.idx[cur];
   const float* lat = a.lat[cur];
   const float tau = a.tau_cur[r.proj];
+  const float xi0 = a.xi0p[r.proj];
   ExactAcc acc;
   ea_zero(acc);
   uint32_t kept = 0, dropped = 0;
@@ -585,10 +613,11 @@ __global__ void __launch_bounds__(1024) k_scan_simple(MaskArgs a, uint32_t n, ui
   }
 }
 
-__global__ void __launch_bounds__(TPB) k_shrink_scatter(MaskArgs a, int cur, float xi0) {
+__global__ void __launch_bounds__(TPB) k_shrink_scatter(MaskArgs a, int cur) {
   __shared__ uint32_t sh[TPB / 32];
   const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
   const float tau = a.tau_cur[r.proj];
+  const float xi0 = a.xi0p[r.proj];
   uint32_t pos = a.blk_c[blockIdx.x];
   for (uint32_t base = r.beg; base < r.end; base += TPB) {
     const uint32_t e = base + threadIdx.x;
@@ -628,18 +657,19 @@ __global__ void k_normal(uint64_t seed, const uint32_t* idx, uint64_t n, float* 
 // ----------------------------------------------------------- host side ----
 
 void mask_build(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_t s) {
-  kernel_launches() += 12;
+  kernel_launches() += 13;
   k_dense_sum<<<a.NBD, TPB, 0, s>>>(a, w);
   k_reduce_proj<<<a.P, TPB, 0, s>>>(a.partials, a.dpre, 1, 0, nullptr, a.base, a.S_total, a.gamma_cur, a.tau_cur,
                                     a.sw_cur);
   for (int pass = 0; pass < 3; ++pass) {
     k_hist<<<a.NBD, TPB, 0, s>>>(a, w, pass);
-    k_select<<<1, 256, 0, s>>>(a, pass);
+    k_select<<<a.groups, 256, 0, s>>>(a, pass);
   }
   k_count<<<a.NBD, TPB, 0, s>>>(a, w);
   k_scan_dense<<<1, 1024, 0, s>>>(a, a.NBD);
   k_compact<<<a.NBD, TPB, 0, s>>>(a, w);
   k_dense_offsets<<<1, 256, 0, s>>>(a, (uint32_t)k0);
+  k_xi0<<<1, 256, 0, s>>>(a);
 }
 
 void mask_finish(const MaskArgs& a, cudaStream_t s) {
@@ -689,12 +719,12 @@ void sparse_restore(const MaskArgs& a, int cur, uint64_t seed, float eps, cudaSt
   k_sparse_restore<<<a.NBS, TPB, 0, s>>>(a, cur, seed, eps);
 }
 
-void sparse_shrink(const MaskArgs& a, int cur, float xi0, uint32_t* d_total, cudaStream_t s) {
+void sparse_shrink(const MaskArgs& a, int cur, uint32_t* d_total, cudaStream_t s) {
   kernel_launches() += 5;
-  k_shrink_mark<<<a.NBS, TPB, 0, s>>>(a, cur, xi0);
+  k_shrink_mark<<<a.NBS, TPB, 0, s>>>(a, cur);
   k_frozen_add<<<a.P, TPB, 0, s>>>(a);
   k_scan_simple<<<1, 1024, 0, s>>>(a, a.NBS, d_total);
-  k_shrink_scatter<<<a.NBS, TPB, 0, s>>>(a, cur, xi0);
+  k_shrink_scatter<<<a.NBS, TPB, 0, s>>>(a, cur);
   k_sparse_offsets<<<1, 256, 0, s>>>(a, cur ^ 1, d_total);
 }
 

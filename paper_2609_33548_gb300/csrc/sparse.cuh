@@ -35,13 +35,19 @@ struct MaskArgs {
   float *gamma_cur, *tau_cur, *sw_cur;       // [P+2] of the current latents
   float *gamma_plus, *tau_plus, *sw_plus;    // [P+2] of w + eps z
   float *gamma_minus, *tau_minus, *sw_minus; // [P+2] of w - eps z
-  unsigned long long* hist;     // [2048]
-  SelectState* sel;
+  int groups;                   // selection groups: 1 (the global quantile of Eq. 4) or P
+                                // (one per projection: the per-tensor variant)
+  unsigned long long* hist;     // [groups x 2048]
+  SelectState* sel;             // [groups]
+  unsigned long long* grp_tie0; // [P] ties before the first dense block of each group
+  float* xi0p;                  // [P] xi_0 of each projection (Eq. 5)
   uint32_t *blk_a, *blk_b, *blk_c, *blk_d;   // per-block scratch
   unsigned long long* counters; // [0] flipped, [1] jumps, [2] dropped, [3] packed words rewritten
   unsigned* err;
 };
 
+// Selects S_0 (the a.groups groups' select states must hold their k) and
+// writes the sparse store, the codes at tau_0 and xi0p.
 void mask_build(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_t s);
 void mask_finish(const MaskArgs& a, cudaStream_t s);
 void sparse_pm_taus(const MaskArgs& a, int cur, uint64_t seed, float eps, cudaStream_t s);
@@ -79,7 +85,7 @@ void sparse_update_dirs(const MaskArgs& a, int cur, const UpdateDirs& d, float e
                         cudaStream_t s);
 void sparse_update(const MaskArgs& a, int cur, uint64_t seed, float eps, float lr, const double* g_dev,
                    double g_host, int use_host, cudaStream_t s);
-void sparse_shrink(const MaskArgs& a, int cur, float xi0, uint32_t* d_total, cudaStream_t s);
+void sparse_shrink(const MaskArgs& a, int cur, uint32_t* d_total, cudaStream_t s);
 void launch_grad(const double* loss, float eps, double* g, cudaStream_t s);
 void launch_normal(uint64_t seed, const uint32_t* idx, uint64_t n, float* z, cudaStream_t s);
 

@@ -20,7 +20,7 @@ OK, WMASKFIXED, EINVAL, ESTATE, ENOMEM, ECUDA, ETIMEOUT = 0, 1, -1, -2, -3, -4, 
 # Every function declared in include/termezo.h.
 EXPORTS = (
     "termezo_workspace_bytes", "termezo_memory", "termezo_create", "termezo_load_params", "termezo_build_mask",
-    "termezo_forward_loss", "termezo_step", "termezo_step_k", "termezo_step_joint", "termezo_shrink", "termezo_requantize", "termezo_update",
+    "termezo_build_mask_rule", "termezo_forward_loss", "termezo_step", "termezo_step_k", "termezo_step_joint", "termezo_shrink", "termezo_requantize", "termezo_update",
     "termezo_bitlinear", "termezo_state_sizes", "termezo_export_state", "termezo_normal",
     "termezo_absmean_noalloc", "termezo_attention", "termezo_profile", "termezo_destroy", "termezo_strerror",
 )
@@ -62,6 +62,9 @@ class ProfileOut(ctypes.Structure):
         return {n: getattr(self, n) for n, _ in self._fields_}
 
 
+MASK_GLOBAL, MASK_PER_TENSOR = 0, 1
+
+
 class TermezoError(RuntimeError):
     def __init__(self, fn, status, msg):
         super().__init__(f"{fn} failed: {msg} (status {status})")
@@ -93,6 +96,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         "termezo_create": (I32, [ctypes.POINTER(ModelCfg), F64, P, ctypes.c_size_t, P, ctypes.POINTER(P)]),
         "termezo_load_params": (I32, [P, P, P, P, P]),
         "termezo_build_mask": (I32, [P, F64, ctypes.POINTER(U64), ctypes.POINTER(F32)]),
+        "termezo_build_mask_rule": (I32, [P, F64, I32, ctypes.POINTER(U64), P]),
         "termezo_forward_loss": (I32, [P, P, P, ctypes.POINTER(F64), P]),
         "termezo_step": (I32, [P, U64, F32, F32, F64, P, P, ctypes.POINTER(StepOut), P, P]),
         "termezo_step_k": (I32, [P, P, I32, F32, F32, F64, P, P, ctypes.POINTER(StepOut), P, P]),
@@ -199,6 +203,17 @@ class Context:
                                                                ctypes.byref(xi0)))
         self._keep[0] = None  # the library no longer reads the dense latents
         return k0.value, np.float32(xi0.value)
+
+    def termezo_build_mask_rule(self, density: float, rule: int):
+        """Mask rule MASK_GLOBAL (Eq. 4) or MASK_PER_TENSOR; returns (k0,
+        xi0: a float32, or an array with one xi_0 per projection)."""
+        k0 = ctypes.c_uint64(0)
+        n = self.termezo_state_sizes()[2] if rule == MASK_PER_TENSOR else 1
+        xi0 = np.zeros(n, dtype=np.float32)
+        _check("termezo_build_mask_rule", load().termezo_build_mask_rule(
+            self.handle, density, rule, ctypes.byref(k0), xi0.ctypes.data_as(ctypes.c_void_p)))
+        self._keep[0] = None
+        return k0.value, (xi0 if rule == MASK_PER_TENSOR else xi0[0])
 
     def termezo_forward_loss(self, tokens, targets):
         loss = ctypes.c_double(0)

@@ -106,6 +106,21 @@ def test_full_size_mask_requant_and_gemm(name):
         np.testing.assert_array_equal(acc.cpu().numpy()[rows], bitnet.int_matmul(q, codes))
 
 
+def test_full_size_per_tensor_mask():
+    """The per-tensor quantile at the full 2B shape (210 projections, 2.08 G
+    latents): k0, every projection's xi_0 and the sorted index list
+    bit-exact against the oracle."""
+    cfg, density = synth.BITNET_2B, 0.01
+    ctx, dev, (w, *_r) = _setup(cfg, density)
+    k0, xi0 = ctx.termezo_build_mask_rule(density, tz.MASK_PER_TENSOR)
+    sel, xi_o, k0_o, tau = otz.initial_mask_per_tensor(w, otz.registry(cfg), density)
+    assert k0 == k0_o
+    np.testing.assert_array_equal(xi0.view(np.uint32), xi_o.view(np.uint32))
+    st = ctx.termezo_export_state(packed=False)
+    np.testing.assert_array_equal(st["idx"], sel.astype(np.uint32))
+    np.testing.assert_array_equal(st["latents"], w[sel])
+
+
 def test_step_sampled_sequences_0_7b():
     cfg, density = synth.BITNET_07B, 0.01
     ctx, dev, (w, emb, gains, head, tok, tgt) = _setup(cfg, density)

@@ -126,3 +126,30 @@ def test_bitlinear_int32_accumulators_bit_exact(shape):
     np.testing.assert_array_equal(acc.cpu().numpy(), acc_o)
     y_o = acc_o.astype(np.float64) * (a.astype(np.float64)[:, None] / 127.0) * float(sw[0])
     np.testing.assert_allclose(y.cpu().numpy(), y_o, rtol=2e-6, atol=1e-30)
+
+
+PER_TENSOR_DENSITIES = (0.003, 0.02, 0.1)
+
+
+@pytest.mark.parametrize("density", PER_TENSOR_DENSITIES)
+def test_per_tensor_mask_bit_exact(density):
+    """The per-tensor quantile on the 14 projections of the tiny decoder:
+    the sorted index list, latents, every projection's xi_0 and every
+    packed code equal the oracle's bit for bit."""
+    cfg = synth.TINY
+    w = synth.latents(cfg)
+    ctx = tz.Context(tz.make_cfg(cfg), density)
+    emb, gains, head = synth.theta(cfg)
+    ctx.termezo_load_params(w.cuda(), emb.cuda(), gains.cuda(), head.cuda())
+    k0, xi0 = ctx.termezo_build_mask_rule(density, tz.MASK_PER_TENSOR)
+    reg = otz.registry(cfg)
+    wn = w.numpy()
+    sel, xi_o, k0_o, tau = otz.initial_mask_per_tensor(wn, reg, density)
+    assert k0 == k0_o
+    np.testing.assert_array_equal(xi0.view(np.uint32), xi_o.view(np.uint32))
+    st = ctx.termezo_export_state()
+    np.testing.assert_array_equal(st["idx"], sel.astype(np.uint32))
+    np.testing.assert_array_equal(st["latents"], wn[sel])
+    np.testing.assert_array_equal(st["tau_cur"].view(np.uint32), tau.view(np.uint32))
+    codes = np.concatenate([ternary.quantize(wn[p.base:p.base + p.n], tau[j]) for j, p in enumerate(reg)])
+    np.testing.assert_array_equal(st["packed"], ternary.pack_codes(codes))

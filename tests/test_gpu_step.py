@@ -301,3 +301,76 @@ def test_joint_theta_step_matches_oracle(inputs):
     assert np.count_nonzero(diff) <= max(3, int(1e-4 * diff.size)), np.count_nonzero(diff)
     assert np.all(diff <= 2 * ulp)
     assert not np.array_equal(got[2], th0[2])
+
+
+def test_per_tensor_mask_replay_many_steps(inputs):
+    """The shrink of Eq. 5 with one xi_0 per projection (per-tensor mask):
+    20 iterations with a given g sequence, index lists bit-exact, latents
+    within the rounding of the restore arithmetic."""
+    w0 = inputs[0].numpy()
+    reg = otz.registry(_cfg(inputs))
+    ctx, dev = _gpu_ctx(inputs)
+    ctx.termezo_build_mask_rule(DENSITY, tz.MASK_PER_TENSOR)
+    state = otz.build(w0, reg, DENSITY, per_tensor=True)
+    eps, lr = np.float32(EPS), np.float32(2e-3)
+    rng = np.random.default_rng(6)
+    sizes = []
+    for t in range(20):
+        g = float(rng.standard_normal() * 20.0)
+        seed = synth.step_seed(100 + t)
+        if t:
+            ctx.termezo_shrink()
+            state.active, _ = otz.shrink(state.w, reg, state.active, state.xi0)
+        act = state.active
+        ctx.termezo_requantize(seed, float(eps), +1)
+        ctx.termezo_requantize(seed, float(eps), -1)
+        ctx.termezo_update(seed, float(eps), float(lr), g)
+        z = philox.normal(seed, act)
+        w_next, *_ = otz.masked_spsa(state.w, act, z, eps, 0.0, lambda v: 0.0)
+        c = np.float32(float(lr) * g)
+        state.w = w_next
+        state.w[act] = (state.w[act] - (c * z).astype(np.float32)).astype(np.float32)
+        st = ctx.termezo_export_state(packed=False)
+        np.testing.assert_array_equal(st["idx"], act.astype(np.uint32))
+        tol = (t + 1) * 1e-5 * (np.abs(state.w[act]) + 2 * np.abs(eps * z))
+        assert np.all(np.abs(st["latents"].astype(np.float64) - state.w[act]) <= tol)
+        sizes.append(act.size)
+    assert sizes[-1] < sizes[0]
+
+
+def test_full_density_step_matches_oracle():
+    """rho_0 = 1: every latent is active (full MeZO on the latents); one step
+    against the oracle as in the masked case."""
+    cfg = synth.TINY
+    w = synth.latents(cfg)
+    emb, gains, head = synth.theta(cfg)
+    tok, tgt = synth.batch(cfg)
+    ctx = tz.Context(tz.make_cfg(cfg), 1.0)
+    dev = [t.cuda() for t in (w, emb, gains, head, tok, tgt)]
+    ctx.termezo_load_params(dev[0], dev[1], dev[2], dev[3])
+    k0, _ = ctx.termezo_build_mask(1.0)
+    assert k0 == cfg.d_lat
+    reg = otz.registry(cfg)
+    state = otz.build(w.numpy(), reg, 1.0)
+    th = (emb.numpy(), gains.numpy(), head.float().numpy(), tok.numpy(), tgt.numpy())
+    fn = otz.bitnet_loss_fn(cfg, *th)
+    seed = synth.step_seed(7)
+    w_before = state.w.copy()
+    out = ctx.termezo_step(seed, EPS, LR, 1.0, dev[4], dev[5])
+    rec = otz.step(state, fn, seed, EPS, LR)
+    z = philox.normal(seed, np.arange(cfg.d_lat))
+    e = (np.float32(EPS) * z).astype(np.float32)
+    wp = (w_before + e).astype(np.float32)
+    wm = (wp - np.float32(2) * e).astype(np.float32)
+    cp, _, swp = otz.requantize(wp, reg)
+    cm, _, swm = otz.requantize(wm, reg)
+    lp = rounding.loss_ensemble(cfg, (_split(cp, reg), swp), th, n=4).mean(axis=1)
+    lm = rounding.loss_ensemble(cfg, (_split(cm, reg), swm), th, n=4).mean(axis=1)
+    assert rounding.within(out["loss_plus"], rec["loss_plus"], lp)
+    assert rounding.within(out["loss_minus"], rec["loss_minus"], lm)
+    assert rounding.g_within_ensemble(out["g"], rec["g"], (lp - lm) / (2 * float(np.float32(EPS))))
+    assert out["k_active"] == cfg.d_lat
+    st = ctx.termezo_export_state(packed=False)
+    np.testing.assert_array_equal(st["idx"], np.arange(cfg.d_lat, dtype=np.uint32))
+    tol = 1e-5 * (np.abs(w_before) + 2 * np.abs(e)) + float(np.float32(LR)) * abs(out["g"] - rec["g"]) * np.abs(z) * 1.01
+    assert np.all(np.abs(st["latents"].astype(np.float64) - state.w) <= tol)
