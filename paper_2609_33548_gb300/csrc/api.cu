@@ -160,10 +160,20 @@ struct termezo_ctx {
   bool prof_on = false;
   std::vector<ProfRec> prof;
   std::vector<cudaEvent_t> ev_pool;
+  // weight expansion overlapped with the previous GEMM: a side stream and two
+  // bf16 weight buffers (q,k,v and gate,up in wexp; o and down in wexp2)
+  uint16_t* wexp2 = nullptr;
+  cudaStream_t xstream = nullptr;
+  cudaEvent_t ev_free[2] = {nullptr, nullptr};   // buffer b no longer read
+  cudaEvent_t ev_ready[2] = {nullptr, nullptr};  // buffer b holds the next group's weights
+  cudaEvent_t ev_codes = nullptr;                // the codes of this forward are final
   size_t ev_used = 0;
   uint64_t launch_base = 0;
   ~termezo_ctx() {
     for (cudaEvent_t e : ev_pool) cudaEventDestroy(e);
+    for (cudaEvent_t e : {ev_free[0], ev_free[1], ev_ready[0], ev_ready[1], ev_codes})
+      if (e) cudaEventDestroy(e);
+    if (xstream) cudaStreamDestroy(xstream);
   }
 };
 
@@ -234,6 +244,7 @@ void carve(termezo_ctx* c, Carver& cv) {
   c->xq = cv.take<uint16_t>(T * xq_cols(s));
   c->deq = cv.take<float>(T);
   c->wexp = cv.take<uint16_t>(wexp_elems(s));
+  c->wexp2 = s.op ? nullptr : cv.take<uint16_t>(wexp_elems(s));
   if (!s.op) {
     const size_t hq = (size_t)s.H * s.hd, hkv = (size_t)s.KV * s.hd;
     c->x = cv.take<float>(T * s.D);
@@ -338,11 +349,45 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
   cudaStream_t st = c->stream;
   const int T = s.T, D = s.D, F = s.F, hq = s.H * s.hd, hkv = s.KV * s.hd;
   tmz::launch_embed(tokens, c->embed, T, D, s.V, c->x, c->ma.err, st);
+  // Projection group g of layer l (0 q,k,v; 1 o; 2 gate,up; 3 down) is
+  // expanded to bf16 on the side stream into buffer g % 2 while the GEMM of
+  // the group before it runs; the GEMM waits for its weights, and the next
+  // expansion into a buffer waits for the GEMM that read it last.
+  uint16_t* wbuf[2] = {c->wexp, c->wexp2};
+  cudaStream_t xs = c->xstream;
+  auto expand = [&](int l, int g) {
+    const int b = g & 1;
+    cudaStreamWaitEvent(xs, c->ev_free[b], 0);
+    const uint32_t* pk = c->ma.packed;
+    if (g == 0)
+      tmz::launch_expand_codes(pk + s.base[proj_of(s, l, 0)] / 16, (uint64_t)(hq + 2 * hkv), D, wbuf[b], xs);
+    else if (g == 1)
+      tmz::launch_expand_codes(pk + s.base[proj_of(s, l, 3)] / 16, (uint64_t)D, hq, wbuf[b], xs);
+    else if (g == 2)
+      tmz::launch_expand_gate_up(pk + s.base[proj_of(s, l, 4)] / 16, pk + s.base[proj_of(s, l, 5)] / 16, F, D,
+                                 wbuf[b], xs);
+    else
+      tmz::launch_expand_codes(pk + s.base[proj_of(s, l, 6)] / 16, (uint64_t)D, F, wbuf[b], xs);
+    cudaEventRecord(c->ev_ready[b], xs);
+  };
+  auto gemm = [&](int l, int g, const GemmPlan& plan, const GemmArgs& a, double flops) -> bool {
+    cudaStreamWaitEvent(st, c->ev_ready[g & 1], 0);
+    {
+      ProfScope ps(c, 0, flops);
+      if (tmz::gemm_launch(plan, a, st) != cudaSuccess) return false;
+    }
+    cudaEventRecord(c->ev_free[g & 1], st);
+    const int nl = g == 3 ? l + 1 : l, ng = (g + 1) & 3;
+    if (nl < s.L) expand(nl, ng);
+    return true;
+  };
+  cudaEventRecord(c->ev_codes, st);
+  cudaStreamWaitEvent(xs, c->ev_codes, 0);
+  expand(0, 0);
   for (int l = 0; l < s.L; ++l) {
     const int pq = proj_of(s, l, 0), po = proj_of(s, l, 3), pg = proj_of(s, l, 4), pd = proj_of(s, l, 6);
     // attention block
     tmz::launch_norm_quant(c->x, c->gains + (size_t)(2 * l) * D, T, D, c->xq, c->deq, st);
-    tmz::launch_expand_codes(c->ma.packed + s.base[pq] / 16, (uint64_t)(hq + 2 * hkv), D, c->wexp, st);
     GemmArgs a{};
     a.out = c->qkv;
     a.ldo = hq + 2 * hkv;
@@ -362,10 +407,7 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
       a.KV = s.KV;
       a.hd = s.hd;
     }
-    {
-      ProfScope ps(c, 0, gemm_flops(c->plan_qkv));
-      if (tmz::gemm_launch(c->plan_qkv, a, st) != cudaSuccess) return TERMEZO_ECUDA;
-    }
+    if (!gemm(l, 0, c->plan_qkv, a, gemm_flops(c->plan_qkv))) return TERMEZO_ECUDA;
     if (!c->plan_qkv.rope)
       tmz::launch_rope_pack(c->qkv, c->cosb, c->sinb, s.B, s.S, s.H, s.KV, s.hd, c->qb, c->kb, c->vt, st);
     a.rope = 0;  // the remaining projections of the layer reuse a
@@ -379,20 +421,14 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
       }
     }
     tmz::launch_norm_quant(c->attn, nullptr, T, hq, c->xq, c->deq, st);
-    tmz::launch_expand_codes(c->ma.packed + s.base[po] / 16, (uint64_t)D, hq, c->wexp, st);
     a.out = c->x;
     a.ldo = D;
     a.mode = 1;
     a.sw = sw + po;
     a.n1 = a.n2 = D;
-    {
-      ProfScope ps(c, 0, gemm_flops(c->plan_o));
-      if (tmz::gemm_launch(c->plan_o, a, st) != cudaSuccess) return TERMEZO_ECUDA;
-    }
+    if (!gemm(l, 1, c->plan_o, a, gemm_flops(c->plan_o))) return TERMEZO_ECUDA;
     // MLP block
     tmz::launch_norm_quant(c->x, c->gains + (size_t)(2 * l + 1) * D, T, D, c->xq, c->deq, st);
-    tmz::launch_expand_gate_up(c->ma.packed + s.base[pg] / 16, c->ma.packed + s.base[pg + 1] / 16, F, D, c->wexp,
-                               st);
     a.out = c->gu;  // hid = relu(gate)^2 * up, fp32 [T, F]
     a.ldo = F;
     a.mode = 0;
@@ -400,22 +436,15 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
     a.n1 = a.n2 = a.N;
     a.relu2 = 1;
     a.n_out = F;
-    {
-      ProfScope ps(c, 0, 2.0 * T * (2.0 * F) * D);
-      if (tmz::gemm_launch(c->plan_gu, a, st) != cudaSuccess) return TERMEZO_ECUDA;
-    }
+    if (!gemm(l, 2, c->plan_gu, a, 2.0 * T * (2.0 * F) * D)) return TERMEZO_ECUDA;
     a.relu2 = 0;
     tmz::launch_norm_quant(c->gu, nullptr, T, F, c->xq, c->deq, st);
-    tmz::launch_expand_codes(c->ma.packed + s.base[pd] / 16, (uint64_t)D, F, c->wexp, st);
     a.out = c->x;
     a.ldo = D;
     a.mode = 1;
     a.sw = sw + pd;
     a.n1 = a.n2 = D;
-    {
-      ProfScope ps(c, 0, gemm_flops(c->plan_down));
-      if (tmz::gemm_launch(c->plan_down, a, st) != cudaSuccess) return TERMEZO_ECUDA;
-    }
+    if (!gemm(l, 3, c->plan_down, a, gemm_flops(c->plan_down))) return TERMEZO_ECUDA;
   }
   if (s.mode == 0) {
     tmz::launch_head_ce_last(c->x, c->gains + (size_t)(2 * s.L) * D, c->head, targets, s.B, s.S, D, s.V, s.C,
@@ -540,9 +569,12 @@ int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspa
     const int T = s.T, D = s.D, F = s.F, hq = s.H * s.hd, hkv = s.KV * s.hd;
     const bool rope_fused = rope_fused_shape(s);
     bool ok = tmz::gemm_make_plan(&c->plan_qkv, c->xq, T, D, c->wexp, hq + 2 * hkv, !rope_fused) &&
-              tmz::gemm_make_plan(&c->plan_o, c->xq, T, hq, c->wexp, D, true) &&
+              tmz::gemm_make_plan(&c->plan_o, c->xq, T, hq, c->wexp2, D, true) &&
               tmz::gemm_make_plan(&c->plan_gu, c->xq, T, D, c->wexp, 256 * ((F + 127) / 128), false) &&
-              tmz::gemm_make_plan(&c->plan_down, c->xq, T, F, c->wexp, D, true);
+              tmz::gemm_make_plan(&c->plan_down, c->xq, T, F, c->wexp2, D, true);
+    ok = ok && cudaStreamCreateWithFlags(&c->xstream, cudaStreamNonBlocking) == cudaSuccess;
+    for (cudaEvent_t* e : {&c->ev_free[0], &c->ev_free[1], &c->ev_ready[0], &c->ev_ready[1], &c->ev_codes})
+      ok = ok && cudaEventCreateWithFlags(e, cudaEventDisableTiming) == cudaSuccess;
     if (!ok) {
       delete c;
       return TERMEZO_ECUDA;
