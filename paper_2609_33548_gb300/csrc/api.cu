@@ -163,6 +163,9 @@ struct termezo_ctx {
   // weight expansion overlapped with the previous GEMM: a side stream and two
   // bf16 weight buffers (q,k,v and gate,up in wexp; o and down in wexp2)
   uint16_t* wexp2 = nullptr;
+  float* split_ws = nullptr;     // GEMM tail-wave split-K partial tiles
+  unsigned* split_cnt = nullptr;
+  int split_cap = 0;
   cudaStream_t xstream = nullptr;
   cudaEvent_t ev_free[2] = {nullptr, nullptr};   // buffer b no longer read
   cudaEvent_t ev_ready[2] = {nullptr, nullptr};  // buffer b holds the next group's weights
@@ -185,6 +188,15 @@ size_t xq_cols(const Shape& s) {
   if ((size_t)s.H * s.hd > m) m = (size_t)s.H * s.hd;
   if ((size_t)s.F > m) m = s.F;
   return m;
+}
+
+// Partial-tile slots of the GEMM's tail-wave split (at most one wave of
+// 128-row tiles, and no more than the context's GEMMs can have).
+int split_slots(const Shape& s) {
+  const size_t mt = ((size_t)s.T + 127) / 128;
+  const size_t nmax = s.op ? (size_t)s.F : (size_t)(s.H + 2 * s.KV) * s.hd + 2 * (size_t)s.F + s.D;
+  const size_t tiles = mt * ((nmax + 127) / 128);
+  return (int)(tiles < 192 ? tiles : 192);
 }
 
 size_t wexp_elems(const Shape& s) {
@@ -245,6 +257,9 @@ void carve(termezo_ctx* c, Carver& cv) {
   c->deq = cv.take<float>(T);
   c->wexp = cv.take<uint16_t>(wexp_elems(s));
   c->wexp2 = s.op ? nullptr : cv.take<uint16_t>(wexp_elems(s));
+  c->split_cap = split_slots(s);
+  c->split_ws = cv.take<float>((size_t)c->split_cap * 128 * 256);
+  c->split_cnt = cv.take<unsigned>((size_t)c->split_cap * 4);
   if (!s.op) {
     const size_t hq = (size_t)s.H * s.hd, hkv = (size_t)s.KV * s.hd;
     c->x = cv.take<float>(T * s.D);
@@ -370,7 +385,10 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
       tmz::launch_expand_codes(pk + s.base[proj_of(s, l, 6)] / 16, (uint64_t)D, F, wbuf[b], xs);
     cudaEventRecord(c->ev_ready[b], xs);
   };
-  auto gemm = [&](int l, int g, const GemmPlan& plan, const GemmArgs& a, double flops) -> bool {
+  auto gemm = [&](int l, int g, const GemmPlan& plan, GemmArgs a, double flops) -> bool {
+    a.split_ws = c->split_ws;
+    a.split_cnt = c->split_cnt;
+    a.split_cap = c->split_cap;
     cudaStreamWaitEvent(st, c->ev_ready[g & 1], 0);
     {
       ProfScope ps(c, 0, flops);
@@ -560,6 +578,7 @@ int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspa
     cudaMemcpy((void*)c->ma.dproj, dproj.data(), dproj.size() * sizeof(uint16_t), cudaMemcpyHostToDevice);
   }
   cudaMemsetAsync(c->ma.err, 0, sizeof(unsigned), st);
+  cudaMemsetAsync(c->split_cnt, 0, (size_t)c->split_cap * 4 * sizeof(unsigned), st);
   cudaMemsetAsync(c->ma.counters, 0, 4 * sizeof(unsigned long long), st);
   for (float* f : {c->ma.gamma_cur, c->ma.tau_cur, c->ma.sw_cur, c->ma.gamma_plus, c->ma.tau_plus, c->ma.sw_plus,
                    c->ma.gamma_minus, c->ma.tau_minus, c->ma.sw_minus})
@@ -923,6 +942,9 @@ int termezo_bitlinear(termezo_ctx* c, int32_t proj, const uint16_t* d_x, int32_t
   a.ldo = N;
   a.mode = 0;
   a.acc_out = d_acc;
+  a.split_ws = c->split_ws;
+  a.split_cnt = c->split_cnt;
+  a.split_cap = c->split_cap;
   a.deq = c->deq;
   a.sw = c->code_sw + proj;
   a.n1 = a.n2 = N;

@@ -57,7 +57,30 @@ struct GemmSmem {
   static constexpr uint32_t ACC_STRIDE = TMEM_COLS / 2;
 };
 
-// Persistent: CTA c processes tiles c, c + gridDim.x, ...  With m fastest the
+// Work units: the tiles of the full waves, then (split_s > 1) every tile of
+// the last, partial wave split into split_s ranges of k-blocks.  The
+// accumulator is an exact integer (< 2^24) in fp32, so partial accumulators
+// add up exactly and a split tile equals the unsplit one bit for bit.
+struct Unit {
+  int tile, kb0, kb1, tail, split;  // tail: index among the split tiles, -1 for a whole tile
+};
+
+__device__ __forceinline__ Unit unit_of(const GemmArgs& p, int u, int KB) {
+  Unit w;
+  if (p.split_s <= 1 || u < p.full_units) {
+    w.tile = u, w.kb0 = 0, w.kb1 = KB, w.tail = -1, w.split = 0;
+  } else {
+    const int v = u - p.full_units;
+    w.tail = v / p.split_s;
+    w.split = v % p.split_s;
+    w.tile = p.full_units + w.tail;
+    w.kb0 = w.split * KB / p.split_s;
+    w.kb1 = (w.split + 1) * KB / p.split_s;
+  }
+  return w;
+}
+
+// Persistent: CTA c processes units c, c + gridDim.x, ...  With m fastest the
 // CTAs running together share B tiles and sweep A through L2; with n fastest
 // (an A too large for L2, a B that fits) they share A tiles, so A streams from
 // HBM once.  The
@@ -83,6 +106,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   const int n_mt = (p.M + BM - 1) / BM, n_nt = (p.N + BN - 1) / BN;
   const int tiles = n_mt * n_nt;
   const int KB = (p.K + BK - 1) / BK;
+  const int units = p.split_s > 1 ? p.full_units + (tiles - p.full_units) * p.split_s : tiles;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -111,10 +135,12 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmA) : "memory");
       asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmB) : "memory");
       uint32_t it = 0;
-      for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+        const Unit w = unit_of(p, u, KB);
+        const int tile = w.tile;
         const int m0 = (p.n_fast ? tile / n_nt : tile % n_mt) * BM;
         const int n0 = (p.n_fast ? tile % n_nt : tile / n_mt) * BN;
-        for (int kb = 0; kb < KB; ++kb, ++it) {
+        for (int kb = w.kb0; kb < w.kb1; ++kb, ++it) {
           const uint32_t s = it % STAGES, use = it / STAGES;
           if (it >= (uint32_t)STAGES && !(ok = mbar_wait(bar_empty + 8 * s, (use & 1u) ^ 1u))) break;
           const uint32_t sa = sbase + s * L::STAGE_BYTES;
@@ -128,12 +154,13 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16(BM, BN);
       uint32_t it = 0, local = 0;
-      for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x, ++local) {
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++local) {
+        const Unit w = unit_of(p, u, KB);
         const uint32_t b = local & 1u, j = local >> 1;
         if (j >= 1 && !(ok = mbar_wait(bar_tempty + 8 * b, (j & 1u) ^ 1u))) break;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         const uint32_t d = tmem + b * L::ACC_STRIDE;
-        for (int kb = 0; kb < KB; ++kb, ++it) {
+        for (int kb = w.kb0; kb < w.kb1; ++kb, ++it) {
           const uint32_t s = it % STAGES;
           if (!(ok = mbar_wait(bar_full + 8 * s, (it / STAGES) & 1u))) break;
           asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
@@ -141,7 +168,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           const uint64_t da = sw128_desc(sa), db = sw128_desc(sa + A_BYTES);
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
-            mma_bf16(d, da + (uint64_t)(2 * k), db + (uint64_t)(2 * k), idesc, (kb | k) ? 1u : 0u);
+            mma_bf16(d, da + (uint64_t)(2 * k), db + (uint64_t)(2 * k), idesc, (kb > w.kb0 || k) ? 1u : 0u);
           mma_commit(bar_empty + 8 * s);
         }
         if (!ok) break;
@@ -161,7 +188,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     float* dqs = stage + 32 * EPI_LD;  // the 32 rows' activation scales
     const float s0 = p.sw[0], s1 = p.sw[1], s2 = p.sw[2];
     uint32_t local = 0;
-    for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++local) {
+    for (int u = blockIdx.x; u < units; u += gridDim.x, ++local) {
+      const Unit w = unit_of(p, u, KB);
+      const int tile = w.tile;
       const int m0 = (p.n_fast ? tile / n_nt : tile % n_mt) * BM;
       const int n0 = (p.n_fast ? tile % n_nt : tile / n_mt) * BN;
       const uint32_t b = local & 1u, j = local >> 1;
@@ -186,6 +215,51 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       ok = mbar_wait(bar_tfull + 8 * b, j & 1u);
       if (!ok) break;
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      const uint32_t tacc = tmem + ((uint32_t)(quarter * 32) << 16) + b * L::ACC_STRIDE;
+      bool from_parts = false;
+      // split partials, lane-contiguous: [unit][quarter][column][lane] floats,
+      // so every warp access is one 128-byte line
+      auto part_at = [&](int split, int col) {
+        return p.split_ws + (((size_t)(w.tail * p.split_s + split) * 4 + quarter) * BN + col) * 32 + lane;
+      };
+      if (w.tail >= 0) {
+        // a split of a tail tile: its partial accumulator goes to the
+        // workspace; the last split to finish these 32 rows keeps its own in
+        // TMEM and adds the others
+        for (int c = 0; c < BN / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld32(tacc + (uint32_t)(c * 32), r);
+          float* dst = part_at(w.split, 32 * c);
+#pragma unroll
+          for (int q = 0; q < 32; ++q) dst[32 * q] = __uint_as_float(r[q]);
+        }
+        __threadfence();
+        unsigned prev = 0;
+        if (lane == 0) prev = atomicAdd(p.split_cnt + w.tail * 4 + quarter, 1u);
+        prev = __shfl_sync(0xffffffffu, prev, 0);
+        if (prev + 1 != (unsigned)p.split_s) {
+          asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+          __syncwarp();
+          if (lane == 0) mbar_arrive(bar_tempty + 8 * b);
+          continue;
+        }
+        __threadfence();
+        if (lane == 0) p.split_cnt[w.tail * 4 + quarter] = 0;  // ready for the next launch
+        from_parts = true;
+      }
+      // 32 accumulator columns col .. col+31 of this thread's row, plus (last
+      // split of a tail tile) the other splits' partials: integers below 2^24,
+      // so the fp32 sum is exact
+      auto load_acc = [&](int col, uint32_t(&r)[32]) {
+        tmem_ld32(tacc + (uint32_t)col, r);
+        if (!from_parts) return;
+        for (int sp = 0; sp < p.split_s; ++sp) {
+          if (sp == w.split) continue;
+          const float* src = part_at(sp, col);
+#pragma unroll
+          for (int q = 0; q < 32; ++q) r[q] = __float_as_uint(__fadd_rn(__uint_as_float(r[q]), __ldcg(src + 32 * q)));
+        }
+      };
       if (p.lse) {
         // lane = row: running max and sum of exp over this tile's columns
         const int row = row0 + lane;
@@ -256,14 +330,14 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           const int col0 = n0 + hb * p.hd;
           if (col0 >= p.N) break;
           const int head = col0 / p.hd;
-          const uint32_t tb = tmem + ((uint32_t)(quarter * 32) << 16) + b * L::ACC_STRIDE + (uint32_t)(hb * p.hd);
+          const int hc = hb * p.hd;  // this head's first accumulator column
           if (head >= p.H + p.KV) {
             // v: bf16 into vt[b, kvh, d, pos]; the warp's 32 positions of
             // one d are 64 contiguous bytes
             uint16_t* vcol = p.vt + ((size_t)(sb * p.KV + head - p.H - p.KV) * p.hd) * p.S + pos;
             for (int c = 0; c < p.hd / 32; ++c) {
               uint32_t r[32];
-              tmem_ld32(tb + (uint32_t)(c * 32), r);
+              load_acc(hc + c * 32, r);
 #pragma unroll
               for (int q = 0; q < 32; ++q) {
                 const __nv_bfloat16 v = __float2bfloat16_rn(__fmul_rn(__fmul_rn(__uint_as_float(r[q]), dq), s2));
@@ -282,8 +356,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           }
           for (int c = 0; c < half / 32; ++c) {
             uint32_t r1[32], r2[32];
-            tmem_ld32(tb + (uint32_t)(c * 32), r1);
-            tmem_ld32(tb + (uint32_t)(half + c * 32), r2);
+            load_acc(hc + c * 32, r1);
+            load_acc(hc + half + c * 32, r2);
             const float4* cr = reinterpret_cast<const float4*>(p.cosb + (size_t)pos * half + c * 32);
             const float4* sr = reinterpret_cast<const float4*>(p.sinb + (size_t)pos * half + c * 32);
             uint32_t w1[16], w2[16];
@@ -343,7 +417,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           const int col0 = n0 + c * 32;
           if (col0 >= p.N) break;
           uint32_t r[32];
-          tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + b * L::ACC_STRIDE + (uint32_t)(c * 32), r);
+          load_acc(c * 32, r);
           if (p.acc_out && lane < nrows) {
 #pragma unroll
             for (int q = 0; q < 32; ++q)
@@ -582,7 +656,26 @@ cudaError_t launch_bn(const GemmPlan& plan, const GemmArgs& args, cudaStream_t s
   const int sms = sm_count();
   const int tiles = ((plan.N + BN - 1) / BN) * ((plan.M + BM - 1) / BM);
   dim3 grid(tiles < sms ? tiles : sms);
-  k_bitlinear_gemm<BN><<<grid, GEMM_THREADS, smem, stream>>>(plan.a, plan.b, plan.o, plan.q, plan.k, args);
+  // the last, partial wave: its tiles split along K so that all CTAs finish
+  // together (store / residual / fused-RoPE epilogues only; measured on GB300
+  // to pay off for K >= 4096)
+  GemmArgs a = args;
+  a.split_s = 1;
+  a.full_units = tiles;
+  const int full = (tiles / (int)grid.x) * (int)grid.x, rem = tiles - full;
+  const int KB = (plan.K + BK - 1) / BK;
+  // (only long reductions: for K of a few thousand a tile's main loop is
+  // short next to the cost of writing and re-reading the partials)
+  if (a.split_ws && a.split_cnt && rem > 0 && full > 0 && KB >= 64 && !a.relu2 && !a.lse && (a.tma_out || a.rope)) {
+    int S = (int)grid.x / rem;
+    if (S > 4) S = 4;
+    if (S > KB) S = KB;
+    if (S >= 2 && rem * S <= a.split_cap) {
+      a.split_s = S;
+      a.full_units = full;
+    }
+  }
+  k_bitlinear_gemm<BN><<<grid, GEMM_THREADS, smem, stream>>>(plan.a, plan.b, plan.o, plan.q, plan.k, a);
   return cudaGetLastError();
 }
 

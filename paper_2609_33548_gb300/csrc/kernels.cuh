@@ -41,6 +41,13 @@ struct GemmArgs {
   // (row mod S) with the cos / sin tables [S, hd/2], rounded to bf16 and
   // stored as [B, H, S, hd] / [B, KV, S, hd]; v rounded to bf16 into vt
   // [B, KV, hd, S].  out is not written.
+  // split K of the last wave (set in gemm_launch from the split workspace):
+  // split_ws fp32 [split_cap x 128 x 256] partial accumulators, split_cnt
+  // [split_cap x 4] counters (zero between launches), split_s 1: no split
+  float* split_ws;
+  unsigned* split_cnt;
+  int split_cap;
+  int split_s, full_units;
   int rope;
   const float* cosb;
   const float* sinb;

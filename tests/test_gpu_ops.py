@@ -106,8 +106,10 @@ def test_perturb_requantize_update(op_latents):
 # (N, K, M): the GEMM picks its output tile width per shape to fill the last
 # wave of the persistent grid; these shapes take widths 256, 128, 128, 160
 # (ragged M) and 192 on a 152-SM GB300.
+# (2560, 6912, 8192): 640 tiles on 152 CTAs; the 32 of the last wave are
+# split along K into four partial accumulators summed by the last finisher.
 @pytest.mark.parametrize("shape", [(N, K, M), (688, 688, 200), (256, 2560, 130), (2560, 1536, 1000),
-                                   (1536, 768, 4096)])
+                                   (1536, 768, 4096), (2560, 6912, 8192)])
 def test_bitlinear_int32_accumulators_bit_exact(shape):
     n, k, m = shape
     w = synth.op_latents(n, k, seed=11).numpy().reshape(-1)
