@@ -53,7 +53,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # profiles/step_2b_launch_list.md.  It describes the kernel source with this
 # SHA-1 only; any other source, or another workload, reports null.
 GEMM_TRAFFIC = {"workload": "2b", "source": "paper_2609_33548_gb300/csrc/gemm.cu",
-                "sha1": "f1f8230b074097b4cba674b0d28eb081f660aa9c", "bytes_per_launch": 251.9e6}
+                "sha1": "785aeb65e495c4e925e1d6511d7cbac6f902fab2", "bytes_per_launch": 243.6e6}
 
 
 def gemm_traffic(workload):
