@@ -243,4 +243,37 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
   return t;
 }
 
+// ---------------------------------------------------------------------------
+// Programmatic dependent launch.  The forward's kernels are launched so that
+// each starts as soon as every CTA of the kernel before it on the stream has
+// exited, without waiting for that grid's completion to be signalled: the
+// launch and the set-up (barrier init, tensor-memory allocation, descriptor
+// prefetch) overlap the predecessor's completion.  Every thread of such a
+// kernel calls grid_dep_wait before its first global-memory access; the wait
+// returns once the predecessor has completed and its writes are visible.  A
+// grid completes only after all its threads passed the wait, so the ordering
+// is transitive along the stream.  No kernel signals its dependents early:
+// measured on GB300, successors resident next to a running persistent GEMM
+// slowed the forward down (27.8 ms against 27.4 ms without the attribute,
+// 27.0 ms with the successors released only as CTAs exit).  Launched without
+// the attribute, the wait is a no-op.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_dependent(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                             Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 }  // namespace tmz

@@ -88,6 +88,7 @@ template <int VPT>
 __global__ void __launch_bounds__(256) k_norm_quant_vec(const float* __restrict__ x, const float* __restrict__ gain,
                                                         int D, uint16_t* __restrict__ q, float* __restrict__ deq) {
   __shared__ float red[32];
+  grid_dep_wait();
   const size_t row = blockIdx.x;
   const float4* xr = reinterpret_cast<const float4*>(x + row * (size_t)D);
   const float4* gr = reinterpret_cast<const float4*>(gain);
@@ -598,14 +599,14 @@ void launch_norm_quant(const float* x, const float* gain, int M, int D, uint16_t
     return;
   }
   switch (vpt) {
-    case 1: k_norm_quant_vec<1><<<M, 256, 0, s>>>(x, gain, D, q, deq); break;
-    case 2: k_norm_quant_vec<2><<<M, 256, 0, s>>>(x, gain, D, q, deq); break;
-    case 3: k_norm_quant_vec<3><<<M, 256, 0, s>>>(x, gain, D, q, deq); break;
-    case 4: k_norm_quant_vec<4><<<M, 256, 0, s>>>(x, gain, D, q, deq); break;
-    case 5: k_norm_quant_vec<5><<<M, 256, 0, s>>>(x, gain, D, q, deq); break;
-    case 6: k_norm_quant_vec<6><<<M, 256, 0, s>>>(x, gain, D, q, deq); break;
-    case 7: k_norm_quant_vec<7><<<M, 256, 0, s>>>(x, gain, D, q, deq); break;
-    default: k_norm_quant_vec<8><<<M, 256, 0, s>>>(x, gain, D, q, deq); break;
+    case 1: launch_dependent(k_norm_quant_vec<1>, dim3(M), dim3(256), 0, s, x, gain, D, q, deq); break;
+    case 2: launch_dependent(k_norm_quant_vec<2>, dim3(M), dim3(256), 0, s, x, gain, D, q, deq); break;
+    case 3: launch_dependent(k_norm_quant_vec<3>, dim3(M), dim3(256), 0, s, x, gain, D, q, deq); break;
+    case 4: launch_dependent(k_norm_quant_vec<4>, dim3(M), dim3(256), 0, s, x, gain, D, q, deq); break;
+    case 5: launch_dependent(k_norm_quant_vec<5>, dim3(M), dim3(256), 0, s, x, gain, D, q, deq); break;
+    case 6: launch_dependent(k_norm_quant_vec<6>, dim3(M), dim3(256), 0, s, x, gain, D, q, deq); break;
+    case 7: launch_dependent(k_norm_quant_vec<7>, dim3(M), dim3(256), 0, s, x, gain, D, q, deq); break;
+    default: launch_dependent(k_norm_quant_vec<8>, dim3(M), dim3(256), 0, s, x, gain, D, q, deq); break;
   }
 }
 

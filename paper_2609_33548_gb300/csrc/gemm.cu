@@ -57,17 +57,28 @@ struct GemmSmem {
   static constexpr uint32_t ACC_STRIDE = TMEM_COLS / 2;
 };
 
-// Work units: the tiles of the full waves, then (split_s > 1) every tile of
-// the last, partial wave split into split_s ranges of k-blocks.  The
-// accumulator is an exact integer (< 2^24) in fp32, so partial accumulators
-// add up exactly and a split tile equals the unsplit one bit for bit.
+// Work units: the tiles of the full waves, then the tiles of the last,
+// partial wave either split into split_s ranges of k-blocks (split_s > 1) or
+// into nsplit ranges of BN / nsplit columns (nsplit > 1).  The accumulator is
+// an exact integer (< 2^24) in fp32, so partial accumulators add up exactly
+// and a split tile equals the unsplit one bit for bit; a column range is a
+// narrower tile computed whole.
 struct Unit {
-  int tile, kb0, kb1, tail, split;  // tail: index among the split tiles, -1 for a whole tile
+  int tile, kb0, kb1, tail, split;  // tail: index among the K-split tiles, -1 for a whole tile
+  int c0, nw;                       // the unit's columns n0 + c0 .. n0 + c0 + nw - 1 of its tile
 };
 
+template <int BN>
 __device__ __forceinline__ Unit unit_of(const GemmArgs& p, int u, int KB) {
   Unit w;
-  if (p.split_s <= 1 || u < p.full_units) {
+  w.c0 = 0, w.nw = BN;
+  if (p.nsplit > 1 && u >= p.full_units) {
+    const int v = u - p.full_units;
+    w.tile = p.full_units + v / p.nsplit;
+    w.nw = BN / p.nsplit;
+    w.c0 = (v % p.nsplit) * w.nw;
+    w.kb0 = 0, w.kb1 = KB, w.tail = -1, w.split = 0;
+  } else if (p.split_s <= 1 || u < p.full_units) {
     w.tile = u, w.kb0 = 0, w.kb1 = KB, w.tail = -1, w.split = 0;
   } else {
     const int v = u - p.full_units;
@@ -89,8 +100,8 @@ __device__ __forceinline__ Unit unit_of(const GemmArgs& p, int u, int KB) {
 template <int BN>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     k_bitlinear_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                     const __grid_constant__ CUtensorMap tmO, const __grid_constant__ CUtensorMap tmQ,
-                     const __grid_constant__ CUtensorMap tmK, GemmArgs p) {
+                     const __grid_constant__ CUtensorMap tmBn, const __grid_constant__ CUtensorMap tmO,
+                     const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK, GemmArgs p) {
   using L = GemmSmem<BN>;
   constexpr int STAGES = L::STAGES;
   extern __shared__ uint8_t smem_raw[];
@@ -106,7 +117,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   const int n_mt = (p.M + BM - 1) / BM, n_nt = (p.N + BN - 1) / BN;
   const int tiles = n_mt * n_nt;
   const int KB = (p.K + BK - 1) / BK;
-  const int units = p.split_s > 1 ? p.full_units + (tiles - p.full_units) * p.split_s : tiles;
+  const int units = p.split_s > 1   ? p.full_units + (tiles - p.full_units) * p.split_s
+                    : p.nsplit > 1 ? p.full_units + (tiles - p.full_units) * p.nsplit
+                                   : tiles;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -119,6 +132,11 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  if (warp == 0 && lane == 0) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmA) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmB) : "memory");
+    if (p.nsplit > 1) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmBn) : "memory");
+  }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
                  "r"(L::TMEM_COLS));
@@ -129,37 +147,41 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = *tmem_slot;
   bool ok = true;
+  // everything above touched only this CTA's own resources; A, the output
+  // and the residual stream belong to the kernels before this one
+  grid_dep_wait();
 
   if (warp == 0) {
     if (lane == 0) {
-      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmA) : "memory");
-      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmB) : "memory");
       uint32_t it = 0;
       for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
-        const Unit w = unit_of(p, u, KB);
+        const Unit w = unit_of<BN>(p, u, KB);
         const int tile = w.tile;
         const int m0 = (p.n_fast ? tile / n_nt : tile % n_mt) * BM;
         const int n0 = (p.n_fast ? tile % n_nt : tile / n_mt) * BN;
+        const bool narrow = w.nw < BN;
         for (int kb = w.kb0; kb < w.kb1; ++kb, ++it) {
           const uint32_t s = it % STAGES, use = it / STAGES;
           if (it >= (uint32_t)STAGES && !(ok = mbar_wait(bar_empty + 8 * s, (use & 1u) ^ 1u))) break;
           const uint32_t sa = sbase + s * L::STAGE_BYTES;
-          mbar_expect_tx(bar_full + 8 * s, L::STAGE_BYTES);
+          mbar_expect_tx(bar_full + 8 * s, narrow ? A_BYTES + w.nw * BK * 2 : L::STAGE_BYTES);
           tma_load_2d(sa, &tmA, kb * BK, m0, bar_full + 8 * s);
-          tma_load_2d(sa + A_BYTES, &tmB, kb * BK, n0, bar_full + 8 * s);
+          tma_load_2d(sa + A_BYTES, narrow ? &tmBn : &tmB, kb * BK, n0 + w.c0, bar_full + 8 * s);
         }
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      const uint32_t idesc = idesc_bf16(BM, BN);
+      const uint32_t idesc_full = idesc_bf16(BM, BN);
+      const uint32_t idesc_narrow = idesc_bf16(BM, BN / (p.nsplit > 1 ? p.nsplit : 1));
       uint32_t it = 0, local = 0;
       for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++local) {
-        const Unit w = unit_of(p, u, KB);
+        const Unit w = unit_of<BN>(p, u, KB);
         const uint32_t b = local & 1u, j = local >> 1;
         if (j >= 1 && !(ok = mbar_wait(bar_tempty + 8 * b, (j & 1u) ^ 1u))) break;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         const uint32_t d = tmem + b * L::ACC_STRIDE;
+        const uint32_t idesc = w.nw < BN ? idesc_narrow : idesc_full;
         for (int kb = w.kb0; kb < w.kb1; ++kb, ++it) {
           const uint32_t s = it % STAGES;
           if (!(ok = mbar_wait(bar_full + 8 * s, (it / STAGES) & 1u))) break;
@@ -189,10 +211,12 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     const float s0 = p.sw[0], s1 = p.sw[1], s2 = p.sw[2];
     uint32_t local = 0;
     for (int u = blockIdx.x; u < units; u += gridDim.x, ++local) {
-      const Unit w = unit_of(p, u, KB);
+      const Unit w = unit_of<BN>(p, u, KB);
       const int tile = w.tile;
       const int m0 = (p.n_fast ? tile / n_nt : tile % n_mt) * BM;
-      const int n0 = (p.n_fast ? tile % n_nt : tile / n_mt) * BN;
+      // a narrow unit's accumulator columns 0 .. nw-1 are output columns n0 ..
+      const int n0 = (p.n_fast ? tile % n_nt : tile / n_mt) * BN + w.c0;
+      const int ncols = w.nw;
       const uint32_t b = local & 1u, j = local >> 1;
       const int row0 = m0 + quarter * 32;
       const int nrows = min(32, p.M - row0);
@@ -326,7 +350,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         const float dq = dq_row;
         const int sb = row0 / p.S, pos0 = row0 - sb * p.S, pos = pos0 + lane;
         const int half = p.hd >> 1;
-        for (int hb = 0; hb < BN / p.hd; ++hb) {
+        for (int hb = 0; hb < ncols / p.hd; ++hb) {
           const int col0 = n0 + hb * p.hd;
           if (col0 >= p.N) break;
           const int head = col0 / p.hd;
@@ -413,7 +437,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         // nearest, per element: the same value as out + y)
         const float dq = dq_row;
         const int row = row0 + lane;
-        for (int c = 0; c < BN / 32; ++c) {
+        for (int c = 0; c < ncols / 32; ++c) {
           const int col0 = n0 + c * 32;
           if (col0 >= p.N) break;
           uint32_t r[32];
@@ -459,7 +483,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           ++n_out_tiles;
         }
       }
-      for (int c = 0; c < ((p.relu2 || p.lse || p.tma_out || p.rope) ? 0 : BN / 32); ++c) {
+      for (int c = 0; c < ((p.relu2 || p.lse || p.tma_out || p.rope) ? 0 : ncols / 32); ++c) {
         {
           uint32_t r[32];
           tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + b * L::ACC_STRIDE + (uint32_t)(c * 32), r);
@@ -481,7 +505,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
             if (p.mode) {
               float nxt[32];
               const int ncol = col + 32;
-              const bool more = c + 1 < BN / 32 && ncol < p.N;
+              const bool more = c + 1 < ncols / 32 && ncol < p.N;
 #pragma unroll
               for (int rr = 0; rr < 32; ++rr) nxt[rr] = (more && rr < nrows) ? o[(size_t)rr * p.ldo + 32] : 0.f;
 #pragma unroll
@@ -595,8 +619,19 @@ bool gemm_make_plan(GemmPlan* plan, const uint16_t* a, int M, int K, const uint1
   // n fastest when A (M x K bf16) is too large to stay in L2 and B is not
   const double a_bytes = 2.0 * M * K, b_bytes = 2.0 * N * K;
   plan->n_fast = (a_bytes > 64e6 && b_bytes < a_bytes) ? 1 : 0;
-  return encode_bf16_kmajor(&plan->a, a, (uint64_t)M, (uint64_t)K, BM) &&
-         encode_bf16_kmajor(&plan->b, b, (uint64_t)N, (uint64_t)K, (uint32_t)plan->bn);
+  if (!encode_bf16_kmajor(&plan->a, a, (uint64_t)M, (uint64_t)K, BM) ||
+      !encode_bf16_kmajor(&plan->b, b, (uint64_t)N, (uint64_t)K, (uint32_t)plan->bn))
+    return false;
+  // narrow units of the last wave: whole 32-column epilogue chunks, at least
+  // 64 columns (an MMA of N 64 still reads all of A per k-step)
+  plan->narrow_ok = 0;
+  for (int f = 2; f <= 4; f *= 2) {
+    const int w = plan->bn / f;
+    if (w % 32 == 0 && w >= 64 &&
+        encode_bf16_kmajor(f == 2 ? &plan->b2 : &plan->b4, b, (uint64_t)N, (uint64_t)K, (uint32_t)w))
+      plan->narrow_ok |= f;
+  }
+  return true;
 }
 
 int gemm_col_tiles(int N) { return (N + GEMM_BN - 1) / GEMM_BN; }
@@ -675,8 +710,22 @@ cudaError_t launch_bn(const GemmPlan& plan, const GemmArgs& args, cudaStream_t s
       a.full_units = full;
     }
   }
-  k_bitlinear_gemm<BN><<<grid, GEMM_THREADS, smem, stream>>>(plan.a, plan.b, plan.o, plan.q, plan.k, a);
-  return cudaGetLastError();
+  // otherwise split the last wave's tiles along N, as finely as the idle CTAs
+  // allow (fused RoPE: whole heads per unit; not for the gate/up and
+  // LM-head epilogues, whose tiles pair or reduce columns)
+  a.nsplit = 1;
+  const CUtensorMap* bn_map = &plan.b;
+  if (a.split_s == 1 && rem > 0 && full > 0 && !a.relu2 && !a.lse) {
+    for (int f = 4; f >= 2; f /= 2) {
+      if (!(plan.narrow_ok & f) || rem * f > (int)grid.x || (a.rope && (BN / f) % a.hd)) continue;
+      a.nsplit = f;
+      a.full_units = full;
+      bn_map = f == 2 ? &plan.b2 : &plan.b4;
+      break;
+    }
+  }
+  return launch_dependent(k_bitlinear_gemm<BN>, grid, dim3(GEMM_THREADS), smem, stream, plan.a, plan.b, *bn_map,
+                          plan.o, plan.q, plan.k, a);
 }
 
 }  // namespace
@@ -689,6 +738,7 @@ cudaError_t gemm_launch(const GemmPlan& plan, GemmArgs args, cudaStream_t stream
   if (args.rope && (!plan.rope || plan.bn % args.hd)) return cudaErrorInvalidValue;
   args.tma_out = (plan.o_ptr && args.out == plan.o_ptr && args.ldo == plan.o_ld && !args.relu2 && !args.lse) ? 1 : 0;
   if ((args.relu2 || args.lse) && plan.bn != GEMM_BN) return cudaErrorInvalidValue;
+  if (!args.sw) return cudaErrorInvalidValue;  // every epilogue reads sw[0..2]
   ++kernel_launches();
   switch (plan.bn) {
     case 256: return launch_bn<256>(plan, args, stream);

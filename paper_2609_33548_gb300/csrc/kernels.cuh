@@ -48,6 +48,9 @@ struct GemmArgs {
   unsigned* split_cnt;
   int split_cap;
   int split_s, full_units;
+  // split N of the last wave (set at launch; exclusive with split_s > 1):
+  // its tiles become nsplit units of BN / nsplit columns each (1: no split)
+  int nsplit;
   int rope;
   const float* cosb;
   const float* sinb;
@@ -60,6 +63,8 @@ int gemm_col_tiles(int N);
 
 struct GemmPlan {
   CUtensorMap a, b;
+  CUtensorMap b2, b4;  // B with boxes of bn / 2 and bn / 4 rows (the narrow last-wave units)
+  int narrow_ok;       // bit 1: b2 valid, bit 2: b4 valid
   int M, N, K, bn;  // bn: output tile width (columns of B per tile)
   int n_fast;       // tile order: n fastest (A streamed once, B kept in L2)
   CUtensorMap o;    // fp32 output [M, N] (row stride o_ld): TMA store / reduce-add

@@ -25,6 +25,10 @@ MATRIX = {
                                      batch=2),
     "gqa-long-sft": dataclasses.replace(T, name="gqa-long-sft", hidden=256, heads=4, kv_heads=1, seq=512, batch=1,
                                         vocab=3000, loss_mode=1, n_labels=0),
+    # fused-RoPE QKV GEMM of 160 tiles: the 8 of the last wave run as 16
+    # units of one 128-column head each
+    "narrow-tail": dataclasses.replace(T, name="narrow-tail", hidden=512, heads=4, kv_heads=2, ffn=1376, seq=128,
+                                       batch=40),
 }
 
 

@@ -108,8 +108,11 @@ def test_perturb_requantize_update(op_latents):
 # (ragged M) and 192 on a 152-SM GB300.
 # (2560, 6912, 8192): 640 tiles on 152 CTAs; the 32 of the last wave are
 # split along K into four partial accumulators summed by the last finisher.
+# (2560, 2560, 8192): the same 640 tiles with a short K; the last wave's 32
+# tiles become 128 units of 64 columns.  (1536, 768, 4096): 192 tiles, the
+# last 40 split into 80 units of 128 columns.
 @pytest.mark.parametrize("shape", [(N, K, M), (688, 688, 200), (256, 2560, 130), (2560, 1536, 1000),
-                                   (1536, 768, 4096), (2560, 6912, 8192)])
+                                   (1536, 768, 4096), (2560, 6912, 8192), (2560, 2560, 8192)])
 def test_bitlinear_int32_accumulators_bit_exact(shape):
     n, k, m = shape
     w = synth.op_latents(n, k, seed=11).numpy().reshape(-1)
