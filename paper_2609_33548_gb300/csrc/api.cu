@@ -126,13 +126,13 @@ struct termezo_ctx {
   const uint16_t* head = nullptr;
   // forward buffers
   float* x = nullptr;
-  uint16_t* xq = nullptr;
+  uint8_t* xq = nullptr;  // e4m3 (hi, lo) activation codes [2, T, K]
   float* deq = nullptr;
   float* qkv = nullptr;
   uint16_t *qb = nullptr, *kb = nullptr, *vt = nullptr;
   float* attn = nullptr;
   float* gu = nullptr;
-  uint16_t* wexp = nullptr;
+  uint8_t* wexp = nullptr;
   float *cosb = nullptr, *sinb = nullptr;
   double* per_seq = nullptr;  // [2B]
   double* loss = nullptr;     // [2]
@@ -161,8 +161,8 @@ struct termezo_ctx {
   std::vector<ProfRec> prof;
   std::vector<cudaEvent_t> ev_pool;
   // weight expansion overlapped with the previous GEMM: a side stream and two
-  // bf16 weight buffers (q,k,v and gate,up in wexp; o and down in wexp2)
-  uint16_t* wexp2 = nullptr;
+  // e4m3 weight buffers (q,k,v and gate,up in wexp; o and down in wexp2)
+  uint8_t* wexp2 = nullptr;
   float* split_ws = nullptr;     // GEMM tail-wave split-K partial tiles
   unsigned* split_cnt = nullptr;
   int split_cap = 0;
@@ -253,10 +253,10 @@ void carve(termezo_ctx* c, Carver& cv) {
   c->d_total = cv.take<uint32_t>(1);
   const size_t T = s.T;
   cv.sec = SEC_FORWARD;
-  c->xq = cv.take<uint16_t>(T * xq_cols(s));
+  c->xq = cv.take<uint8_t>(2 * T * xq_cols(s));
   c->deq = cv.take<float>(T);
-  c->wexp = cv.take<uint16_t>(wexp_elems(s));
-  c->wexp2 = s.op ? nullptr : cv.take<uint16_t>(wexp_elems(s));
+  c->wexp = cv.take<uint8_t>(wexp_elems(s));
+  c->wexp2 = s.op ? nullptr : cv.take<uint8_t>(wexp_elems(s));
   c->split_cap = split_slots(s);
   c->split_ws = cv.take<float>((size_t)c->split_cap * 128 * 256);
   c->split_cnt = cv.take<unsigned>((size_t)c->split_cap * 4);
@@ -368,7 +368,7 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
   // expanded to bf16 on the side stream into buffer g % 2 while the GEMM of
   // the group before it runs; the GEMM waits for its weights, and the next
   // expansion into a buffer waits for the GEMM that read it last.
-  uint16_t* wbuf[2] = {c->wexp, c->wexp2};
+  uint8_t* wbuf[2] = {c->wexp, c->wexp2};
   cudaStream_t xs = c->xstream;
   auto expand = [&](int l, int g) {
     const int b = g & 1;
@@ -587,10 +587,10 @@ int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspa
     tmz::launch_rope_tables(s.S, s.hd, c->cosb, c->sinb, st);
     const int T = s.T, D = s.D, F = s.F, hq = s.H * s.hd, hkv = s.KV * s.hd;
     const bool rope_fused = rope_fused_shape(s);
-    bool ok = tmz::gemm_make_plan(&c->plan_qkv, c->xq, T, D, c->wexp, hq + 2 * hkv, !rope_fused) &&
-              tmz::gemm_make_plan(&c->plan_o, c->xq, T, hq, c->wexp2, D, true) &&
-              tmz::gemm_make_plan(&c->plan_gu, c->xq, T, D, c->wexp, 256 * ((F + 127) / 128), false) &&
-              tmz::gemm_make_plan(&c->plan_down, c->xq, T, F, c->wexp2, D, true);
+    bool ok = tmz::gemm_make_plan_f8(&c->plan_qkv, c->xq, T, D, c->wexp, hq + 2 * hkv, !rope_fused) &&
+              tmz::gemm_make_plan_f8(&c->plan_o, c->xq, T, hq, c->wexp2, D, true) &&
+              tmz::gemm_make_plan_f8(&c->plan_gu, c->xq, T, D, c->wexp, 256 * ((F + 127) / 128), false) &&
+              tmz::gemm_make_plan_f8(&c->plan_down, c->xq, T, F, c->wexp2, D, true);
     ok = ok && cudaStreamCreateWithFlags(&c->xstream, cudaStreamNonBlocking) == cudaSuccess;
     for (cudaEvent_t* e : {&c->ev_free[0], &c->ev_free[1], &c->ev_ready[0], &c->ev_ready[1], &c->ev_codes})
       ok = ok && cudaEventCreateWithFlags(e, cudaEventDisableTiming) == cudaSuccess;
@@ -935,7 +935,7 @@ int termezo_bitlinear(termezo_ctx* c, int32_t proj, const uint16_t* d_x, int32_t
   tmz::launch_norm_quant_bf16(d_x, M, K, c->xq, c->deq, st);
   tmz::launch_expand_codes(c->ma.packed + c->sh.base[proj] / 16, (uint64_t)N, K, c->wexp, st);
   GemmPlan plan;
-  if (!tmz::gemm_make_plan(&plan, c->xq, M, K, c->wexp, N, true)) return TERMEZO_ECUDA;
+  if (!tmz::gemm_make_plan_f8(&plan, c->xq, M, K, c->wexp, N, true)) return TERMEZO_ECUDA;
   if (d_y) tmz::gemm_plan_output(&plan, d_y, N);
   GemmArgs a{};
   a.out = d_y;

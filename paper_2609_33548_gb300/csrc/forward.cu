@@ -37,21 +37,31 @@ __device__ __forceinline__ float block_max(float v, float* red) {
   return t;
 }
 
-__device__ __forceinline__ uint16_t int_to_bf16_bits(float v) {
-  return (uint16_t)(__float_as_uint(v) >> 16);  // exact for |v| <= 256 integers
-}
-
 __device__ __forceinline__ float quant_code(float h, float s) {
   float v = rintf(__fmul_rn(h, s));
   return fminf(fmaxf(v, -128.f), 127.f);
 }
 
+// The BitLinear GEMM takes an int8 code q as two e4m3 values, hi = 16
+// floor(q / 16) in [-128, 112] and lo = q - hi in [0, 15]: both have at most
+// four significant bits, so both are exact in e4m3 (1 sign, 4 exponent bits
+// with bias 7, 3 mantissa bits), and hi w + lo w = q w exactly.  hi and lo
+// are formed exactly in fp32 and converted by the hardware, two per
+// instruction (x0 in the low byte).
+__device__ __forceinline__ uint32_t e4m3x2(float x0, float x1) {
+  uint16_t d;
+  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(d) : "f"(x1), "f"(x0));
+  return d;
+}
+__device__ __forceinline__ float code_hi(float q) { return __fmul_rn(floorf(__fmul_rn(q, 0.0625f)), 16.f); }
+
 // One block per row.  h_k = (x_k * r) * g_k with r = 1/sqrt(mean(x^2)+1e-5)
-// (RMSNorm) or h_k = x_k; a = max(max|h|, 1e-5); q_k = rint(h_k * (127/a)).
+// (RMSNorm) or h_k = x_k; a = max(max|h|, 1e-5); q_k = rint(h_k * (127/a)),
+// stored as its e4m3 (hi, lo) pair in q [2, M, D] (hi rows, then lo rows).
 // Generic version (any D, any input type): three passes over the row.
 template <typename In>
 __global__ void k_norm_quant(const In* __restrict__ x, const float* __restrict__ gain, int D,
-                             uint16_t* __restrict__ q, float* __restrict__ deq) {
+                             uint8_t* __restrict__ q, float* __restrict__ deq) {
   __shared__ float red[32];
   const size_t row = blockIdx.x;
   const In* xr = x + row * (size_t)D;
@@ -73,11 +83,14 @@ __global__ void k_norm_quant(const In* __restrict__ x, const float* __restrict__
   }
   const float a = fmaxf(block_max(amax, red), 1e-5f);
   const float s = __fdiv_rn(127.f, a);
-  uint16_t* qr = q + row * (size_t)D;
+  uint8_t* qh = q + row * (size_t)D;
+  uint8_t* ql = qh + (size_t)gridDim.x * D;
   for (int k = threadIdx.x; k < D; k += blockDim.x) {
     const float v = (float)xr[k];
     const float h = gain ? __fmul_rn(__fmul_rn(v, r), gain[k]) : v;
-    qr[k] = int_to_bf16_bits(quant_code(h, s));
+    const float c = quant_code(h, s), hi = code_hi(c);
+    qh[k] = (uint8_t)(e4m3x2(hi, 0.f) & 0xFFu);
+    ql[k] = (uint8_t)(e4m3x2(__fsub_rn(c, hi), 0.f) & 0xFFu);
   }
   if (threadIdx.x == 0) deq[row] = __fdiv_rn(a, 127.f);
 }
@@ -86,7 +99,7 @@ __global__ void k_norm_quant(const In* __restrict__ x, const float* __restrict__
 // row is read once (float4) and kept in registers.
 template <int VPT>
 __global__ void __launch_bounds__(256) k_norm_quant_vec(const float* __restrict__ x, const float* __restrict__ gain,
-                                                        int D, uint16_t* __restrict__ q, float* __restrict__ deq) {
+                                                        int D, uint8_t* __restrict__ q, float* __restrict__ deq) {
   __shared__ float red[32];
   grid_dep_wait();
   const size_t row = blockIdx.x;
@@ -129,14 +142,17 @@ __global__ void __launch_bounds__(256) k_norm_quant_vec(const float* __restrict_
     amax = fmaxf(fmaxf(fmaxf(amax, fabsf(v[i].x)), fmaxf(fabsf(v[i].y), fabsf(v[i].z))), fabsf(v[i].w));
   const float a = fmaxf(block_max(amax, red), 1e-5f);
   const float s = __fdiv_rn(127.f, a);
-  uint2* qr = reinterpret_cast<uint2*>(q + row * (size_t)D);
+  uint32_t* qh = reinterpret_cast<uint32_t*>(q + row * (size_t)D);
+  uint32_t* ql = reinterpret_cast<uint32_t*>(q + ((size_t)gridDim.x + row) * D);
 #pragma unroll
   for (int i = 0; i < VPT; ++i) {
     const int k = i * 256 + threadIdx.x;
     if (k < D4) {
-      const uint32_t b0 = int_to_bf16_bits(quant_code(v[i].x, s)), b1 = int_to_bf16_bits(quant_code(v[i].y, s));
-      const uint32_t b2 = int_to_bf16_bits(quant_code(v[i].z, s)), b3 = int_to_bf16_bits(quant_code(v[i].w, s));
-      qr[k] = make_uint2(b0 | (b1 << 16), b2 | (b3 << 16));
+      const float c0 = quant_code(v[i].x, s), c1 = quant_code(v[i].y, s);
+      const float c2 = quant_code(v[i].z, s), c3 = quant_code(v[i].w, s);
+      const float h0 = code_hi(c0), h1 = code_hi(c1), h2 = code_hi(c2), h3 = code_hi(c3);
+      qh[k] = e4m3x2(h0, h1) | (e4m3x2(h2, h3) << 16);
+      ql[k] = e4m3x2(__fsub_rn(c0, h0), __fsub_rn(c1, h1)) | (e4m3x2(__fsub_rn(c2, h2), __fsub_rn(c3, h3)) << 16);
     }
   }
   if (threadIdx.x == 0) deq[row] = __fdiv_rn(a, 127.f);
@@ -147,41 +163,33 @@ struct Bf16In {
   __device__ __forceinline__ explicit operator float() const { return __uint_as_float((uint32_t)bits << 16); }
 };
 
-// One thread per packed word: 16 codes -> 16 bf16 values (32 bytes).
-__global__ void k_expand_codes(const uint32_t* __restrict__ words, uint64_t n_words, uint16_t* __restrict__ out) {
-  const uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= n_words) return;
-  const uint32_t w = words[i];
-  uint32_t v[8];
+// 16 packed codes (2 bits each: 0 -> -1, 1 -> 0, 2 -> +1) -> 16 e4m3 bytes
+// (+1 = 0x38, -1 = 0xB8, 0 = 0x00), one 16-byte store.
+__device__ __forceinline__ void expand_word(uint32_t w, uint8_t* dst) {
+  uint32_t v[4];
 #pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    const uint32_t c0 = (w >> (4 * j)) & 3u, c1 = (w >> (4 * j + 2)) & 3u;
-    const uint32_t b0 = c0 == 2u ? 0x3F80u : (c0 == 0u ? 0xBF80u : 0u);
-    const uint32_t b1 = c1 == 2u ? 0x3F80u : (c1 == 0u ? 0xBF80u : 0u);
-    v[j] = b0 | (b1 << 16);
+  for (int j = 0; j < 4; ++j) {
+    uint32_t b = 0;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const uint32_t c = (w >> (8 * j + 2 * e)) & 3u;
+      b |= (c == 2u ? 0x38u : (c == 0u ? 0xB8u : 0u)) << (8 * e);
+    }
+    v[j] = b;
   }
-  uint4* o = reinterpret_cast<uint4*>(out + i * 16);
-  o[0] = make_uint4(v[0], v[1], v[2], v[3]);
-  o[1] = make_uint4(v[4], v[5], v[6], v[7]);
+  *reinterpret_cast<uint4*>(dst) = make_uint4(v[0], v[1], v[2], v[3]);
 }
 
-__device__ __forceinline__ void expand_word(uint32_t w, uint16_t* dst) {
-  uint32_t v[8];
-#pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    const uint32_t c0 = (w >> (4 * j)) & 3u, c1 = (w >> (4 * j + 2)) & 3u;
-    const uint32_t b0 = c0 == 2u ? 0x3F80u : (c0 == 0u ? 0xBF80u : 0u);
-    const uint32_t b1 = c1 == 2u ? 0x3F80u : (c1 == 0u ? 0xBF80u : 0u);
-    v[j] = b0 | (b1 << 16);
-  }
-  uint4* o = reinterpret_cast<uint4*>(dst);
-  o[0] = make_uint4(v[0], v[1], v[2], v[3]);
-  o[1] = make_uint4(v[4], v[5], v[6], v[7]);
+// One thread per packed word.
+__global__ void k_expand_codes(const uint32_t* __restrict__ words, uint64_t n_words, uint8_t* __restrict__ out) {
+  const uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n_words) return;
+  expand_word(words[i], out + i * 16);
 }
 
 // One thread per (interleaved row, word).
 __global__ void k_expand_gate_up(const uint32_t* __restrict__ gw, const uint32_t* __restrict__ uw, int F, int wpr,
-                                 uint64_t n_words, uint16_t* __restrict__ out) {
+                                 uint64_t n_words, uint8_t* __restrict__ out) {
   const uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n_words) return;
   const uint64_t r = i / wpr;
@@ -589,10 +597,10 @@ uint64_t& kernel_launches() {
   return n;
 }
 
-void launch_norm_quant(const float* x, const float* gain, int M, int D, uint16_t* q, float* deq, cudaStream_t s) {
+void launch_norm_quant(const float* x, const float* gain, int M, int D, uint8_t* q, float* deq, cudaStream_t s) {
   kernel_launches() += 1;
   const int vpt = (D + 1023) / 1024;
-  const bool aligned = (D % 4 == 0) && ((uintptr_t)x % 16 == 0) && ((uintptr_t)q % 8 == 0) &&
+  const bool aligned = (D % 4 == 0) && ((uintptr_t)x % 16 == 0) && ((uintptr_t)q % 4 == 0) &&
                        (!gain || (uintptr_t)gain % 16 == 0);
   if (!aligned || vpt > 8) {
     k_norm_quant<float><<<M, 256, 0, s>>>(x, gain, D, q, deq);
@@ -610,18 +618,18 @@ void launch_norm_quant(const float* x, const float* gain, int M, int D, uint16_t
   }
 }
 
-void launch_norm_quant_bf16(const uint16_t* x, int M, int D, uint16_t* q, float* deq, cudaStream_t s) {
+void launch_norm_quant_bf16(const uint16_t* x, int M, int D, uint8_t* q, float* deq, cudaStream_t s) {
   kernel_launches() += 1;
   k_norm_quant<Bf16In><<<M, 256, 0, s>>>(reinterpret_cast<const Bf16In*>(x), nullptr, D, q, deq);
 }
 
-void launch_expand_codes(const uint32_t* words, uint64_t rows, int K, uint16_t* out, cudaStream_t s) {
+void launch_expand_codes(const uint32_t* words, uint64_t rows, int K, uint8_t* out, cudaStream_t s) {
   kernel_launches() += 1;
   const uint64_t n = rows * (uint64_t)(K / 16);
   k_expand_codes<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(words, n, out);
 }
 
-void launch_expand_gate_up(const uint32_t* gate_words, const uint32_t* up_words, int F, int K, uint16_t* out,
+void launch_expand_gate_up(const uint32_t* gate_words, const uint32_t* up_words, int F, int K, uint8_t* out,
                            cudaStream_t s) {
   kernel_launches() += 1;
   const int wpr = K / 16;

@@ -30,16 +30,20 @@ namespace tmz {
 namespace {
 
 constexpr int BM = 128;
-constexpr int BK = 64;
+constexpr int BK = 64;  // bf16 elements per k-block (128 bytes)
 constexpr int GEMM_THREADS = 192;
-constexpr int A_BYTES = BM * BK * 2;
 
 constexpr int EPI_WARPS = 4;
 constexpr int EPI_LD = 33;  // staging row stride (floats): conflict-free transpose
 
-template <int BN>
+// A ring stage holds one k-block of 128 bytes per row: 64 bf16 elements, or
+// 128 e4m3 elements with A as two tiles (the hi and lo halves of the codes).
+template <int BN, bool F8>
 struct GemmSmem {
-  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int KE = F8 ? 128 : BK;            // K elements per k-block
+  static constexpr int A_TILE = BM * 128;
+  static constexpr int A_BYTES = F8 ? 2 * A_TILE : A_TILE;
+  static constexpr int B_BYTES = BN * 128;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   // as many ring stages as fit next to the epilogue staging (at most 6)
   // epilogue staging: per warp two 32 x 32 fp32 tiles (128-byte swizzle) for
@@ -97,12 +101,13 @@ __device__ __forceinline__ Unit unit_of(const GemmArgs& p, int u, int KB) {
 // HBM once.  The
 // accumulator is double-buffered in tensor memory (2 x BN columns) so that
 // the epilogue of one tile overlaps the main loop of the next.
-template <int BN>
+template <int BN, bool F8>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
-    k_bitlinear_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                     const __grid_constant__ CUtensorMap tmBn, const __grid_constant__ CUtensorMap tmO,
-                     const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK, GemmArgs p) {
-  using L = GemmSmem<BN>;
+    k_bitlinear_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmA2,
+                     const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmBn,
+                     const __grid_constant__ CUtensorMap tmO, const __grid_constant__ CUtensorMap tmQ,
+                     const __grid_constant__ CUtensorMap tmK, GemmArgs p) {
+  using L = GemmSmem<BN, F8>;
   constexpr int STAGES = L::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -116,7 +121,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n_mt = (p.M + BM - 1) / BM, n_nt = (p.N + BN - 1) / BN;
   const int tiles = n_mt * n_nt;
-  const int KB = (p.K + BK - 1) / BK;
+  const int KB = (p.K + L::KE - 1) / L::KE;
   const int units = p.split_s > 1   ? p.full_units + (tiles - p.full_units) * p.split_s
                     : p.nsplit > 1 ? p.full_units + (tiles - p.full_units) * p.nsplit
                                    : tiles;
@@ -134,6 +139,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   }
   if (warp == 0 && lane == 0) {
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmA) : "memory");
+    if (F8) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmA2) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmB) : "memory");
     if (p.nsplit > 1) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmBn) : "memory");
   }
@@ -164,16 +170,18 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           const uint32_t s = it % STAGES, use = it / STAGES;
           if (it >= (uint32_t)STAGES && !(ok = mbar_wait(bar_empty + 8 * s, (use & 1u) ^ 1u))) break;
           const uint32_t sa = sbase + s * L::STAGE_BYTES;
-          mbar_expect_tx(bar_full + 8 * s, narrow ? A_BYTES + w.nw * BK * 2 : L::STAGE_BYTES);
-          tma_load_2d(sa, &tmA, kb * BK, m0, bar_full + 8 * s);
-          tma_load_2d(sa + A_BYTES, narrow ? &tmBn : &tmB, kb * BK, n0 + w.c0, bar_full + 8 * s);
+          mbar_expect_tx(bar_full + 8 * s, narrow ? L::A_BYTES + w.nw * 128 : L::STAGE_BYTES);
+          tma_load_2d(sa, &tmA, kb * L::KE, m0, bar_full + 8 * s);
+          if (F8) tma_load_2d(sa + L::A_TILE, &tmA2, kb * L::KE, m0, bar_full + 8 * s);
+          tma_load_2d(sa + L::A_BYTES, narrow ? &tmBn : &tmB, kb * L::KE, n0 + w.c0, bar_full + 8 * s);
         }
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      const uint32_t idesc_full = idesc_bf16(BM, BN);
-      const uint32_t idesc_narrow = idesc_bf16(BM, BN / (p.nsplit > 1 ? p.nsplit : 1));
+      const int n_narrow = BN / (p.nsplit > 1 ? p.nsplit : 1);
+      const uint32_t idesc_full = F8 ? idesc_e4m3(BM, BN) : idesc_bf16(BM, BN);
+      const uint32_t idesc_narrow = F8 ? idesc_e4m3(BM, n_narrow) : idesc_bf16(BM, n_narrow);
       uint32_t it = 0, local = 0;
       for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++local) {
         const Unit w = unit_of<BN>(p, u, KB);
@@ -187,10 +195,21 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           if (!(ok = mbar_wait(bar_full + 8 * s, (it / STAGES) & 1u))) break;
           asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
           const uint32_t sa = sbase + s * L::STAGE_BYTES;
-          const uint64_t da = sw128_desc(sa), db = sw128_desc(sa + A_BYTES);
+          const uint64_t da = sw128_desc(sa), db = sw128_desc(sa + L::A_BYTES);
+          // each MMA step reads 32 bytes of every row: 16 bf16 or 32 e4m3
+          // elements; the e4m3 path adds hi B and lo B into one accumulator
+          if (F8) {
+            const uint64_t dl = sw128_desc(sa + L::A_TILE);
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k)
-            mma_bf16(d, da + (uint64_t)(2 * k), db + (uint64_t)(2 * k), idesc, (kb > w.kb0 || k) ? 1u : 0u);
+            for (int k = 0; k < 4; ++k) {
+              mma_e4m3(d, da + (uint64_t)(2 * k), db + (uint64_t)(2 * k), idesc, (kb > w.kb0 || k) ? 1u : 0u);
+              mma_e4m3(d, dl + (uint64_t)(2 * k), db + (uint64_t)(2 * k), idesc, 1u);
+            }
+          } else {
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+              mma_bf16(d, da + (uint64_t)(2 * k), db + (uint64_t)(2 * k), idesc, (kb > w.kb0 || k) ? 1u : 0u);
+          }
           mma_commit(bar_empty + 8 * s);
         }
         if (!ok) break;
@@ -557,16 +576,19 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 
 constexpr int GEMM_BN = 256;  // fixed for the fused gate/up and LM-head modes
 
-bool encode_bf16_kmajor(CUtensorMap* map, const void* base, uint64_t rows, uint64_t k, uint32_t box_rows) {
+// K-major operand [rows, k] (bf16 or bytes) with boxes of 128 bytes x
+// box_rows, 128-byte swizzle; columns past k read as zero.
+bool encode_kmajor(CUtensorMap* map, const void* base, uint64_t rows, uint64_t k, uint32_t box_rows, bool bytes) {
   auto fn = encode_fn();
-  if (!fn || (k * 2) % 16 != 0 || ((uintptr_t)base & 15)) return false;
+  const uint64_t esz = bytes ? 1 : 2;
+  if (!fn || (k * esz) % 16 != 0 || ((uintptr_t)base & 15)) return false;
   cuuint64_t dims[2] = {k, rows};
-  cuuint64_t strides[1] = {k * 2};
-  cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
+  cuuint64_t strides[1] = {k * esz};
+  cuuint32_t box[2] = {(cuuint32_t)(128 / esz), box_rows};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  CUresult r = fn(map, bytes ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                  const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
 
@@ -608,19 +630,26 @@ int gemm_pick_bn(int M, int N, int sms) {
   return best;
 }
 
-bool gemm_make_plan(GemmPlan* plan, const uint16_t* a, int M, int K, const uint16_t* b, int N, bool any_bn) {
+namespace {
+
+bool make_plan(GemmPlan* plan, const void* a, int M, int K, const void* b, int N, bool any_bn, bool f8) {
   plan->M = M;
   plan->N = N;
   plan->K = K;
-  plan->bn = any_bn ? gemm_pick_bn(M, N, sm_count()) : GEMM_BN;
+  plan->f8 = f8 ? 1 : 0;
+  plan->bn = (any_bn && f8) ? gemm_pick_bn(M, N, sm_count()) : GEMM_BN;
   plan->o_ptr = nullptr;
   plan->o_ld = 0;
   plan->rope = 0;
-  // n fastest when A (M x K bf16) is too large to stay in L2 and B is not
-  const double a_bytes = 2.0 * M * K, b_bytes = 2.0 * N * K;
+  // n fastest when A (2 bytes per element either way) is too large to stay
+  // in L2 and B is not
+  const double a_bytes = 2.0 * M * K, b_bytes = (f8 ? 1.0 : 2.0) * N * K;
   plan->n_fast = (a_bytes > 64e6 && b_bytes < a_bytes) ? 1 : 0;
-  if (!encode_bf16_kmajor(&plan->a, a, (uint64_t)M, (uint64_t)K, BM) ||
-      !encode_bf16_kmajor(&plan->b, b, (uint64_t)N, (uint64_t)K, (uint32_t)plan->bn))
+  if (!encode_kmajor(&plan->a, a, (uint64_t)M, (uint64_t)K, BM, f8) ||
+      !encode_kmajor(&plan->b, b, (uint64_t)N, (uint64_t)K, (uint32_t)plan->bn, f8))
+    return false;
+  plan->a2 = plan->a;
+  if (f8 && !encode_kmajor(&plan->a2, (const uint8_t*)a + (size_t)M * K, (uint64_t)M, (uint64_t)K, BM, true))
     return false;
   // narrow units of the last wave: whole 32-column epilogue chunks, at least
   // 64 columns (an MMA of N 64 still reads all of A per k-step)
@@ -628,10 +657,20 @@ bool gemm_make_plan(GemmPlan* plan, const uint16_t* a, int M, int K, const uint1
   for (int f = 2; f <= 4; f *= 2) {
     const int w = plan->bn / f;
     if (w % 32 == 0 && w >= 64 &&
-        encode_bf16_kmajor(f == 2 ? &plan->b2 : &plan->b4, b, (uint64_t)N, (uint64_t)K, (uint32_t)w))
+        encode_kmajor(f == 2 ? &plan->b2 : &plan->b4, b, (uint64_t)N, (uint64_t)K, (uint32_t)w, f8))
       plan->narrow_ok |= f;
   }
   return true;
+}
+
+}  // namespace
+
+bool gemm_make_plan(GemmPlan* plan, const uint16_t* a, int M, int K, const uint16_t* b, int N, bool any_bn) {
+  return make_plan(plan, a, M, K, b, N, any_bn, false);
+}
+
+bool gemm_make_plan_f8(GemmPlan* plan, const uint8_t* a, int M, int K, const uint8_t* b, int N, bool any_bn) {
+  return make_plan(plan, a, M, K, b, N, any_bn, true);
 }
 
 int gemm_col_tiles(int N) { return (N + GEMM_BN - 1) / GEMM_BN; }
@@ -678,13 +717,14 @@ bool gemm_plan_output(GemmPlan* plan, float* out, int ldo) {
 
 namespace {
 
-template <int BN>
+template <int BN, bool F8>
 cudaError_t launch_bn(const GemmPlan& plan, const GemmArgs& args, cudaStream_t stream) {
   static bool attr_set = false;
-  constexpr int smem = GemmSmem<BN>::BYTES;
+  constexpr int smem = GemmSmem<BN, F8>::BYTES;
   static_assert(smem <= 232448, "shared memory");
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(k_bitlinear_gemm<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaError_t e =
+        cudaFuncSetAttribute(k_bitlinear_gemm<BN, F8>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
@@ -698,10 +738,11 @@ cudaError_t launch_bn(const GemmPlan& plan, const GemmArgs& args, cudaStream_t s
   a.split_s = 1;
   a.full_units = tiles;
   const int full = (tiles / (int)grid.x) * (int)grid.x, rem = tiles - full;
-  const int KB = (plan.K + BK - 1) / BK;
-  // (only long reductions: for K of a few thousand a tile's main loop is
-  // short next to the cost of writing and re-reading the partials)
-  if (a.split_ws && a.split_cnt && rem > 0 && full > 0 && KB >= 64 && !a.relu2 && !a.lse && (a.tma_out || a.rope)) {
+  const int KB = (plan.K + GemmSmem<BN, F8>::KE - 1) / GemmSmem<BN, F8>::KE;
+  // (only long reductions, K >= 4096: for K of a few thousand a tile's main
+  // loop is short next to the cost of writing and re-reading the partials)
+  if (a.split_ws && a.split_cnt && rem > 0 && full > 0 && plan.K >= 4096 && !a.relu2 && !a.lse &&
+      (a.tma_out || a.rope)) {
     int S = (int)grid.x / rem;
     if (S > 4) S = 4;
     if (S > KB) S = KB;
@@ -724,8 +765,8 @@ cudaError_t launch_bn(const GemmPlan& plan, const GemmArgs& args, cudaStream_t s
       break;
     }
   }
-  return launch_dependent(k_bitlinear_gemm<BN>, grid, dim3(GEMM_THREADS), smem, stream, plan.a, plan.b, *bn_map,
-                          plan.o, plan.q, plan.k, a);
+  return launch_dependent(k_bitlinear_gemm<BN, F8>, grid, dim3(GEMM_THREADS), smem, stream, plan.a, plan.a2, plan.b,
+                          *bn_map, plan.o, plan.q, plan.k, a);
 }
 
 }  // namespace
@@ -740,11 +781,12 @@ cudaError_t gemm_launch(const GemmPlan& plan, GemmArgs args, cudaStream_t stream
   if ((args.relu2 || args.lse) && plan.bn != GEMM_BN) return cudaErrorInvalidValue;
   if (!args.sw) return cudaErrorInvalidValue;  // every epilogue reads sw[0..2]
   ++kernel_launches();
+  if (!plan.f8) return plan.bn == 256 ? launch_bn<256, false>(plan, args, stream) : cudaErrorInvalidValue;
   switch (plan.bn) {
-    case 256: return launch_bn<256>(plan, args, stream);
-    case 192: return launch_bn<192>(plan, args, stream);
-    case 160: return launch_bn<160>(plan, args, stream);
-    case 128: return launch_bn<128>(plan, args, stream);
+    case 256: return launch_bn<256, true>(plan, args, stream);
+    case 192: return launch_bn<192, true>(plan, args, stream);
+    case 160: return launch_bn<160, true>(plan, args, stream);
+    case 128: return launch_bn<128, true>(plan, args, stream);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -63,8 +63,10 @@ int gemm_col_tiles(int N);
 
 struct GemmPlan {
   CUtensorMap a, b;
+  CUtensorMap a2;      // e4m3 plans: the lo matrix of A (a holds hi)
   CUtensorMap b2, b4;  // B with boxes of bn / 2 and bn / 4 rows (the narrow last-wave units)
   int narrow_ok;       // bit 1: b2 valid, bit 2: b4 valid
+  int f8;              // 1: e4m3 operands, kind::f8f6f4 (BitLinear); 0: bf16, kind::f16
   int M, N, K, bn;  // bn: output tile width (columns of B per tile)
   int n_fast;       // tile order: n fastest (A streamed once, B kept in L2)
   CUtensorMap o;    // fp32 output [M, N] (row stride o_ld): TMA store / reduce-add
@@ -86,27 +88,36 @@ bool gemm_plan_output(GemmPlan* plan, float* out, int ldo);
 
 // any_bn: the plan may use any tile width (store / residual-add epilogues);
 // otherwise 256 (fused gate/up and LM-head epilogues).
+// bf16 operands (the LM head): A [M, K], B [N, K]; 256-column tiles only.
 bool gemm_make_plan(GemmPlan* plan, const uint16_t* a, int M, int K, const uint16_t* b, int N, bool any_bn);
+// BitLinear: A the e4m3 (hi, lo) code pair [2, M, K] of launch_norm_quant, B
+// e4m3 ternary weights [N, K] (launch_expand_*); K a multiple of 16.  Every
+// product is an integer and every partial sum below 2^24, so the fp32
+// accumulator is the exact int32 dot product.
+bool gemm_make_plan_f8(GemmPlan* plan, const uint8_t* a, int M, int K, const uint8_t* b, int N, bool any_bn);
 int gemm_pick_bn(int M, int N, int sms);
 cudaError_t gemm_launch(const GemmPlan& plan, GemmArgs args, cudaStream_t stream);
 
 // ------------------------------------------------------------ forward ----
 // Per-row absmax int8 quantisation of h = RMSNorm(x) (gain != nullptr) or
-// of h = x (gain == nullptr): q bf16 [M, D] (ld = D), deq[m] = a / 127.
-void launch_norm_quant(const float* x, const float* gain, int M, int D, uint16_t* q, float* deq,
+// of h = x (gain == nullptr), deq[m] = a / 127.  Each code q is stored as the
+// e4m3 pair hi = 16 floor(q/16), lo = q - hi (both exact): q [2, M, D] bytes,
+// the hi matrix then the lo matrix (ld = D).
+void launch_norm_quant(const float* x, const float* gain, int M, int D, uint8_t* q, float* deq,
                        cudaStream_t s);
-// Packed 2-bit codes [rows, K/16] -> bf16 {-1, 0, +1} [rows, K].
-void launch_expand_codes(const uint32_t* words, uint64_t rows, int K, uint16_t* out, cudaStream_t s);
-// gate, up codes (two [F, K/16] word matrices) -> bf16 [256 * ceil(F/128), K]
+// Packed 2-bit codes [rows, K/16] -> e4m3 {-1, 0, +1} [rows, K] bytes.
+void launch_expand_codes(const uint32_t* words, uint64_t rows, int K, uint8_t* out, cudaStream_t s);
+// gate, up codes (two [F, K/16] word matrices) -> e4m3 [256 * ceil(F/128), K]
 // with 256-row tiles [gate rows 128b..128b+127 | up rows 128b..128b+127]
 // (rows beyond F are zero).
-void launch_expand_gate_up(const uint32_t* gate_words, const uint32_t* up_words, int F, int K, uint16_t* out,
+void launch_expand_gate_up(const uint32_t* gate_words, const uint32_t* up_words, int F, int K, uint8_t* out,
                            cudaStream_t s);
 // x[t] = embed[tok[t]].
 void launch_embed(const int32_t* tok, const float* embed, int T, int D, int V, float* x, unsigned* err,
                   cudaStream_t s);
-// Per-row absmax int8 quantisation of raw bf16 activations (no norm).
-void launch_norm_quant_bf16(const uint16_t* x, int M, int D, uint16_t* q, float* deq, cudaStream_t s);
+// Per-row absmax int8 quantisation of raw bf16 activations (no norm); q as
+// for launch_norm_quant.
+void launch_norm_quant_bf16(const uint16_t* x, int M, int D, uint8_t* q, float* deq, cudaStream_t s);
 // RoPE tables cos/sin fp32 [S, hd/2] computed in float64, rounded to fp32.
 void launch_rope_tables(int S, int hd, float* cosb, float* sinb, cudaStream_t s);
 // qkv fp32 [B*S, (H + 2 KV) hd] -> Q bf16 [B, H, S, hd] (RoPE), K bf16
