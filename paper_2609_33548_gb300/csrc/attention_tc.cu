@@ -33,12 +33,15 @@ namespace tmz {
 
 namespace {
 
-// Warp 0 TMA, warp 1 MMA (warps 2-3 idle): 136 registers a thread; warps 4-7
-// tile A, warps 8-11 tile B: 184.  128 x 136 + 256 x 184 = 384 x 168, the
-// registers the block is launched with.
-constexpr int ATT_THREADS = 384;
-constexpr int REG_CTRL = 136, REG_SOFTMAX = 184;
-static_assert(128 * REG_CTRL + 256 * REG_SOFTMAX == ATT_THREADS * 168, "register split");
+// Registers a thread after setmaxnreg: warp 0 TMA, warp 1 MMA (warps 2-3
+// idle) 96; the softmax warps 4-7 (tile A) and 8-11 (tile B) 168; the
+// epilogue warps 12-15 80.  128 x 96 + 256 x 168 + 128 x 80 = 512 x 128, the
+// registers the block is launched with (the host checks the kernel's register
+// count before its first launch: a smaller one would leave setmaxnreg.inc
+// waiting).  Of the splits that add up, this one spills least (24 bytes).
+constexpr int ATT_THREADS = 512;
+constexpr int REG_CTRL = 96, REG_SOFTMAX = 168, REG_EPI = 80, REG_LAUNCH = 128;
+static_assert(128 * REG_CTRL + 256 * REG_SOFTMAX + 128 * REG_EPI == ATT_THREADS * REG_LAUNCH, "register split");
 constexpr int BQ = 128, BKEY = 128;
 constexpr int ATOM = 128 * 128;  // one 128-row x 64-element bf16 swizzle atom block
 
@@ -51,7 +54,8 @@ struct AttTc {
   static constexpr int R_OFF = Q_OFF + 2 * TILE;   // ring
   static constexpr int P_OFF = R_OFF + NS * TILE;  // P_A, P_B: 128 x 128 bf16 each
   static constexpr int BAR_OFF = P_OFF + 2 * 2 * ATOM;
-  static constexpr int BYTES = BAR_OFF + 256 + 1024;
+  static constexpr int L_OFF = BAR_OFF + 512;      // l of each row of A, B (fp32)
+  static constexpr int BYTES = L_OFF + 2 * BQ * 4 + 1024;
 };
 
 struct AttItem {
@@ -225,8 +229,10 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
   const uint32_t bar = sb + L::BAR_OFF;
   const uint32_t q_full = bar, q_empty = bar + 8, ring_full = bar + 16, ring_empty = ring_full + 8 * NS,
                  s_full = ring_empty + 8 * NS, s_free = s_full + 16, p_full = s_free + 16, p_free = p_full + 16,
-                 o_full = p_free + 16, o_free = o_full + 16, fin = o_free + 16;
-  uint32_t* tmem_slot = (uint32_t*)(smem + L::BAR_OFF + 240);
+                 o_full = p_free + 16, o_free = o_full + 16, fin = o_free + 16, l_full = fin + 8,
+                 st_free = l_full + 16;
+  uint32_t* tmem_slot = (uint32_t*)(smem + L::BAR_OFF + 496);
+  static_assert(8 * (2 + 2 * (HD == 64 ? 6 : 3) + 12 + 1 + 4) <= 496, "barrier area");
 
   const int G = H / KV, NQ = S / BQ;
   const int n_items = B * KV * ((G * NQ + 1) / 2);
@@ -246,6 +252,8 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
       mbar_init(p_free + 8 * t, 1);
       mbar_init(o_full + 8 * t, 1);
       mbar_init(o_free + 8 * t, 4);
+      mbar_init(l_full + 8 * t, 4);
+      mbar_init(st_free + 8 * t, 4);
     }
     mbar_init(fin, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -396,18 +404,19 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
       if (!mbar_wait(fin, 0)) ok = false;
     }
   }
-  } else {
+  } else if (warp < 12) {
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(REG_SOFTMAX));
     // Softmax warps: warp w reads TMEM lanes 32 (w % 4) .. +31; lane = row.
     const int t = warp >= 8 ? 1 : 0;
     const int quarter = warp & 3;
     const int row = quarter * 32 + lane;
     const uint32_t lanes = (uint32_t)(quarter * 32) << 16;
-    const uint32_t tS = tmem + lanes + t * BKEY, tO = tmem + lanes + 256 + t * 128;
+    const uint32_t tS = tmem + lanes + t * BKEY;
     const uint32_t sfull = s_full + 8 * t, sfree = s_free + 8 * t, pfull = p_full + 8 * t, pfree = p_free + 8 * t,
-                   ofull = o_full + 8 * t, ofree = o_free + 8 * t;
+                   lfull = l_full + 8 * t, stfree = st_free + 8 * t;
     uint8_t* prow = smem + L::P_OFF + t * 2 * ATOM + row * 128;
-    uint32_t ns = 0, np = 0, no = 0;
+    float* lrow = reinterpret_cast<float*>(smem + L::L_OFF) + t * BQ + row;
+    uint32_t ns = 0, np = 0, nit = 0;
     auto arrive = [&](uint32_t b) {
       __syncwarp();
       if (lane == 0) mbar_arrive(b);
@@ -454,6 +463,9 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
         uint4 pk[8];
 #pragma unroll
         for (int ch = 0; ch < 8; ++ch) pk[ch] = p_chunk(sv, 8 * ch, sc2, m2, (ch & 1) ? lb : la);
+        // P of the item's first block overwrites the epilogue's staging of
+        // the previous item; later blocks wait for the P V that read P last
+        if (j == 0 && nit >= 1 && !(ok = mbar_wait_warp(stfree, (nit - 1) & 1u))) break;
         if (np >= 1 && !(ok = mbar_wait_warp(pfree, (np - 1) & 1u))) break;
 #pragma unroll
         for (int ch = 0; ch < 8; ++ch) *reinterpret_cast<uint4*>(prow + (((ch & 7) ^ (row & 7)) * 16)) = pk[ch];
@@ -466,48 +478,77 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
         ++np;
       }
       if (!ok) break;
-      const float l = __fadd_rn(__fadd_rn(la.x, la.y), __fadd_rn(lb.x, lb.y));
-      if (!(ok = mbar_wait_warp(ofull, no & 1u))) break;
-      ++no;
-      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-      // O / l staged through this tile's (now idle) P buffer in the 128-byte
-      // swizzled layout; each warp writes its own 32 rows with TMA stores of
-      // 32 x 32 fp32 boxes, so no warp waits on another
-      const float2 l2 = make_float2(l, l), y2 = make_float2(__frcp_rn(l), __frcp_rn(l));
-      const int orow = it.b * S + qt * BQ + quarter * 32, ocol0 = h * HD;
-      const uint32_t wbase = sb + L::P_OFF + t * 2 * ATOM + quarter * 32 * 128;
+      *lrow = __fadd_rn(__fadd_rn(la.x, la.y), __fadd_rn(lb.x, lb.y));
+      arrive(lfull);
+      ++nit;
+    }
+  } else {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(REG_EPI));
+    // Epilogue warps 12-15: warp w reads TMEM lanes 32 (w % 4) .. +31; lane =
+    // row.  Per item, tile A then tile B: O / l staged through the tile's P
+    // buffer (free once the item's last P V has completed) in the 128-byte
+    // swizzled layout; each warp writes its own 32 rows with TMA stores of
+    // 32 x 32 fp32 boxes.  The softmax warps meanwhile start the next item.
+    const int quarter = warp & 3;
+    const int row = quarter * 32 + lane;
+    const uint32_t lanes = (uint32_t)(quarter * 32) << 16;
+    uint32_t ne[2] = {0, 0};
+    auto arrive = [&](uint32_t b) {
+      __syncwarp();
+      if (lane == 0) mbar_arrive(b);
+    };
+    for (int r = 0; ok; ++r) {
+      if (r * (int)gridDim.x >= n_items) break;
+      const int i = att_sched(r, gridDim.x, blockIdx.x);
+      if (i >= n_items) continue;
+      const AttItem it = att_item(i, B, KV, G, NQ);
+      for (int t = 0; t < 2 && ok; ++t) {
+        const int qt = t ? it.qb : it.qa, h = t ? it.hb : it.ha;
+        if (h < 0) continue;
+        if (!(ok = mbar_wait_warp(l_full + 8 * t, ne[t] & 1u))) break;
+        if (!(ok = mbar_wait_warp(o_full + 8 * t, ne[t] & 1u))) break;
+        ++ne[t];
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        const float l = reinterpret_cast<const float*>(smem + L::L_OFF)[t * BQ + row];
+        const float2 l2 = make_float2(l, l), y2 = make_float2(__frcp_rn(l), __frcp_rn(l));
+        const int orow = it.b * S + qt * BQ + quarter * 32, ocol0 = h * HD;
+        const uint32_t tO = tmem + lanes + 256 + t * 128;
+        uint8_t* prow = smem + L::P_OFF + t * 2 * ATOM + row * 128;
+        const uint32_t wbase = sb + L::P_OFF + t * 2 * ATOM + quarter * 32 * 128;
 #pragma unroll 1
-      for (int rd = 0; rd < HD / 64; ++rd) {
-        if (rd > 0) {
-          if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+        for (int rd = 0; rd < HD / 64; ++rd) {
+          if (rd > 0) {
+            if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+            __syncwarp();
+          }
+#pragma unroll
+          for (int cc = 0; cc < 2; ++cc) {
+            uint32_t ov[32];
+            tmem_ld_cols<1>(tO + 64 * rd + 32 * cc, ov);
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              const float2 a = div2(make_float2(__uint_as_float(ov[4 * k]), __uint_as_float(ov[4 * k + 1])), l2, y2);
+              const float2 b =
+                  div2(make_float2(__uint_as_float(ov[4 * k + 2]), __uint_as_float(ov[4 * k + 3])), l2, y2);
+              *reinterpret_cast<float4*>(prow + cc * ATOM + ((k ^ (row & 7)) * 16)) = make_float4(a.x, a.y, b.x, b.y);
+            }
+          }
+          if (rd + 1 == HD / 64) {
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            arrive(o_free + 8 * t);
+          }
+          fence_async_smem();
           __syncwarp();
-        }
-#pragma unroll
-        for (int cc = 0; cc < 2; ++cc) {
-          uint32_t ov[32];
-          tmem_ld_cols<1>(tO + 64 * rd + 32 * cc, ov);
-#pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            const float2 a = div2(make_float2(__uint_as_float(ov[4 * k]), __uint_as_float(ov[4 * k + 1])), l2, y2);
-            const float2 b = div2(make_float2(__uint_as_float(ov[4 * k + 2]), __uint_as_float(ov[4 * k + 3])), l2, y2);
-            *reinterpret_cast<float4*>(prow + cc * ATOM + ((k ^ (row & 7)) * 16)) = make_float4(a.x, a.y, b.x, b.y);
+          if (lane == 0) {
+            tma_store_2d(&tmO, wbase, ocol0 + 64 * rd, orow);
+            tma_store_2d(&tmO, wbase + ATOM, ocol0 + 64 * rd + 32, orow);
+            asm volatile("cp.async.bulk.commit_group;" ::: "memory");
           }
         }
-        if (rd + 1 == HD / 64) {
-          asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-          arrive(ofree);
-        }
-        fence_async_smem();
-        __syncwarp();
-        if (lane == 0) {
-          tma_store_2d(&tmO, wbase, ocol0 + 64 * rd, orow);
-          tma_store_2d(&tmO, wbase + ATOM, ocol0 + 64 * rd + 32, orow);
-          asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-        }
+        // the staging (the tile's P buffer) is P again once the stores read it
+        if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+        arrive(st_free + 8 * t);
       }
-      // this warp's P rows are written again only after the stores have read them
-      if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
-      __syncwarp();
     }
     if (lane == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
   }
@@ -563,7 +604,13 @@ cudaError_t launch_tc(const AttnPlan& p, int B, int S, int H, int KV, unsigned* 
   static bool attr = false;
   constexpr int smem = AttTc<HD>::BYTES;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(k_attention_tc<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    // the warpgroups' setmaxnreg split adds up to exactly the registers of a
+    // launch at REG_LAUNCH per thread: any other count is refused here
+    cudaFuncAttributes fa;
+    cudaError_t e = cudaFuncGetAttributes(&fa, k_attention_tc<HD>);
+    if (e != cudaSuccess) return e;
+    if (fa.numRegs != REG_LAUNCH) return cudaErrorInvalidConfiguration;
+    e = cudaFuncSetAttribute(k_attention_tc<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     attr = true;
   }
