@@ -211,20 +211,22 @@ class OracleSample:
         return est, t_rq, t_fw
 
 
-def memory_report(cfg, density, peak_bytes):
+def memory_report(cfg, density, peak_bytes, weight_cache=False):
     """Device bytes by part (termezo_memory) next to the memory equation of
     Sec. 5 evaluated with this build's precisions (B = 4 fp32 latents,
     B_Q = 1/4, 32-bit active indices), and the peak torch allocation over the
-    timed steps (workspace + theta + batches)."""
+    timed steps (workspace + theta + batches).  The e4m3 weight cache, when
+    on, is its own part (d bytes, outside the equation)."""
     from paper_2609_33548_gb300 import termezo as tz
-    m = tz.termezo_memory(tz.make_cfg(cfg), density)
+    m = tz.termezo_memory(tz.make_cfg(cfg, weight_cache), density)
     d, k0 = m["d"], m["k_cap"]
     B, BQ = 4, 0.25
     eq_latent = d * B - math.ceil(d * (1 - density) * (B - BQ)) + math.ceil(density * d * BQ) + math.ceil(k0 * 4)
     gb = 1e9
     return {"workspace_gb": m["workspace"] / gb, "packed_codes_gb": m["packed"] / gb,
             "sparse_store_gb": (m["sparse_index"] + m["sparse_latents"]) / gb, "forward_gb": m["forward"] / gb,
-            "theta_gb": m["theta"] / gb, "peak_allocated_gb": peak_bytes / gb,
+            "theta_gb": m["theta"] / gb, "weight_cache_gb": m["weight_cache"] / gb,
+            "peak_allocated_gb": peak_bytes / gb,
             "latents": {"mezo_fp32_gb": d * B / gb, "equation_gb": eq_latent / gb,
                         "build_gb": (m["packed"] + m["sparse_index"] + m["sparse_latents"]) / gb,
                         "note": "build = equation + the second sparse-store buffer of the shrink"},
@@ -284,7 +286,7 @@ def run_mine(args):
     emb, gains, head = synth.theta(cfg, device=dev)
     nb = args.warmup + args.steps
     batches = [synth.batch(cfg, device=dev, step=i) for i in range(nb)]
-    ctx = tz.Context(tz.make_cfg(cfg), density, device=dev)
+    ctx = tz.Context(tz.make_cfg(cfg, args.weight_cache), density, device=dev)
     ctx.termezo_load_params(w, emb, gains, head)
     stream = torch.cuda.current_stream()
 
@@ -373,6 +375,7 @@ def run_mine(args):
                    "parallelism": f"replicas{world}", "layers": cfg.layers, "hidden": cfg.hidden,
                    "density": density, "k_active": int(outs[-1]["k_active"]), "eps": EPS, "lr": LR,
                    "directions": K, "theta_trained": bool(args.theta),
+                   "weight_cache": bool(args.weight_cache),
                    "l2": "no flush: per-step working set (521 MB packed codes, >1 GB activations) exceeds L2"},
         "steps_per_s": world * args.steps / (ms_max / 1e3),
         "roofline": {"bound": "tensor",
@@ -391,7 +394,7 @@ def run_mine(args):
                     "sparse_share": prof["sparse_ms"] / ms,
                     "mask_build_ms": build_ms, "mask_build_gbs": build_bytes / (build_ms / 1e3) / 1e9},
         "e2e": {"value": tokens / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-        "memory": memory_report(cfg, density, torch.cuda.max_memory_allocated(dev)),
+        "memory": memory_report(cfg, density, torch.cuda.max_memory_allocated(dev), args.weight_cache),
         "gpu_launches": int(prof["launches"]),
         "clocks": clocks,
         "last_step": {k: outs[-1][k] for k in ("loss_plus", "loss_minus", "g", "n_flipped", "n_jumps")},
@@ -524,6 +527,8 @@ def main():
                     help="Algorithm 1 as written: also perturb and update embeddings, norm gains and LM head")
     ap.add_argument("--op-shape", default="", help="N,K,M of the op workload's projection (default 6912,2560,2048)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--weight-cache", action="store_true",
+                    help="keep an e4m3 copy of the codes (d bytes) instead of expanding them before every GEMM")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -48,11 +48,18 @@ typedef struct termezo_ctx termezo_ctx;
  * loss_mode 0: cross-entropy of the last position over the n_labels label
  * tokens vocab-n_labels .. vocab-1 (targets = class ids [batch]).
  * loss_mode 1: token-level cross-entropy over the full vocabulary at every
- * position (targets = token ids [batch, seq]). */
+ * position (targets = token ids [batch, seq]).
+ * weight_cache != 0 (decoder contexts): the workspace also holds every
+ * weight's ternary code as one e4m3 byte (d bytes), kept equal to the packed
+ * 2-bit store by every call that rewrites codes, and the forward's GEMMs read
+ * it directly instead of expanding the packed codes of each projection
+ * before its GEMM.  It trades d bytes of device memory (not part of the
+ * paper's memory equation) for the expansion work.  Ignored for layers == 0. */
 typedef struct {
   int32_t layers, hidden, heads, kv_heads, ffn, vocab, seq, batch;
   int32_t loss_mode;
   int32_t n_labels;
+  int32_t weight_cache;
 } termezo_model_cfg;
 
 /* Per-step report (Algorithm 1 with K = 1; counters of Eq. 11). */
@@ -89,6 +96,7 @@ typedef struct {
   uint64_t theta;           /* the caller's embeddings (fp32), norm gains (fp32), LM head (bf16) */
   uint64_t mask_bitmask;    /* the paper's dense bit-mask option, ceil(d / 8) */
   uint64_t mask_index_list; /* the paper's index-list option, ceil(rho_0 d ceil(log2 d) / 8) */
+  uint64_t weight_cache;    /* e4m3 copy of the codes (weight_cache != 0), d bytes; else 0 */
 } termezo_memory_out;
 
 int termezo_memory(const termezo_model_cfg* cfg, double density, termezo_memory_out* out);

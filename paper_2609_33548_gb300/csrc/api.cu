@@ -22,6 +22,7 @@ constexpr uint32_t SPARSE_CHUNK = 4096;
 
 struct Shape {
   bool op;
+  bool wcache;  // e4m3 weight cache (decoder contexts)
   int L, D, H, KV, hd, F, V, S, B, T, C, mode;
   int P;
   std::vector<uint64_t> base;  // [P+1]
@@ -32,6 +33,7 @@ struct Shape {
 int make_shape(const termezo_model_cfg* c, Shape* s) {
   if (!c) return TERMEZO_EINVAL;
   s->op = c->layers == 0;
+  s->wcache = !s->op && c->weight_cache != 0;
   s->L = c->layers;
   s->D = c->hidden;
   s->F = c->ffn;
@@ -81,7 +83,7 @@ uint64_t keep_count(double density, uint64_t d) { return (uint64_t)std::floor(de
 
 // Bump allocator over the workspace; with base == nullptr it only measures.
 // Workspace sections, for the memory report.
-enum Section { SEC_PACKED, SEC_INDEX, SEC_LATENTS, SEC_MASK, SEC_FORWARD, SEC_COUNT };
+enum Section { SEC_PACKED, SEC_INDEX, SEC_LATENTS, SEC_MASK, SEC_FORWARD, SEC_WCACHE, SEC_COUNT };
 
 struct Carver {
   uint8_t* base;
@@ -133,6 +135,8 @@ struct termezo_ctx {
   float* attn = nullptr;
   float* gu = nullptr;
   uint8_t* wexp = nullptr;
+  uint8_t* wbyte = nullptr;  // weight cache: e4m3 code of every weight [d]
+  std::vector<GemmPlan> cplan;  // weight cache: per layer the q,k,v / o / gate,up / down plans
   float *cosb = nullptr, *sinb = nullptr;
   double* per_seq = nullptr;  // [2B]
   double* loss = nullptr;     // [2]
@@ -255,8 +259,15 @@ void carve(termezo_ctx* c, Carver& cv) {
   cv.sec = SEC_FORWARD;
   c->xq = cv.take<uint8_t>(2 * T * xq_cols(s));
   c->deq = cv.take<float>(T);
-  c->wexp = cv.take<uint8_t>(wexp_elems(s));
-  c->wexp2 = s.op ? nullptr : cv.take<uint8_t>(wexp_elems(s));
+  // expansion buffers, or (weight cache) one e4m3 byte per weight
+  c->wexp = s.wcache ? nullptr : cv.take<uint8_t>(wexp_elems(s));
+  c->wexp2 = (s.op || s.wcache) ? nullptr : cv.take<uint8_t>(wexp_elems(s));
+  if (s.wcache) {
+    cv.sec = SEC_WCACHE;
+    c->wbyte = cv.take<uint8_t>(s.d);
+    cv.sec = SEC_FORWARD;
+  }
+  a.wbyte = c->wbyte;
   c->split_cap = split_slots(s);
   c->split_ws = cv.take<float>((size_t)c->split_cap * 128 * 256);
   c->split_cnt = cv.take<unsigned>((size_t)c->split_cap * 4);
@@ -365,9 +376,11 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
   const int T = s.T, D = s.D, F = s.F, hq = s.H * s.hd, hkv = s.KV * s.hd;
   tmz::launch_embed(tokens, c->embed, T, D, s.V, c->x, c->ma.err, st);
   // Projection group g of layer l (0 q,k,v; 1 o; 2 gate,up; 3 down) is
-  // expanded to bf16 on the side stream into buffer g % 2 while the GEMM of
+  // expanded to e4m3 on the side stream into buffer g % 2 while the GEMM of
   // the group before it runs; the GEMM waits for its weights, and the next
-  // expansion into a buffer waits for the GEMM that read it last.
+  // expansion into a buffer waits for the GEMM that read it last.  With the
+  // weight cache the GEMMs read the cached codes and nothing is expanded.
+  const bool cached = c->wbyte != nullptr;
   uint8_t* wbuf[2] = {c->wexp, c->wexp2};
   cudaStream_t xs = c->xstream;
   auto expand = [&](int l, int g) {
@@ -385,23 +398,31 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
       tmz::launch_expand_codes(pk + s.base[proj_of(s, l, 6)] / 16, (uint64_t)D, F, wbuf[b], xs);
     cudaEventRecord(c->ev_ready[b], xs);
   };
-  auto gemm = [&](int l, int g, const GemmPlan& plan, GemmArgs a, double flops) -> bool {
+  auto plan_of = [&](int l, int g) -> const GemmPlan& {
+    if (cached) return c->cplan[(size_t)4 * l + g];
+    return g == 0 ? c->plan_qkv : g == 1 ? c->plan_o : g == 2 ? c->plan_gu : c->plan_down;
+  };
+  auto gemm = [&](int l, int g, GemmArgs a, double flops) -> bool {
+    const GemmPlan& plan = plan_of(l, g);
     a.split_ws = c->split_ws;
     a.split_cnt = c->split_cnt;
     a.split_cap = c->split_cap;
-    cudaStreamWaitEvent(st, c->ev_ready[g & 1], 0);
+    if (!cached) cudaStreamWaitEvent(st, c->ev_ready[g & 1], 0);
     {
-      ProfScope ps(c, 0, flops);
+      ProfScope ps(c, 0, flops > 0 ? flops : gemm_flops(plan));
       if (tmz::gemm_launch(plan, a, st) != cudaSuccess) return false;
     }
+    if (cached) return true;
     cudaEventRecord(c->ev_free[g & 1], st);
     const int nl = g == 3 ? l + 1 : l, ng = (g + 1) & 3;
     if (nl < s.L) expand(nl, ng);
     return true;
   };
-  cudaEventRecord(c->ev_codes, st);
-  cudaStreamWaitEvent(xs, c->ev_codes, 0);
-  expand(0, 0);
+  if (!cached) {
+    cudaEventRecord(c->ev_codes, st);
+    cudaStreamWaitEvent(xs, c->ev_codes, 0);
+    expand(0, 0);
+  }
   for (int l = 0; l < s.L; ++l) {
     const int pq = proj_of(s, l, 0), po = proj_of(s, l, 3), pg = proj_of(s, l, 4), pd = proj_of(s, l, 6);
     // attention block
@@ -415,7 +436,8 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
     a.n1 = hq;
     a.n2 = hq + hkv;
     a.err = c->ma.err;
-    if (c->plan_qkv.rope) {
+    const bool rope = plan_of(l, 0).rope != 0;
+    if (rope) {
       a.rope = 1;
       a.cosb = c->cosb;
       a.sinb = c->sinb;
@@ -425,8 +447,8 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
       a.KV = s.KV;
       a.hd = s.hd;
     }
-    if (!gemm(l, 0, c->plan_qkv, a, gemm_flops(c->plan_qkv))) return TERMEZO_ECUDA;
-    if (!c->plan_qkv.rope)
+    if (!gemm(l, 0, a, 0.0)) return TERMEZO_ECUDA;
+    if (!rope)
       tmz::launch_rope_pack(c->qkv, c->cosb, c->sinb, s.B, s.S, s.H, s.KV, s.hd, c->qb, c->kb, c->vt, st);
     a.rope = 0;  // the remaining projections of the layer reuse a
     {
@@ -444,7 +466,7 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
     a.mode = 1;
     a.sw = sw + po;
     a.n1 = a.n2 = D;
-    if (!gemm(l, 1, c->plan_o, a, gemm_flops(c->plan_o))) return TERMEZO_ECUDA;
+    if (!gemm(l, 1, a, 0.0)) return TERMEZO_ECUDA;
     // MLP block
     tmz::launch_norm_quant(c->x, c->gains + (size_t)(2 * l + 1) * D, T, D, c->xq, c->deq, st);
     a.out = c->gu;  // hid = relu(gate)^2 * up, fp32 [T, F]
@@ -454,7 +476,7 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
     a.n1 = a.n2 = a.N;
     a.relu2 = 1;
     a.n_out = F;
-    if (!gemm(l, 2, c->plan_gu, a, 2.0 * T * (2.0 * F) * D)) return TERMEZO_ECUDA;
+    if (!gemm(l, 2, a, 2.0 * T * (2.0 * F) * D)) return TERMEZO_ECUDA;
     a.relu2 = 0;
     tmz::launch_norm_quant(c->gu, nullptr, T, F, c->xq, c->deq, st);
     a.out = c->x;
@@ -462,7 +484,7 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
     a.mode = 1;
     a.sw = sw + pd;
     a.n1 = a.n2 = D;
-    if (!gemm(l, 3, c->plan_down, a, gemm_flops(c->plan_down))) return TERMEZO_ECUDA;
+    if (!gemm(l, 3, a, 0.0)) return TERMEZO_ECUDA;
   }
   if (s.mode == 0) {
     tmz::launch_head_ce_last(c->x, c->gains + (size_t)(2 * s.L) * D, c->head, targets, s.B, s.S, D, s.V, s.C,
@@ -535,6 +557,7 @@ int termezo_memory(const termezo_model_cfg* cfg, double density, termezo_memory_
   out->sparse_latents = cv.bytes[SEC_LATENTS];
   out->mask_state = cv.bytes[SEC_MASK];
   out->forward = cv.bytes[SEC_FORWARD];
+  out->weight_cache = cv.bytes[SEC_WCACHE];
   out->workspace = cv.off + 256;
   out->theta = s.op ? 0
                     : (uint64_t)s.V * s.D * 4 + (uint64_t)(2 * s.L + 1) * s.D * 4 + (uint64_t)s.V * s.D * 2;
@@ -587,10 +610,24 @@ int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspa
     tmz::launch_rope_tables(s.S, s.hd, c->cosb, c->sinb, st);
     const int T = s.T, D = s.D, F = s.F, hq = s.H * s.hd, hkv = s.KV * s.hd;
     const bool rope_fused = rope_fused_shape(s);
-    bool ok = tmz::gemm_make_plan_f8(&c->plan_qkv, c->xq, T, D, c->wexp, hq + 2 * hkv, !rope_fused) &&
-              tmz::gemm_make_plan_f8(&c->plan_o, c->xq, T, hq, c->wexp2, D, true) &&
-              tmz::gemm_make_plan_f8(&c->plan_gu, c->xq, T, D, c->wexp, 256 * ((F + 127) / 128), false) &&
-              tmz::gemm_make_plan_f8(&c->plan_down, c->xq, T, F, c->wexp2, D, true);
+    // the expansion buffers' plans, or (weight cache) every layer's own
+    bool ok = s.wcache ||
+              (tmz::gemm_make_plan_f8(&c->plan_qkv, c->xq, T, D, c->wexp, hq + 2 * hkv, !rope_fused) &&
+               tmz::gemm_make_plan_f8(&c->plan_o, c->xq, T, hq, c->wexp2, D, true) &&
+               tmz::gemm_make_plan_f8(&c->plan_gu, c->xq, T, D, c->wexp, 256 * ((F + 127) / 128), false) &&
+               tmz::gemm_make_plan_f8(&c->plan_down, c->xq, T, F, c->wexp2, D, true));
+    if (s.wcache) {
+      c->cplan.resize((size_t)4 * s.L);
+      for (int l = 0; l < s.L && ok; ++l) {
+        GemmPlan* p = &c->cplan[(size_t)4 * l];
+        const uint8_t* w = c->wbyte;
+        ok = tmz::gemm_make_plan_f8(&p[0], c->xq, T, D, w + s.base[proj_of(s, l, 0)], hq + 2 * hkv, !rope_fused) &&
+             tmz::gemm_make_plan_f8(&p[1], c->xq, T, hq, w + s.base[proj_of(s, l, 3)], D, true) &&
+             tmz::gemm_make_plan_f8_gu(&p[2], c->xq, T, D, w + s.base[proj_of(s, l, 4)], w + s.base[proj_of(s, l, 5)],
+                                       F) &&
+             tmz::gemm_make_plan_f8(&p[3], c->xq, T, F, w + s.base[proj_of(s, l, 6)], D, true);
+      }
+    }
     ok = ok && cudaStreamCreateWithFlags(&c->xstream, cudaStreamNonBlocking) == cudaSuccess;
     for (cudaEvent_t* e : {&c->ev_free[0], &c->ev_free[1], &c->ev_ready[0], &c->ev_ready[1], &c->ev_codes})
       ok = ok && cudaEventCreateWithFlags(e, cudaEventDisableTiming) == cudaSuccess;
@@ -601,17 +638,22 @@ int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspa
     // TMA output maps (a layout that does not allow one keeps the plain stores)
     // q, k, v written by the QKV GEMM's epilogue (RoPE fused) where the head
     // layout allows it
-    if (rope_fused) {
-      // the workspace has no fp32 QKV buffer for these shapes
-      if (!tmz::gemm_plan_rope(&c->plan_qkv, c->qb, c->kb, s.B, s.S, s.H, s.KV, s.hd)) {
-        delete c;
-        return TERMEZO_ECUDA;
+    const int n_sets = s.wcache ? s.L : 1;
+    for (int l = 0; l < n_sets; ++l) {
+      GemmPlan *pq = s.wcache ? &c->cplan[(size_t)4 * l] : &c->plan_qkv,
+               *po = s.wcache ? pq + 1 : &c->plan_o, *pd = s.wcache ? pq + 3 : &c->plan_down;
+      if (rope_fused) {
+        // the workspace has no fp32 QKV buffer for these shapes
+        if (!tmz::gemm_plan_rope(pq, c->qb, c->kb, s.B, s.S, s.H, s.KV, s.hd)) {
+          delete c;
+          return TERMEZO_ECUDA;
+        }
+      } else {
+        tmz::gemm_plan_output(pq, c->qkv, hq + 2 * hkv);
       }
-    } else {
-      tmz::gemm_plan_output(&c->plan_qkv, c->qkv, hq + 2 * hkv);
+      tmz::gemm_plan_output(po, c->x, D);
+      tmz::gemm_plan_output(pd, c->x, D);
     }
-    tmz::gemm_plan_output(&c->plan_o, c->x, D);
-    tmz::gemm_plan_output(&c->plan_down, c->x, D);
     c->att_tc = tmz::attention_tc_supported(s.S, s.hd) &&
                 tmz::attention_tc_plan(&c->att_plan, c->qb, c->kb, c->vt, c->attn, s.B, s.S, s.H, s.KV, s.hd);
   }

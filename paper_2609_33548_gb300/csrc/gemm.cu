@@ -105,8 +105,9 @@ template <int BN, bool F8>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     k_bitlinear_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmA2,
                      const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmBn,
-                     const __grid_constant__ CUtensorMap tmO, const __grid_constant__ CUtensorMap tmQ,
-                     const __grid_constant__ CUtensorMap tmK, GemmArgs p) {
+                     const __grid_constant__ CUtensorMap tmBu, const __grid_constant__ CUtensorMap tmO,
+                     const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                     GemmArgs p) {
   using L = GemmSmem<BN, F8>;
   constexpr int STAGES = L::STAGES;
   extern __shared__ uint8_t smem_raw[];
@@ -142,6 +143,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     if (F8) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmA2) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmB) : "memory");
     if (p.nsplit > 1) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmBn) : "memory");
+    if (p.gu_split) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmBu) : "memory");
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
@@ -173,7 +175,13 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           mbar_expect_tx(bar_full + 8 * s, narrow ? L::A_BYTES + w.nw * 128 : L::STAGE_BYTES);
           tma_load_2d(sa, &tmA, kb * L::KE, m0, bar_full + 8 * s);
           if (F8) tma_load_2d(sa + L::A_TILE, &tmA2, kb * L::KE, m0, bar_full + 8 * s);
-          tma_load_2d(sa + L::A_BYTES, narrow ? &tmBn : &tmB, kb * L::KE, n0 + w.c0, bar_full + 8 * s);
+          if (p.gu_split) {
+            // gate rows 128 j.. then up rows 128 j.. of tile j (BN 256)
+            tma_load_2d(sa + L::A_BYTES, &tmB, kb * L::KE, n0 / 2, bar_full + 8 * s);
+            tma_load_2d(sa + L::A_BYTES + 128 * 128, &tmBu, kb * L::KE, n0 / 2, bar_full + 8 * s);
+          } else {
+            tma_load_2d(sa + L::A_BYTES, narrow ? &tmBn : &tmB, kb * L::KE, n0 + w.c0, bar_full + 8 * s);
+          }
         }
       }
     }
@@ -649,6 +657,8 @@ bool make_plan(GemmPlan* plan, const void* a, int M, int K, const void* b, int N
       !encode_kmajor(&plan->b, b, (uint64_t)N, (uint64_t)K, (uint32_t)plan->bn, f8))
     return false;
   plan->a2 = plan->a;
+  plan->b_up = plan->b;
+  plan->gu_split = 0;
   if (f8 && !encode_kmajor(&plan->a2, (const uint8_t*)a + (size_t)M * K, (uint64_t)M, (uint64_t)K, BM, true))
     return false;
   // narrow units of the last wave: whole 32-column epilogue chunks, at least
@@ -671,6 +681,16 @@ bool gemm_make_plan(GemmPlan* plan, const uint16_t* a, int M, int K, const uint1
 
 bool gemm_make_plan_f8(GemmPlan* plan, const uint8_t* a, int M, int K, const uint8_t* b, int N, bool any_bn) {
   return make_plan(plan, a, M, K, b, N, any_bn, true);
+}
+
+bool gemm_make_plan_f8_gu(GemmPlan* plan, const uint8_t* a, int M, int K, const uint8_t* gate, const uint8_t* up,
+                          int F) {
+  if (!make_plan(plan, a, M, K, gate, 256 * ((F + 127) / 128), false, true)) return false;
+  // B boxes of 128 rows from each matrix; no narrow last-wave units
+  plan->narrow_ok = 0;
+  plan->gu_split = 1;
+  return encode_kmajor(&plan->b, gate, (uint64_t)F, (uint64_t)K, 128, true) &&
+         encode_kmajor(&plan->b_up, up, (uint64_t)F, (uint64_t)K, 128, true);
 }
 
 int gemm_col_tiles(int N) { return (N + GEMM_BN - 1) / GEMM_BN; }
@@ -766,7 +786,7 @@ cudaError_t launch_bn(const GemmPlan& plan, const GemmArgs& args, cudaStream_t s
     }
   }
   return launch_dependent(k_bitlinear_gemm<BN, F8>, grid, dim3(GEMM_THREADS), smem, stream, plan.a, plan.a2, plan.b,
-                          *bn_map, plan.o, plan.q, plan.k, a);
+                          *bn_map, plan.b_up, plan.o, plan.q, plan.k, a);
 }
 
 }  // namespace
@@ -776,6 +796,8 @@ cudaError_t gemm_launch(const GemmPlan& plan, GemmArgs args, cudaStream_t stream
   args.N = plan.N;
   args.K = plan.K;
   args.n_fast = plan.n_fast;
+  args.gu_split = plan.gu_split;
+  if (plan.gu_split && (!args.relu2 || plan.bn != 256)) return cudaErrorInvalidValue;
   if (args.rope && (!plan.rope || plan.bn % args.hd)) return cudaErrorInvalidValue;
   args.tma_out = (plan.o_ptr && args.out == plan.o_ptr && args.ldo == plan.o_ld && !args.relu2 && !args.lse) ? 1 : 0;
   if ((args.relu2 || args.lse) && plan.bn != GEMM_BN) return cudaErrorInvalidValue;

@@ -51,6 +51,7 @@ struct GemmArgs {
   // split N of the last wave (set at launch; exclusive with split_s > 1):
   // its tiles become nsplit units of BN / nsplit columns each (1: no split)
   int nsplit;
+  int gu_split;  // filled from the plan: gate and up rows from two B maps
   int rope;
   const float* cosb;
   const float* sinb;
@@ -67,6 +68,8 @@ struct GemmPlan {
   CUtensorMap b2, b4;  // B with boxes of bn / 2 and bn / 4 rows (the narrow last-wave units)
   int narrow_ok;       // bit 1: b2 valid, bit 2: b4 valid
   int f8;              // 1: e4m3 operands, kind::f8f6f4 (BitLinear); 0: bf16, kind::f16
+  CUtensorMap b_up;    // gu_split: B tile rows 0..127 from b (gate), 128..255 from b_up
+  int gu_split;
   int M, N, K, bn;  // bn: output tile width (columns of B per tile)
   int n_fast;       // tile order: n fastest (A streamed once, B kept in L2)
   CUtensorMap o;    // fp32 output [M, N] (row stride o_ld): TMA store / reduce-add
@@ -95,6 +98,11 @@ bool gemm_make_plan(GemmPlan* plan, const uint16_t* a, int M, int K, const uint1
 // product is an integer and every partial sum below 2^24, so the fp32
 // accumulator is the exact int32 dot product.
 bool gemm_make_plan_f8(GemmPlan* plan, const uint8_t* a, int M, int K, const uint8_t* b, int N, bool any_bn);
+// The fused gate/up projection straight from two e4m3 weight matrices gate,
+// up [F, K]: tile j pairs gate rows 128 j .. 128 j + 127 with the same up rows
+// (the layout launch_expand_gate_up writes; rows past F read as zero).
+bool gemm_make_plan_f8_gu(GemmPlan* plan, const uint8_t* a, int M, int K, const uint8_t* gate, const uint8_t* up,
+                          int F);
 int gemm_pick_bn(int M, int N, int sms);
 cudaError_t gemm_launch(const GemmPlan& plan, GemmArgs args, cudaStream_t stream);
 

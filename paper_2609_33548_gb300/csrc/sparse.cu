@@ -16,6 +16,9 @@ namespace tmz {
 
 namespace {
 
+// e4m3 byte of a stored code (q + 1 in {0, 1, 2}): -1 = 0xB8, 0 = 0x00, +1 = 0x38.
+__device__ __forceinline__ uint8_t code_e4m3(uint32_t c) { return c == 2u ? 0x38 : (c == 0u ? 0xB8 : 0x00); }
+
 constexpr int TPB = 256;
 constexpr uint32_t DENSE_CHUNK = 4096;  // elements per dense block (16 per thread)
 
@@ -317,6 +320,14 @@ __global__ void __launch_bounds__(TPB) k_compact(MaskArgs a, const float* __rest
       word |= ternary_code(v[j], tau) << (2 * j);
     }
     a.packed[i0 >> 4] = word;
+    if (a.wbyte) {
+      uint32_t b[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        b[q] = code_e4m3((word >> (8 * q)) & 3u) | (code_e4m3((word >> (8 * q + 2)) & 3u) << 8) |
+               (code_e4m3((word >> (8 * q + 4)) & 3u) << 16) | (code_e4m3((word >> (8 * q + 6)) & 3u) << 24);
+      *reinterpret_cast<uint4*>(a.wbyte + i0) = make_uint4(b[0], b[1], b[2], b[3]);
+    }
   }
   unsigned long long tie_rank = (unsigned long long)a.blk_d[blockIdx.x] + block_excl_scan(eq, sh, nullptr);
   uint32_t selmask = 0, nsel = 0;
@@ -448,6 +459,7 @@ __global__ void __launch_bounds__(TPB) k_sparse_requant(MaskArgs a, int cur, uin
         uint32_t c, cp;
         requant_codes(a, sign, seed, eps, tau, taup, idx[r.beg + j], lat[r.beg + j], &c, &cp);
         sc[j] = (uint8_t)(c | (cp << 2));
+        if (a.wbyte) a.wbyte[idx[r.beg + j]] = code_e4m3(c);
       }
     }
   }
@@ -569,8 +581,9 @@ __global__ void __launch_bounds__(TPB) k_shrink_mark(MaskArgs a, int cur) {
       if ((i2 >> 4) != wi) break;
       const float w2 = lat[e2];
       if (boundary_distance(w2, tau) > xi0) {
-        const uint32_t shf = 2 * (i2 & 15u);
-        word = (word & ~(3u << shf)) | (ternary_code(w2, tau) << shf);
+        const uint32_t shf = 2 * (i2 & 15u), code = ternary_code(w2, tau);
+        word = (word & ~(3u << shf)) | (code << shf);
+        if (a.wbyte) a.wbyte[i2] = code_e4m3(code);
         touched = true;
       }
     }

@@ -26,6 +26,8 @@ struct MaskArgs {
   const uint16_t* sproj;        // [NBS] projection of each sparse block
   uint32_t NBS;                 // sparse blocks
   uint32_t* packed;             // [d/16] 2-bit codes
+  uint8_t* wbyte;               // [d] the same codes as e4m3 bytes (+1, 0, -1), or null: every
+                                // kernel that writes packed codes writes these bytes too
   uint32_t* idx[2];             // active global indices (double buffer)
   float* lat[2];                // active latents
   uint32_t* off[2];             // [P+1] segment offsets into idx/lat

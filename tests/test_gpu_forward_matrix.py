@@ -32,13 +32,16 @@ MATRIX = {
 }
 
 
-@pytest.mark.parametrize("name", sorted(MATRIX))
-def test_forward_loss_matrix(name):
+CACHED = ("hd128-gqa", "narrow-tail", "gqa-long-sft")
+
+
+@pytest.mark.parametrize("name,cache", [(n, False) for n in sorted(MATRIX)] + [(n, True) for n in CACHED])
+def test_forward_loss_matrix(name, cache):
     cfg = MATRIX[name]
     w = synth.latents(cfg)
     emb, gains, head = synth.theta(cfg)
     tok, tgt = synth.batch(cfg)
-    ctx = tz.Context(tz.make_cfg(cfg), 0.01)
+    ctx = tz.Context(tz.make_cfg(cfg, cache), 0.01)
     dev = [t.cuda() for t in (w, emb, gains, head, tok, tgt)]
     ctx.termezo_load_params(dev[0], dev[1], dev[2], dev[3])
     ctx.termezo_build_mask(0.01)

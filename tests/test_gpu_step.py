@@ -34,18 +34,21 @@ TINY_SFT = dataclasses.replace(synth.TINY, name="tiny-2L-d256-sft", vocab=1000, 
 DENSITY, EPS, LR = 0.01, 1e-3, 1e-6
 
 
-@pytest.fixture(scope="module", params=[synth.TINY, TINY_SFT], ids=["last-token", "token-level"])
+# every step test runs with the GEMMs reading packed codes expanded before each
+# GEMM and with the e4m3 weight cache that the sparse kernels keep in step
+@pytest.fixture(scope="module", params=[(synth.TINY, False), (TINY_SFT, False), (synth.TINY, True), (TINY_SFT, True)],
+                ids=["last-token", "token-level", "last-token-cache", "token-level-cache"])
 def inputs(request):
-    cfg = request.param
+    cfg, cache = request.param
     w = synth.latents(cfg)
     emb, gains, head = synth.theta(cfg)
     tok, tgt = synth.batch(cfg)
-    return w, emb, gains, head, tok, tgt, cfg
+    return w, emb, gains, head, tok, tgt, cfg, cache
 
 
 def _gpu_ctx(inputs):
-    w, emb, gains, head, tok, tgt, CFG = inputs
-    ctx = tz.Context(tz.make_cfg(CFG), DENSITY)
+    w, emb, gains, head, tok, tgt, CFG, cache = inputs
+    ctx = tz.Context(tz.make_cfg(CFG, cache), DENSITY)
     dev = [t.cuda() for t in (w, emb, gains, head, tok, tgt)]
     ctx.termezo_load_params(dev[0], dev[1], dev[2], dev[3])
     return ctx, dev
@@ -241,7 +244,7 @@ def test_joint_theta_step_matches_oracle(inputs):
     rounding and the bf16 head in all but a rare element that rounds to a
     neighbouring bf16 value."""
     K = 2
-    w0, emb0, gains0, head0, tok, tgt, cfg = inputs
+    w0, emb0, gains0, head0, tok, tgt, cfg, _ = inputs
     ctx, dev = _gpu_ctx(inputs)
     ctx.termezo_build_mask(DENSITY)
     reg = otz.registry(cfg)

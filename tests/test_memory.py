@@ -28,7 +28,8 @@ def test_memory_report_parts(cfg, density):
     assert d // 4 <= m["packed"] < d // 4 + 256
     assert 2 * 4 * k0 <= m["sparse_index"] < 2 * 4 * k0 + 2 * 256
     assert 2 * 4 * k0 <= m["sparse_latents"] < 2 * 4 * k0 + 2 * 256
-    parts = m["packed"] + m["sparse_index"] + m["sparse_latents"] + m["mask_state"] + m["forward"]
+    parts = m["packed"] + m["sparse_index"] + m["sparse_latents"] + m["mask_state"] + m["forward"] + m["weight_cache"]
+    assert m["weight_cache"] == 0
     assert m["workspace"] == parts + 256 == tz.termezo_workspace_bytes(tz.make_cfg(cfg), density)
     assert m["theta"] == cfg.vocab * cfg.hidden * (4 + 2) + (2 * cfg.layers + 1) * cfg.hidden * 4
     # the paper's two mask options
@@ -51,3 +52,17 @@ def test_latent_storage_against_the_memory_equation():
     assert abs(build - eq) <= 4 * 256 + 8
     # at 1 % the index list beats the bit mask, as Sec. 5 expects for small rho_0
     assert m["mask_index_list"] < m["mask_bitmask"]
+
+
+@pytest.mark.parametrize("cfg,density", CASES, ids=[f"{c.name}-{d}" for c, d in CASES])
+def test_weight_cache_part(cfg, density):
+    """The e4m3 weight cache is one byte per weight, its own part; the two
+    expansion buffers it replaces leave the forward part."""
+    m0 = tz.termezo_memory(tz.make_cfg(cfg), density)
+    m1 = tz.termezo_memory(tz.make_cfg(cfg, weight_cache=True), density)
+    d = cfg.d_lat
+    assert d <= m1["weight_cache"] < d + 256
+    assert m1["forward"] < m0["forward"]
+    assert m1["workspace"] - m0["workspace"] == m1["weight_cache"] - (m0["forward"] - m1["forward"])
+    for k in ("packed", "sparse_index", "sparse_latents", "mask_state", "theta"):
+        assert m1[k] == m0[k]
