@@ -101,13 +101,27 @@ __device__ __forceinline__ Unit unit_of(const GemmArgs& p, int u, int KB) {
 // HBM once.  The
 // accumulator is double-buffered in tensor memory (2 x BN columns) so that
 // the epilogue of one tile overlaps the main loop of the next.
+// Named barrier 1 over the four epilogue warps (128 threads).  Every epilogue
+// warp reaches each use in the same unit and chunk: the loop over units is
+// uniform, and a failed wait is made uniform first (epi_all).
+__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+__device__ __forceinline__ bool epi_all(bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.and.pred q, 1, 128, p;\n selp.u32 %0, 1, 0, q;\n}\n"
+      : "=r"(r)
+      : "r"((uint32_t)v)
+      : "memory");
+  return r != 0;
+}
+
 template <int BN, bool F8>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     k_bitlinear_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmA2,
                      const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmBn,
                      const __grid_constant__ CUtensorMap tmBu, const __grid_constant__ CUtensorMap tmO,
-                     const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                     GemmArgs p) {
+                     const __grid_constant__ CUtensorMap tmO32, const __grid_constant__ CUtensorMap tmQ,
+                     const __grid_constant__ CUtensorMap tmK, GemmArgs p) {
   using L = GemmSmem<BN, F8>;
   constexpr int STAGES = L::STAGES;
   extern __shared__ uint8_t smem_raw[];
@@ -234,6 +248,14 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     // TMA output path: this warp's two swizzled 32 x 32 staging tiles
     uint8_t* otile = smem + L::EPI_OFF + (warp - 2) * 2 * 4096;
     uint32_t n_out_tiles = 0;
+    // TMA output of whole tiles: the four warps stage one 128-row x 32-column
+    // fp32 block (16 KB, two buffers) and one thread issues its store or
+    // reduce-add, so the epilogue takes 8 TMA operations a tile instead of 32
+    // and leaves the TMA unit to the operand loads
+    uint8_t* gbuf = smem + L::EPI_OFF;
+    const bool issuer = warp == 2 && lane == 0;
+    uint32_t n_grp = 0;
+    bool drained = false;
     float* dqs = stage + 32 * EPI_LD;  // the 32 rows' activation scales
     const float s0 = p.sw[0], s1 = p.sw[1], s2 = p.sw[2];
     uint32_t local = 0;
@@ -263,8 +285,15 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         for (int rr = 0; rr < 32; ++rr)
           prev[rr] = (rr < nrows && col < p.N) ? p.out[(size_t)(row0 + rr) * p.ldo + col] : 0.f;
       }
-      ok = mbar_wait(bar_tfull + 8 * b, j & 1u);
+      ok = epi_all(mbar_wait(bar_tfull + 8 * b, j & 1u));
       if (!ok) break;
+      // a K-split tail unit stages per warp (each warp decides alone whether
+      // it finishes its rows): the whole-tile buffers must be read out first
+      if (tma_path && w.tail >= 0 && n_grp > 0 && !drained) {
+        if (issuer) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+        epi_bar();
+        drained = true;
+      }
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       const uint32_t tacc = tmem + ((uint32_t)(quarter * 32) << 16) + b * L::ACC_STRIDE;
       bool from_parts = false;
@@ -458,12 +487,14 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         }
       }
       if (tma_path) {
-        // lane = row: y = acc (a/127)[row] s_w[col] written by this warp as
-        // 32 x 32 tiles through shared memory with a TMA store, or added into
-        // the residual stream with a TMA reduce-add (one fp32 add, rounded to
-        // nearest, per element: the same value as out + y)
+        // lane = row: y = acc (a/127)[row] s_w[col] through shared memory with
+        // a TMA store, or added into the residual stream with a TMA
+        // reduce-add (one fp32 add, rounded to nearest, per element: the same
+        // value as out + y); whole tiles as 128 x 32 blocks of the four warps,
+        // K-split tail units as 32 x 32 blocks of each warp
         const float dq = dq_row;
         const int row = row0 + lane;
+        const bool group = w.tail < 0;
         for (int c = 0; c < ncols / 32; ++c) {
           const int col0 = n0 + c * 32;
           if (col0 >= p.N) break;
@@ -474,10 +505,18 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
             for (int q = 0; q < 32; ++q)
               if (col0 + q < p.N) p.acc_out[(size_t)row * p.N + col0 + q] = __float2int_rn(__uint_as_float(r[q]));
           }
-          uint8_t* ot = otile + (n_out_tiles & 1u) * 4096;
-          if (n_out_tiles >= 2) {
-            if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
-            __syncwarp();
+          uint8_t* ot;
+          if (group) {
+            // the buffer was last read by the store of two blocks ago
+            if (issuer && n_grp >= 2) asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+            epi_bar();
+            ot = gbuf + (n_grp & 1u) * 16384 + quarter * 4096;
+          } else {
+            ot = otile + (n_out_tiles & 1u) * 4096;
+            if (n_out_tiles >= 2) {
+              if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+              __syncwarp();
+            }
           }
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
@@ -491,23 +530,32 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
             *reinterpret_cast<float4*>(ot + lane * 128 + ((k ^ (lane & 7)) * 16)) = make_float4(v[0], v[1], v[2], v[3]);
           }
           asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-          __syncwarp();
-          if (lane == 0) {
-            const uint32_t src = smem_u32(ot);
+          if (group) {
+            epi_bar();
+          } else {
+            __syncwarp();
+          }
+          const CUtensorMap* map = group ? &tmO : &tmO32;
+          const int y0 = group ? row0 - quarter * 32 : row0;
+          if (group ? issuer : lane == 0) {
+            const uint32_t src = smem_u32(group ? gbuf + (n_grp & 1u) * 16384 : ot);
             if (p.mode)
               asm volatile(
                   "cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
-                      (uint64_t)&tmO),
-                  "r"(src), "r"(col0), "r"(row0)
+                      (uint64_t)map),
+                  "r"(src), "r"(col0), "r"(y0)
                   : "memory");
             else
               asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
-                               (uint64_t)&tmO),
-                           "r"(src), "r"(col0), "r"(row0)
+                               (uint64_t)map),
+                           "r"(src), "r"(col0), "r"(y0)
                            : "memory");
             asm volatile("cp.async.bulk.commit_group;" ::: "memory");
           }
-          ++n_out_tiles;
+          if (group)
+            ++n_grp;
+          else
+            ++n_out_tiles;
         }
       }
       for (int c = 0; c < ((p.relu2 || p.lse || p.tma_out || p.rope) ? 0 : ncols / 32); ++c) {
@@ -556,7 +604,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       if (lane == 0) mbar_arrive(bar_tempty + 8 * b);
     }
     // the TMA writes complete before the kernel does
-    if (lane == 0 && n_out_tiles) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+    if (lane == 0 && (n_out_tiles || (issuer && n_grp))) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
   }
   if (!ok && p.err) atomicOr(p.err, ERR_TIMEOUT);
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -724,12 +772,15 @@ bool gemm_plan_output(GemmPlan* plan, float* out, int ldo) {
   if (!fn || !out || ldo < plan->N || ((uintptr_t)out & 15) || ((size_t)ldo * 4) % 16) return false;
   cuuint64_t dims[2] = {(cuuint64_t)plan->N, (cuuint64_t)plan->M};
   cuuint64_t strides[1] = {(cuuint64_t)ldo * 4};
-  cuuint32_t box[2] = {32, 32};
   cuuint32_t estr[2] = {1, 1};
-  if (fn(&plan->o, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, out, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-         CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) !=
-      CUDA_SUCCESS)
-    return false;
+  // 32 columns x 128 rows (a whole tile's block) and x 32 rows (one warp's)
+  for (int v = 0; v < 2; ++v) {
+    cuuint32_t box[2] = {32, v ? 32u : 128u};
+    if (fn(v ? &plan->o32 : &plan->o, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, out, dims, strides, box, estr,
+           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return false;
+  }
   plan->o_ptr = out;
   plan->o_ld = ldo;
   return true;
@@ -786,7 +837,7 @@ cudaError_t launch_bn(const GemmPlan& plan, const GemmArgs& args, cudaStream_t s
     }
   }
   return launch_dependent(k_bitlinear_gemm<BN, F8>, grid, dim3(GEMM_THREADS), smem, stream, plan.a, plan.a2, plan.b,
-                          *bn_map, plan.b_up, plan.o, plan.q, plan.k, a);
+                          *bn_map, plan.b_up, plan.o, plan.o32, plan.q, plan.k, a);
 }
 
 }  // namespace

@@ -72,7 +72,8 @@ struct GemmPlan {
   int gu_split;
   int M, N, K, bn;  // bn: output tile width (columns of B per tile)
   int n_fast;       // tile order: n fastest (A streamed once, B kept in L2)
-  CUtensorMap o;    // fp32 output [M, N] (row stride o_ld): TMA store / reduce-add
+  CUtensorMap o;    // fp32 output [M, N] (row stride o_ld): TMA store / reduce-add, 32 x 128 boxes
+  CUtensorMap o32;  // the same output, 32 x 32 boxes (one warp's rows)
   float* o_ptr;     // the output the map was made for (null: none)
   int o_ld;
   CUtensorMap q, k;  // fused RoPE outputs (gemm_plan_rope)
