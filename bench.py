@@ -321,7 +321,13 @@ def run_mine(args):
     with Clocks(local) as clk:
         barrier(dist)
         torch.cuda.synchronize()
-        ctx.termezo_profile(1)
+        # CUDA events around every 13th GEMM / attention / sparse launch (13 is
+        # prime to the 4 GEMMs of a layer and the 5 sparse passes of a step,
+        # so each kind is sampled in turn): the roofline's average launch
+        # time, measured live in this timed region at a thirteenth of the
+        # events' overhead (an event between two launches also ends their
+        # programmatic overlap)
+        ctx.termezo_profile(13)
         e0.record(stream)
         outs = []
         for i in range(args.warmup, nb):
@@ -354,6 +360,12 @@ def run_mine(args):
     tokens = world * args.steps * B * S
     value = job_value(world, args.steps, B * S, ms_max)
     gemm_s = prof["gemm_ms"] / 1e3
+
+    def share(kind):
+        # mean timed launch x every launch of the kind, over the timed region
+        n = prof[f"{kind}_launches"]
+        return prof[f"{kind}_ms"] / n * prof[f"{kind}_seen"] / ms if n else None
+
     achieved = prof["gemm_flops"] / gemm_s / 1e12 if gemm_s > 0 else None
     # The GEMM issues two e4m3 MMAs (the hi and lo halves of every int8 code)
     # per int8 x ternary product, at twice the bf16 rate (the nominal e4m3 :
@@ -386,12 +398,13 @@ def run_mine(args):
                                      "int8 x ternary product"),
                      "executed_e4m3": {"achieved": 2.0 * achieved if achieved else None, "peak": e4m3_peak,
                                        "unit": "TFLOP/s"},
-                     "launches": prof["gemm_launches"], "avg_launch_ms": prof["gemm_ms"] / max(1, prof["gemm_launches"]),
-                     "share_of_step": prof["gemm_ms"] / ms},
-        "kernels": {"attention_tflops": attn_tf, "attention_share": prof["attn_ms"] / ms,
+                     "launches": prof["gemm_seen"], "timed_launches": prof["gemm_launches"],
+                     "avg_launch_ms": prof["gemm_ms"] / max(1, prof["gemm_launches"]),
+                     "share_of_step": share("gemm")},
+        "kernels": {"attention_tflops": attn_tf, "attention_share": share("attn"),
                     "sparse_passes_gbs": sparse_gbs,
                     "sparse_passes_frac_hbm": sparse_gbs / float(pk.get("hbm_gbs", 6800.0)) if sparse_gbs else None,
-                    "sparse_share": prof["sparse_ms"] / ms,
+                    "sparse_share": share("sparse"),
                     "mask_build_ms": build_ms, "mask_build_gbs": build_bytes / (build_ms / 1e3) / 1e9},
         "e2e": {"value": tokens / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "memory": memory_report(cfg, density, torch.cuda.max_memory_allocated(dev), args.weight_cache),

@@ -255,10 +255,13 @@ int termezo_normal(uint64_t seed, const uint32_t* d_idx, uint64_t n, float* d_z,
 #define TERMEZO_NOALLOC_MAX_ELEMS (1ull << 28)
 int termezo_absmean_noalloc(const float* d_w, uint64_t n, float* d_out, void* stream);
 
-/* Kernel timing of a context.  enable = 1 resets the totals and starts
- * recording CUDA events (on the context's stream) around every BitLinear
- * GEMM, attention and sparse-pass launch; enable = 0 stops recording;
- * enable = -1 leaves the state unchanged.  When out is non-NULL the stream
+/* Kernel timing of a context.  enable = n >= 1 resets the totals and starts
+ * recording CUDA events (on the context's stream) around every n-th launch of
+ * each kind: BitLinear GEMM, attention, sparse pass (n = 1: all of them; a
+ * prime n such as 13 samples the four GEMM shapes of a layer and the five
+ * sparse passes of a step in turn, and leaves most launches free of the
+ * events, which also cut the programmatic overlap of the launches around
+ * them); enable = 0 stops recording; enable = -1 leaves the state unchanged.  When out is non-NULL the stream
  * is synchronised and the totals since the last reset are written.
  * Algorithmic work: GEMM 2*M*N*K flops; attention 4*B*H*hd*S(S+1)/2 flops
  * (QK^T and PV over the causal half); sparse passes 8 B per active weight
@@ -272,6 +275,7 @@ typedef struct {
   double attn_ms, attn_flops;
   uint64_t sparse_launches; /* timed sparse passes (each 1-3 kernels) */
   double sparse_ms, sparse_bytes;
+  uint64_t gemm_seen, attn_seen, sparse_seen; /* launches of each kind while recording (timed or not) */
 } termezo_profile_out;
 
 int termezo_profile(termezo_ctx* ctx, int enable, termezo_profile_out* out);

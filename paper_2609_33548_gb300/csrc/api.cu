@@ -162,6 +162,8 @@ struct termezo_ctx {
     double work;
   };
   bool prof_on = false;
+  int prof_stride = 1;
+  uint64_t prof_seq[3] = {0, 0, 0};
   std::vector<ProfRec> prof;
   std::vector<cudaEvent_t> ev_pool;
   // weight expansion overlapped with the previous GEMM: a side stream and two
@@ -355,7 +357,10 @@ struct ProfScope {
   double work;
   cudaEvent_t a = nullptr;
   ProfScope(termezo_ctx* ctx, int category, double w) : c(ctx), cat(category), work(w) {
-    if (c->prof_on && (a = ev_get(c))) cudaEventRecord(a, c->stream);
+    // every prof_stride-th launch of each category (a stride prime to the
+    // four GEMMs of a layer and the five sparse passes of a step samples
+    // every kind in turn)
+    if (c->prof_on && c->prof_seq[category]++ % c->prof_stride == 0 && (a = ev_get(c))) cudaEventRecord(a, c->stream);
   }
   ~ProfScope() {
     if (!a) return;
@@ -1036,12 +1041,14 @@ int termezo_normal(uint64_t seed, const uint32_t* d_idx, uint64_t n, float* d_z,
 }
 
 int termezo_profile(termezo_ctx* c, int enable, termezo_profile_out* out) {
-  if (!c || enable < -1 || enable > 1) return TERMEZO_EINVAL;
-  if (enable == 1) {
+  if (!c || enable < -1 || enable > 1000) return TERMEZO_EINVAL;
+  if (enable >= 1) {
     int rc = sync_status(c);
     if (rc) return rc;
     c->prof.clear();
     c->ev_used = 0;
+    c->prof_stride = enable;
+    c->prof_seq[0] = c->prof_seq[1] = c->prof_seq[2] = 0;
     c->launch_base = tmz::kernel_launches();
     cudaMemsetAsync(c->ma.counters + 3, 0, sizeof(unsigned long long), c->stream);
     c->prof_on = true;
@@ -1070,9 +1077,14 @@ int termezo_profile(termezo_ctx* c, int enable, termezo_profile_out* out) {
         out->sparse_bytes += r.work;
       }
     }
+    out->gemm_seen = c->prof_seq[0];
+    out->attn_seen = c->prof_seq[1];
+    out->sparse_seen = c->prof_seq[2];
+    // packed words rewritten by all passes, in the proportion of the timed ones
     unsigned long long words = 0;
     cudaMemcpy(&words, c->ma.counters + 3, sizeof(words), cudaMemcpyDeviceToHost);
-    out->sparse_bytes += 8.0 * (double)words;
+    if (out->sparse_seen)
+      out->sparse_bytes += 8.0 * (double)words * (double)out->sparse_launches / (double)out->sparse_seen;
   }
   return TERMEZO_OK;
 }

@@ -56,7 +56,8 @@ class ProfileOut(ctypes.Structure):
                 ("gemm_ms", ctypes.c_double), ("gemm_flops", ctypes.c_double),
                 ("attn_launches", ctypes.c_uint64), ("attn_ms", ctypes.c_double),
                 ("attn_flops", ctypes.c_double), ("sparse_launches", ctypes.c_uint64),
-                ("sparse_ms", ctypes.c_double), ("sparse_bytes", ctypes.c_double)]
+                ("sparse_ms", ctypes.c_double), ("sparse_bytes", ctypes.c_double),
+                ("gemm_seen", ctypes.c_uint64), ("attn_seen", ctypes.c_uint64), ("sparse_seen", ctypes.c_uint64)]
 
     def as_dict(self):
         return {n: getattr(self, n) for n, _ in self._fields_}
