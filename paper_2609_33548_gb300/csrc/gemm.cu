@@ -296,11 +296,11 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       }
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       const uint32_t tacc = tmem + ((uint32_t)(quarter * 32) << 16) + b * L::ACC_STRIDE;
-      bool from_parts = false;
-      // split partials, lane-contiguous: [unit][quarter][column][lane] floats,
-      // so every warp access is one 128-byte line
+      // split partials: [unit][quarter][column / 4][lane] float4 (columns 4k .. 4k+3 of the
+      // lane's row): every warp access is 512 contiguous bytes
       auto part_at = [&](int split, int col) {
-        return p.split_ws + (((size_t)(w.tail * p.split_s + split) * 4 + quarter) * BN + col) * 32 + lane;
+        return reinterpret_cast<float4*>(p.split_ws) +
+               (((size_t)(w.tail * p.split_s + split) * 4 + quarter) * (BN / 4) + col / 4) * 32 + lane;
       };
       if (w.tail >= 0) {
         // a split of a tail tile: its partial accumulator goes to the
@@ -309,9 +309,11 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         for (int c = 0; c < BN / 32; ++c) {
           uint32_t r[32];
           tmem_ld32(tacc + (uint32_t)(c * 32), r);
-          float* dst = part_at(w.split, 32 * c);
+          float4* dst = part_at(w.split, 32 * c);
 #pragma unroll
-          for (int q = 0; q < 32; ++q) dst[32 * q] = __uint_as_float(r[q]);
+          for (int q4 = 0; q4 < 8; ++q4)
+            dst[32 * q4] = make_float4(__uint_as_float(r[4 * q4]), __uint_as_float(r[4 * q4 + 1]),
+                                       __uint_as_float(r[4 * q4 + 2]), __uint_as_float(r[4 * q4 + 3]));
         }
         __threadfence();
         unsigned prev = 0;
@@ -325,21 +327,46 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         }
         __threadfence();
         if (lane == 0) p.split_cnt[w.tail * 4 + quarter] = 0;  // ready for the next launch
-        from_parts = true;
-      }
-      // 32 accumulator columns col .. col+31 of this thread's row, plus (last
-      // split of a tail tile) the other splits' partials: integers below 2^24,
-      // so the fp32 sum is exact
-      auto load_acc = [&](int col, uint32_t(&r)[32]) {
-        tmem_ld32(tacc + (uint32_t)col, r);
-        if (!from_parts) return;
-        for (int sp = 0; sp < p.split_s; ++sp) {
-          if (sp == w.split) continue;
-          const float* src = part_at(sp, col);
+        // the other splits' partials added into this split's accumulator,
+        // 16 columns at a time with all of their loads issued before the
+        // first add (one L2 round trip each); integers below 2^24, so the
+        // fp32 sum is exact in any order
+        for (int c = 0; c < BN / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld32(tacc + (uint32_t)(c * 32), r);
 #pragma unroll
-          for (int q = 0; q < 32; ++q) r[q] = __float_as_uint(__fadd_rn(__uint_as_float(r[q]), __ldcg(src + 32 * q)));
+          for (int h = 0; h < 2; ++h) {
+            float4 pv[3][4];
+#pragma unroll
+            for (int t = 0; t < 3; ++t) {
+              const int sp = t + (t >= w.split ? 1 : 0);  // the t-th split other than this one
+              if (sp < p.split_s) {
+                const float4* src = part_at(sp, 32 * c + 16 * h);
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) pv[t][q4] = __ldcg(src + 32 * q4);
+              }
+            }
+#pragma unroll
+            for (int t = 0; t < 3; ++t) {
+              const int sp = t + (t >= w.split ? 1 : 0);
+              if (sp < p.split_s) {
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) {
+                  uint32_t* rr = r + 16 * h + 4 * q4;
+                  rr[0] = __float_as_uint(__fadd_rn(__uint_as_float(rr[0]), pv[t][q4].x));
+                  rr[1] = __float_as_uint(__fadd_rn(__uint_as_float(rr[1]), pv[t][q4].y));
+                  rr[2] = __float_as_uint(__fadd_rn(__uint_as_float(rr[2]), pv[t][q4].z));
+                  rr[3] = __float_as_uint(__fadd_rn(__uint_as_float(rr[3]), pv[t][q4].w));
+                }
+              }
+            }
+          }
+          tmem_st32(tacc + (uint32_t)(c * 32), r);
         }
-      };
+        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+      }
+      // 32 accumulator columns col .. col+31 of this thread's row
+      auto load_acc = [&](int col, uint32_t(&r)[32]) { tmem_ld32(tacc + (uint32_t)col, r); };
       if (p.lse) {
         // lane = row: running max and sum of exp over this tile's columns
         const int row = row0 + lane;
