@@ -1,22 +1,26 @@
 // BitLinear GEMM on the 5th-generation tensor cores (sm_103a).
 //
 // acc[m, n] = sum_k q[m, k] * c[n, k] with q the int8 activation codes and c
-// the ternary codes, both held as bf16 (every int8 value and every ternary
-// value is exact in bf16, every product is exact, and every partial sum is
-// an integer of magnitude <= 128 * K < 2^24, so the fp32 accumulator holds
-// the int32 accumulator exactly).  The int8 MMA kind does not exist on
-// sm_103a (ptxas: "Feature '.kind::i8' not supported on .target
-// 'sm_103a'"), so this exact-integer bf16 formulation is the tensor-core
-// path.
+// the ternary codes.  The int8 MMA kind does not exist on sm_103a (ptxas:
+// "Feature '.kind::i8' not supported on .target 'sm_103a'"), so the codes
+// travel as e4m3: each q as the pair hi = 16 floor(q/16), lo = q - hi (both
+// exact in e4m3), each ternary code as itself.  Two kind::f8f6f4 MMAs per
+// k-step, A_hi B and A_lo B, accumulate into one fp32 accumulator; every
+// product is an integer and every partial sum an integer of magnitude
+// <= 128 * K < 2^24, so the accumulator holds the int32 dot product exactly.
+// The same kernel with bf16 operands (kind::f16, one MMA per k-step) serves
+// the LM head, whose operands are not integers.
 //
 // Structure: a persistent grid (one CTA per SM) walks 128 x BN output tiles
-// (BN 256, 192, 160 or 128, picked per shape to fill the last wave);
-// warp 0 issues TMA loads of 128 x 64 (A) and BN x 64 (B) bf16 tiles with
-// 128-byte swizzle into a STAGES-deep ring; one thread of warp 1 issues
-// tcgen05.mma (M = 128, N = BN, K = 16) into one of two fp32 accumulators in
-// tensor memory; warps 2-5 read the other accumulator back with tcgen05.ld,
-// transpose it through shared memory and store coalesced rows of
-// y = acc * (a/127)[m] * s_w[n] (or add them into the residual stream).
+// (BN 256, 192, 160 or 128, picked per shape to fill the last wave; the last
+// wave's tiles split along N or K); warp 0 issues TMA loads with 128-byte
+// swizzle into a ring whose stages hold 128 bytes of K per row (A hi, A lo and
+// B for 128 K elements, or A and B for 64 bf16); one thread of warp 1 issues
+// tcgen05.mma (M = 128, N = BN) into one of two fp32 accumulators in tensor
+// memory; warps 2-5 read the other accumulator back with tcgen05.ld and write
+// y = acc * (a/127)[m] * s_w[n] (stored, added into the residual stream,
+// fused with RoPE or with the squared-ReLU gating, or reduced to the LM
+// head's log-sum-exp partials).
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
