@@ -53,7 +53,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # profiles/step_2b_launch_list.md.  It describes the kernel source with this
 # SHA-1 only; any other source, or another workload, reports null.
 GEMM_TRAFFIC = {"workload": "2b", "source": "paper_2609_33548_gb300/csrc/gemm.cu",
-                "sha1": "4168bf1e7be8d9281a4ba57c22e9f4d89a686200", "bytes_per_launch": 206.5e6}
+                "sha1": "4c962ad660ddb05afece1b02f6bceecda002c227", "bytes_per_launch": 206.5e6}
 
 
 def gemm_traffic(workload):
