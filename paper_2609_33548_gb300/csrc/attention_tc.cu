@@ -4,9 +4,9 @@
 // Same arithmetic as the mma.sync kernel: Q, K, V bf16; s = fl(acc * scale);
 // pass 1 finds the exact row maximum m over the causal keys; pass 2 forms
 // P = bf16(exp(s - m)) (exp on the special-function unit), l = sum P (fp32)
-// and O = sum P V (fp32) / l.  Since
-// scale > 0 and rounding is monotone, max fl(acc * scale) = fl(max acc *
-// scale), so pass 1 reduces the raw accumulators.
+// and O = sum P V (fp32) / l.  Since scale > 0 and rounding is monotone,
+// max fl(acc * scale) = fl(max acc * scale), so pass 1 reduces the raw
+// accumulators.
 //
 // Persistent CTAs (one per SM, all 512 TMEM columns) walk a list of work
 // items; an item is two 128-query tiles A and B that read the same KV head
@@ -19,9 +19,10 @@
 // from shared memory.  Warps 4-7 own tile A, warps 8-11 tile B (thread = query
 // row): they read S_t with tcgen05.ld, release the buffer at once (so S_t of
 // the next key block is computed while they work), reduce the row maximum
-// (pass 1) or form bf16 P rows in the swizzled K-major layout (pass 2), and at
-// the end of an item divide O_t by l and store it.  While one tile's warps
-// run their softmax the tensor core works on the other tile.
+// (pass 1) or form bf16 P rows in the swizzled K-major layout (pass 2), and
+// hand l to warps 12-15, which divide O_t by l and store it while the softmax
+// warps go on to the next item.  While one tile's warps run their softmax the
+// tensor core works on the other tile.
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
 
