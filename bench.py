@@ -48,6 +48,9 @@ WORKLOADS = {
     "tiny": (synth.TINY, 0.01),
 }
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+# dense passes over the latents that termezo_build_mask's kernels make
+# (absmean, three radix-histogram passes, count, compaction)
+MASK_BUILD_DENSE_PASSES = 6
 # DRAM bytes (read + write) per k_bitlinear_gemm launch, the mean over the 240
 # GEMM launches of one 2B-shaped step, from the one-pass ncu launch list in
 # profiles/step_2b_launch_list.md.  It describes the kernel source with this
@@ -260,7 +263,8 @@ def run_reference(args):
               f"step as layers x (requant + batch x forward)")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": est * 1e3, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "dtype_note": "oracle forward in float32 (the kernels' decision precision), losses and g in float64",
             "config": {"workload": f"{cfg.name} density {density}", "global_batch": cfg.batch,
                        "seq_len": cfg.seq, "parallelism": "cpu"},
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores(), "kind": "oracle",
@@ -307,7 +311,11 @@ def run_mine(args):
     torch.cuda.synchronize()
     build_ms = e0.elapsed_time(e1)
     d = cfg.d_lat
-    build_bytes = 6 * 4 * d + d / 4 + 8 * k0          # 6 reads of w_0, packed codes and S_0 written
+    # algorithmic bytes of the mask build (three reads of the dense latents:
+    # the absmean, the distance histogram and the selection; the packed codes
+    # and S_0 written) and the bytes of the passes the kernels make
+    build_bytes = 3 * 4 * d + d / 4 + 8 * k0
+    build_bytes_kernels = MASK_BUILD_DENSE_PASSES * 4 * d + d / 4 + 8 * k0
     # the dense latents are read only by the mask build: released here, so the
     # footprint measured over the timed steps is the method's (Sec. 5)
     del w
@@ -338,6 +346,14 @@ def run_mine(args):
         barrier(dist)
     prof = ctx.termezo_profile(0, read=True)
     ms = e0.elapsed_time(e1)
+    # the sparse passes one by one: events around every sparse launch of a few
+    # more steps (outside the timed region; the GEMM stride keeps the forward
+    # nearly free of events)
+    ctx.termezo_profile(1)
+    for i in range(nb, nb + 3):
+        tok, tgt = batches[i % nb]
+        do_step(i, tok, tgt)
+    passes = ctx.termezo_profile(0, read=True)
     ms_max = max_over_ranks(dist, ms)
     clocks = clk.summary()
 
@@ -376,6 +392,15 @@ def run_mine(args):
     h2d = tok_h[0].numel() * 4 + tgt_h[0].numel() * 4
     d2h = 2 * 8 + 8 + 4 * 8 + 4 + 2 * B * 8
     sparse_gbs = prof["sparse_bytes"] / (prof["sparse_ms"] / 1e3) / 1e9 if prof["sparse_ms"] > 0 else None
+    hbm = float(pk.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+    pass_table = {}
+    for j, kind in enumerate(tz.PASS_KINDS):
+        n = passes["pass_launches"][j]
+        if n:
+            t_ms = passes["pass_ms"][j] / n
+            gbs = passes["pass_bytes"][j] / n / (t_ms / 1e3) / 1e9
+            pass_table[kind] = {"ms": t_ms, "algorithmic_mb": passes["pass_bytes"][j] / n / 1e6, "gbs": gbs,
+                                "frac_hbm": gbs / hbm, "launches": n}
     attn_tf = prof["attn_flops"] / (prof["attn_ms"] / 1e3) / 1e12 if prof["attn_ms"] > 0 else None
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
@@ -403,14 +428,21 @@ def run_mine(args):
                      "share_of_step": share("gemm")},
         "kernels": {"attention_tflops": attn_tf, "attention_share": share("attn"),
                     "sparse_passes_gbs": sparse_gbs,
-                    "sparse_passes_frac_hbm": sparse_gbs / float(pk.get("hbm_gbs", 6800.0)) if sparse_gbs else None,
+                    "sparse_passes_frac_hbm": sparse_gbs / hbm if sparse_gbs else None,
                     "sparse_share": share("sparse"),
-                    "mask_build_ms": build_ms, "mask_build_gbs": build_bytes / (build_ms / 1e3) / 1e9},
+                    "sparse_passes": pass_table,
+                    "mask_build_ms": build_ms, "mask_build_gbs": build_bytes / (build_ms / 1e3) / 1e9,
+                    "mask_build_frac_hbm": build_bytes / (build_ms / 1e3) / 1e9 / hbm,
+                    "mask_build_kernel_gbs": build_bytes_kernels / (build_ms / 1e3) / 1e9,
+                    "bytes_note": ("algorithmic bytes: sparse passes per include/termezo.h termezo_profile_out "
+                                   "(index + latent per active weight, 64 B per rewritten 32-byte sector of the "
+                                   "packed store, 4 B per updated latent); mask build 3 dense reads + codes + S_0")},
         "e2e": {"value": tokens / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "memory": memory_report(cfg, density, torch.cuda.max_memory_allocated(dev), args.weight_cache),
         "gpu_launches": int(prof["launches"]),
         "clocks": clocks,
-        "last_step": {k: outs[-1][k] for k in ("loss_plus", "loss_minus", "g", "n_flipped", "n_jumps")},
+        "last_step": {k: outs[-1][k] for k in ("loss_plus", "loss_minus", "g", "k_active", "n_flipped", "n_jumps",
+                                               "n_dropped", "n_near_threshold")},
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         est, t_rq, t_fw = OracleSample(cfg, density).run()

@@ -5,9 +5,11 @@
  *
  * Conventions shared by every call
  *  - Pointers named d_* are device pointers owned by the caller; h_* are
- *    host pointers owned by the caller.  The library never allocates device
- *    memory: every internal buffer is carved from the one workspace the
- *    caller passes to termezo_create.
+ *    host pointers owned by the caller.  The library allocates no device
+ *    memory at run time: every buffer of a context is carved from the one
+ *    workspace the caller passes to termezo_create, and the only device
+ *    memory of its own is the fixed 4 MiB array that
+ *    termezo_absmean_noalloc uses.
  *  - All device work is ordered on the stream given to termezo_create (a
  *    cudaStream_t passed as void*; NULL = legacy default stream).  Calls
  *    that return host values synchronise that stream before returning.
@@ -71,6 +73,10 @@ typedef struct {
   uint64_t n_flipped; /* active codes that differ between the two passes */
   uint64_t n_jumps;   /* active codes that moved -1 <-> +1 between them  */
   uint64_t n_dropped; /* weights frozen by this step's shrink           */
+  uint64_t n_near_threshold; /* active latents within 1e-5 s_w of +-tau (Eq. 2
+                        thresholds) in the + pass plus those in the - pass:
+                        the codes excluded from bit-exact comparison, the
+                        distance | |w| - tau | taken in float64          */
 } termezo_step_out;
 
 /* Bytes of device workspace a context needs for cfg and mask density
@@ -150,6 +156,52 @@ int termezo_build_mask_rule(termezo_ctx* ctx, double density, int32_t rule, uint
  * per_seq[batch] (nullable) the loss of each sequence.  Synchronises. */
 int termezo_forward_loss(termezo_ctx* ctx, const int32_t* d_tokens, const int32_t* d_targets,
                          double* loss, double* per_seq);
+
+/* Intermediates of one decoder layer of the forward (Sec. 3 BitNet block;
+ * Eqs. 6-7 evaluate it at the perturbed codes), for layer-by-layer parity
+ * checks.  Every pointer is a caller-owned device buffer that the call fills,
+ * or NULL to skip it; T = batch * seq rows, D = hidden, Hq = heads * hd,
+ * F = ffn.  Activation codes are the int8 values q of the per-token absmax
+ * quantiser that the BitLinear GEMM consumes, with deq = a / 127 per row.
+ *   x_in       fp32 [T, D]   residual stream entering the layer
+ *   codes_attn int8 [T, D], deq_attn fp32 [T]   codes of RMSNorm(x_in)
+ *   q          bf16 [B, H, S, hd]   RoPE-rotated queries (raw bits)
+ *   k          bf16 [B, KV, S, hd]  RoPE-rotated keys
+ *   vt         bf16 [B, KV, hd, S]  values, transposed
+ *   attn       fp32 [T, Hq]  causal attention output
+ *   codes_o    int8 [T, Hq], deq_o fp32 [T]     codes of attn
+ *   x_mid      fp32 [T, D]   x_in + o(attn)
+ *   codes_mlp  int8 [T, D], deq_mlp fp32 [T]    codes of RMSNorm(x_mid)
+ *   hid        fp32 [T, F]   relu(gate)^2 * up
+ *   codes_down int8 [T, F], deq_down fp32 [T]   codes of hid
+ *   x_out      fp32 [T, D]   x_mid + down(hid)
+ * For layer == layers only x_in is filled: the residual stream after the last
+ * layer, which the final RMSNorm and the LM head read. */
+typedef struct {
+  float* x_in;
+  int8_t* codes_attn;
+  float* deq_attn;
+  uint16_t *q, *k, *vt;
+  float* attn;
+  int8_t* codes_o;
+  float* deq_o;
+  float* x_mid;
+  int8_t* codes_mlp;
+  float* deq_mlp;
+  float* hid;
+  int8_t* codes_down;
+  float* deq_down;
+  float* x_out;
+} termezo_layer_trace;
+
+/* The BitNet forward and minibatch loss at the codes now in the packed store
+ * (those of the last termezo_build_mask, termezo_requantize or step, with
+ * their weight scales; nothing is requantised), copying the intermediates of
+ * `layer` (0 <= layer <= layers) into `trace`.  A test and diagnostic call:
+ * the copies cost a device-to-device copy per buffer.  loss, per_seq as
+ * termezo_forward_loss (nullable).  Synchronises. */
+int termezo_forward_trace(termezo_ctx* ctx, const int32_t* d_tokens, const int32_t* d_targets, int32_t layer,
+                          const termezo_layer_trace* trace, double* loss, double* per_seq);
 
 /* One TerMeZO iteration (Algorithm 1 loop body, K = 1):
  *   t >= 1: tau_t recomputed, S_t = {i in S_{t-1}: d_i(w_t) <= xi_0} (Eq. 5);
@@ -250,7 +302,10 @@ int termezo_normal(uint64_t seed, const uint32_t* d_idx, uint64_t n, float* d_z,
  * until the process exits.  n > TERMEZO_NOALLOC_MAX_ELEMS returns
  * TERMEZO_EINVAL (with a message on stderr).  The first call on a device
  * looks up that device's address of the array; make it before any stream
- * capture.  Calls share the array: calls that overlap on the GPU race.
+ * capture.  The address is kept for the life of the process, so a
+ * cudaDeviceReset of that device voids it: do not reset a device that is
+ * still used with this call.  Calls share the array: calls that overlap on
+ * the GPU race.
  * Each call overwrites every partial sum it reads.  Allocates nothing. */
 #define TERMEZO_NOALLOC_MAX_ELEMS (1ull << 28)
 int termezo_absmean_noalloc(const float* d_w, uint64_t n, float* d_out, void* stream);
@@ -264,18 +319,30 @@ int termezo_absmean_noalloc(const float* d_w, uint64_t n, float* d_out, void* st
  * them); enable = 0 stops recording; enable = -1 leaves the state unchanged.  When out is non-NULL the stream
  * is synchronised and the totals since the last reset are written.
  * Algorithmic work: GEMM 2*M*N*K flops; attention 4*B*H*hd*S(S+1)/2 flops
- * (QK^T and PV over the causal half); sparse passes 8 B per active weight
- * (index + latent) read per pass, plus 4 B written per updated latent and
- * 8 B per packed word rewritten. */
+ * (QK^T and PV over the causal half); sparse passes, by kind (pass_*):
+ *   0 perturbation sums (k_sparse_pm_sum + the tau+- reductions): 8 B per
+ *     active weight (index + latent) read;
+ *   1 requantisation (one sign): 8 B per active weight read, plus every
+ *     32-byte sector of the packed store that holds an active weight, read
+ *     and written (64 B per sector);
+ *   2 restore + update: 8 B per active weight read, 4 B written;
+ *   3 shrink (Eq. 5): 8 B per active weight read twice, 8 B per kept weight
+ *     written (counted as 24 B per active weight);
+ *   4 theta perturbation / update (termezo_step_joint): each parameter read
+ *     and written in its stored precision.
+ * sparse_* are the totals over the kinds. */
+#define TERMEZO_PASS_KINDS 5
 typedef struct {
   uint64_t launches;        /* kernels launched by this thread since the reset */
   uint64_t gemm_launches;
   double gemm_ms, gemm_flops;
   uint64_t attn_launches;
   double attn_ms, attn_flops;
-  uint64_t sparse_launches; /* timed sparse passes (each 1-3 kernels) */
+  uint64_t sparse_launches; /* timed sparse passes (each 1-5 kernels) */
   double sparse_ms, sparse_bytes;
   uint64_t gemm_seen, attn_seen, sparse_seen; /* launches of each kind while recording (timed or not) */
+  uint64_t pass_launches[TERMEZO_PASS_KINDS], pass_seen[TERMEZO_PASS_KINDS];
+  double pass_ms[TERMEZO_PASS_KINDS], pass_bytes[TERMEZO_PASS_KINDS];
 } termezo_profile_out;
 
 int termezo_profile(termezo_ctx* ctx, int enable, termezo_profile_out* out);

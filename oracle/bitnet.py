@@ -80,12 +80,23 @@ def int_matmul(q: np.ndarray, codes: np.ndarray) -> np.ndarray:
     return np.rint(acc).astype(np.int64)
 
 
+def bitlinear_codes(q: np.ndarray, dq: np.ndarray, codes: np.ndarray, s_w) -> np.ndarray:
+    """y = (acc * dq) * s_w in float32 for int8 activation codes q [M, K]
+    with per-row dq = fl32(a / 127) (acc is an exact integer)."""
+    acc = int_matmul(q, codes).astype(F32)          # exact: |acc| < 2^24
+    return ((acc * np.asarray(dq, dtype=F32)[:, None]).astype(F32) * F32(s_w)).astype(F32)
+
+
 def bitlinear(x: np.ndarray, codes: np.ndarray, s_w) -> np.ndarray:
     """y = (acc * (a / 127)) * s_w in float32 (acc is an exact integer)."""
     q, a = act_quant(x)
-    acc = int_matmul(q, codes).astype(F32)          # exact: |acc| < 2^24
-    dq = (a / F32(127.0)).astype(F32)
-    return ((acc * dq[:, None]).astype(F32) * F32(s_w)).astype(F32)
+    return bitlinear_codes(q, (a / F32(127.0)).astype(F32), codes, s_w)
+
+
+def gated_hidden(g: np.ndarray, u: np.ndarray) -> np.ndarray:
+    """The squared-ReLU gated MLP hidden relu(g)^2 * u, float32."""
+    g = np.maximum(np.asarray(g, dtype=F32), F32(0.0))
+    return ((g * g).astype(F32) * np.asarray(u, dtype=F32)).astype(F32)
 
 
 def rope(x: np.ndarray, hd: int) -> np.ndarray:
@@ -152,10 +163,17 @@ def sequence_loss(cfg, codes, s_w, embed, gains, head, tokens, target) -> float:
         a = attention(rope(q, hd), rope(k, hd), v)
         x = (x + bitlinear(a, co, so)).astype(np.float32)
         h = rmsnorm(x, gains[2 * l + 1])
-        g = np.maximum(bitlinear(h, cg, sg), F32(0.0))
-        u = bitlinear(h, cu, su)
-        hid = ((g * g).astype(F32) * u).astype(F32)
+        hid = gated_hidden(bitlinear(h, cg, sg), bitlinear(h, cu, su))
         x = (x + bitlinear(hid, cd, sd)).astype(np.float32)
+    return head_loss(cfg, x, gains, head, target)
+
+
+def head_loss(cfg, x, gains, head, target) -> float:
+    """Loss of one sequence from the residual stream x [S, D] after the last
+    layer: final RMSNorm, the LM head on bf16(h), cross-entropy (mode 0:
+    last position over the label tokens; mode 1: every position over the
+    vocabulary, averaged)."""
+    S = x.shape[0]
     h = bf16_round(rmsnorm(x, gains[2 * cfg.layers])).astype(np.float64)
     W = np.asarray(head, dtype=np.float64)
     if cfg.loss_mode == 0:

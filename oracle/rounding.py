@@ -14,7 +14,9 @@ with every value a reduction produces (each RMSNorm mean square, each
 BitLinear output, each attention output) moved by one ulp up or down, each
 with probability 1/4, i.e. rounded the other way; the spread of an ensemble of
 such runs measures how far two correct implementations may disagree on a
-given input.  The oracle's own arithmetic is unchanged.
+given input.  The oracle's own arithmetic is unchanged.  ``within`` accepts
+a value that agrees with the oracle to the stated relative bound, or that
+deviates from it by no more than one of these alternatives does.
 """
 from __future__ import annotations
 
@@ -78,11 +80,23 @@ def g_ensemble(cfg, plus, minus, theta, eps, n: int = 6, rows=None):
 
 
 def within(value, ref, ens, rel=1e-3) -> bool:
-    """True if value agrees with ref to `rel`, or lies inside the range of
-    [ref] + ens widened by that range on both sides."""
+    """True if value agrees with ref to `rel`, or deviates from ref by no
+    more than the largest deviation of an ensemble member: |value - ref| <=
+    max_i |ens_i - ref|.  The members are the oracle itself under other valid
+    fp32 roundings, so this accepts a value exactly when the oracle's own
+    alternatives move at least as far from it (no widening beyond them)."""
+    dev = float(np.max(np.abs(np.ravel(ens) - ref))) if np.size(ens) else 0.0
+    return abs(value - ref) <= rel * abs(ref) or abs(value - ref) <= dev
+
+
+def summary(value, ref, ens) -> dict:
+    """|value - ref| next to the ensemble's largest deviation from ref and
+    its range, for the parity record."""
     allv = np.concatenate([[ref], np.ravel(ens)])
-    spread = allv.max() - allv.min()
-    return abs(value - ref) <= rel * abs(ref) or (allv.min() - spread <= value <= allv.max() + spread)
+    return dict(value=float(value), ref=float(ref), abs_err=abs(float(value) - float(ref)),
+                rel_err=abs(float(value) - float(ref)) / max(abs(float(ref)), 1e-300),
+                ens_max_dev=float(np.max(np.abs(np.ravel(ens) - ref))) if np.size(ens) else 0.0,
+                ens_min=float(allv.min()), ens_max=float(allv.max()), n_ens=int(np.size(ens)))
 
 
 def g_within_ensemble(g, g_ref, ens, rel=1e-3) -> bool:

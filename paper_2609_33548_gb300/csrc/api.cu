@@ -83,6 +83,10 @@ uint64_t keep_count(double density, uint64_t d) { return (uint64_t)std::floor(de
 
 // Bump allocator over the workspace; with base == nullptr it only measures.
 // Workspace sections, for the memory report.
+// Sparse pass kinds of termezo_profile_out::pass_* (see termezo.h).
+enum { PASS_PM = 0, PASS_REQUANT = 1, PASS_UPDATE = 2, PASS_SHRINK = 3, PASS_THETA = 4 };
+static_assert(PASS_THETA + 1 == TERMEZO_PASS_KINDS, "pass kinds");
+
 enum Section { SEC_PACKED, SEC_INDEX, SEC_LATENTS, SEC_MASK, SEC_FORWARD, SEC_WCACHE, SEC_COUNT };
 
 struct Carver {
@@ -157,13 +161,13 @@ struct termezo_ctx {
   bool pm_valid = false;
   // kernel timing (termezo_profile)
   struct ProfRec {
-    int cat;  // 0 GEMM, 1 attention, 2 sparse pass
+    int cat;  // 0 GEMM, 1 attention, 2 + PASS_* a sparse pass
     cudaEvent_t a, b;
     double work;
   };
   bool prof_on = false;
   int prof_stride = 1;
-  uint64_t prof_seq[3] = {0, 0, 0};
+  uint64_t prof_seq[2 + TERMEZO_PASS_KINDS] = {};
   std::vector<ProfRec> prof;
   std::vector<cudaEvent_t> ev_pool;
   // weight expansion overlapped with the previous GEMM: a side stream and two
@@ -178,6 +182,9 @@ struct termezo_ctx {
   cudaEvent_t ev_codes = nullptr;                // the codes of this forward are final
   size_t ev_used = 0;
   uint64_t launch_base = 0;
+  // termezo_forward_trace: the layer whose intermediates run_forward copies
+  const termezo_layer_trace* trace = nullptr;
+  int trace_layer = -1;
   ~termezo_ctx() {
     for (cudaEvent_t e : ev_pool) cudaEventDestroy(e);
     for (cudaEvent_t e : {ev_free[0], ev_free[1], ev_ready[0], ev_ready[1], ev_codes})
@@ -254,7 +261,7 @@ void carve(termezo_ctx* c, Carver& cv) {
   a.blk_b = cv.take<uint32_t>(nblk);
   a.blk_c = cv.take<uint32_t>(nblk);
   a.blk_d = cv.take<uint32_t>(nblk);
-  a.counters = cv.take<unsigned long long>(4);
+  a.counters = cv.take<unsigned long long>(8);
   a.err = cv.take<unsigned>(1);
   c->d_total = cv.take<uint32_t>(1);
   const size_t T = s.T;
@@ -387,6 +394,15 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
   // weight cache the GEMMs read the cached codes and nothing is expanded.
   const bool cached = c->wbyte != nullptr;
   uint8_t* wbuf[2] = {c->wexp, c->wexp2};
+  // termezo_forward_trace copies (stream-ordered, between the kernels)
+  const termezo_layer_trace* tr = c->trace;
+  auto tr_copy = [&](void* dst, const void* src, size_t bytes) {
+    if (dst) cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToDevice, st);
+  };
+  auto tr_codes = [&](int8_t* codes, float* deq, int K) {
+    if (codes) tmz::launch_codes_i8(c->xq, T, K, codes, st);
+    tr_copy(deq, c->deq, (size_t)T * sizeof(float));
+  };
   cudaStream_t xs = c->xstream;
   auto expand = [&](int l, int g) {
     const int b = g & 1;
@@ -430,8 +446,11 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
   }
   for (int l = 0; l < s.L; ++l) {
     const int pq = proj_of(s, l, 0), po = proj_of(s, l, 3), pg = proj_of(s, l, 4), pd = proj_of(s, l, 6);
+    const termezo_layer_trace* lt = (tr && c->trace_layer == l) ? tr : nullptr;
     // attention block
+    if (lt) tr_copy(lt->x_in, c->x, (size_t)T * D * sizeof(float));
     tmz::launch_norm_quant(c->x, c->gains + (size_t)(2 * l) * D, T, D, c->xq, c->deq, st);
+    if (lt) tr_codes(lt->codes_attn, lt->deq_attn, D);
     GemmArgs a{};
     a.out = c->qkv;
     a.ldo = hq + 2 * hkv;
@@ -455,6 +474,11 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
     if (!gemm(l, 0, a, 0.0)) return TERMEZO_ECUDA;
     if (!rope)
       tmz::launch_rope_pack(c->qkv, c->cosb, c->sinb, s.B, s.S, s.H, s.KV, s.hd, c->qb, c->kb, c->vt, st);
+    if (lt) {
+      tr_copy(lt->q, c->qb, (size_t)T * hq * sizeof(uint16_t));
+      tr_copy(lt->k, c->kb, (size_t)T * hkv * sizeof(uint16_t));
+      tr_copy(lt->vt, c->vt, (size_t)T * hkv * sizeof(uint16_t));
+    }
     a.rope = 0;  // the remaining projections of the layer reuse a
     {
       ProfScope ps(c, 1, 4.0 * s.B * s.H * (double)s.hd * (0.5 * s.S * (s.S + 1.0)));
@@ -465,7 +489,9 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
         tmz::launch_attention(c->qb, c->kb, c->vt, s.B, s.S, s.H, s.KV, s.hd, c->attn, st);
       }
     }
+    if (lt) tr_copy(lt->attn, c->attn, (size_t)T * hq * sizeof(float));
     tmz::launch_norm_quant(c->attn, nullptr, T, hq, c->xq, c->deq, st);
+    if (lt) tr_codes(lt->codes_o, lt->deq_o, hq);
     a.out = c->x;
     a.ldo = D;
     a.mode = 1;
@@ -473,7 +499,9 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
     a.n1 = a.n2 = D;
     if (!gemm(l, 1, a, 0.0)) return TERMEZO_ECUDA;
     // MLP block
+    if (lt) tr_copy(lt->x_mid, c->x, (size_t)T * D * sizeof(float));
     tmz::launch_norm_quant(c->x, c->gains + (size_t)(2 * l + 1) * D, T, D, c->xq, c->deq, st);
+    if (lt) tr_codes(lt->codes_mlp, lt->deq_mlp, D);
     a.out = c->gu;  // hid = relu(gate)^2 * up, fp32 [T, F]
     a.ldo = F;
     a.mode = 0;
@@ -483,14 +511,18 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
     a.n_out = F;
     if (!gemm(l, 2, a, 2.0 * T * (2.0 * F) * D)) return TERMEZO_ECUDA;
     a.relu2 = 0;
+    if (lt) tr_copy(lt->hid, c->gu, (size_t)T * F * sizeof(float));
     tmz::launch_norm_quant(c->gu, nullptr, T, F, c->xq, c->deq, st);
+    if (lt) tr_codes(lt->codes_down, lt->deq_down, F);
     a.out = c->x;
     a.ldo = D;
     a.mode = 1;
     a.sw = sw + pd;
     a.n1 = a.n2 = D;
     if (!gemm(l, 3, a, 0.0)) return TERMEZO_ECUDA;
+    if (lt) tr_copy(lt->x_out, c->x, (size_t)T * D * sizeof(float));
   }
+  if (tr && c->trace_layer == s.L) tr_copy(tr->x_in, c->x, (size_t)T * D * sizeof(float));
   if (s.mode == 0) {
     tmz::launch_head_ce_last(c->x, c->gains + (size_t)(2 * s.L) * D, c->head, targets, s.B, s.S, D, s.V, s.C,
                              c->per_seq + (size_t)slot * s.B, c->loss + slot, st);
@@ -523,7 +555,7 @@ void ensure_pm(termezo_ctx* c, uint64_t seed, float eps) {
 }
 
 int do_shrink(termezo_ctx* c) {
-  ProfScope ps(c, 2, 3.0 * 8.0 * (double)c->k_active);
+  ProfScope ps(c, 2 + PASS_SHRINK, 3.0 * 8.0 * (double)c->k_active);
   tmz::sparse_shrink(c->ma, c->cur, c->d_total, c->stream);
   c->cur ^= 1;
   c->pm_valid = false;
@@ -607,7 +639,7 @@ int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspa
   }
   cudaMemsetAsync(c->ma.err, 0, sizeof(unsigned), st);
   cudaMemsetAsync(c->split_cnt, 0, (size_t)c->split_cap * 4 * sizeof(unsigned), st);
-  cudaMemsetAsync(c->ma.counters, 0, 4 * sizeof(unsigned long long), st);
+  cudaMemsetAsync(c->ma.counters, 0, 8 * sizeof(unsigned long long), st);
   for (float* f : {c->ma.gamma_cur, c->ma.tau_cur, c->ma.sw_cur, c->ma.gamma_plus, c->ma.tau_plus, c->ma.sw_plus,
                    c->ma.gamma_minus, c->ma.tau_minus, c->ma.sw_minus})
     cudaMemsetAsync(f, 0, (s.P + 2) * sizeof(float), st);
@@ -785,6 +817,27 @@ int termezo_forward_loss(termezo_ctx* c, const int32_t* d_tokens, const int32_t*
   return TERMEZO_OK;
 }
 
+int termezo_forward_trace(termezo_ctx* c, const int32_t* d_tokens, const int32_t* d_targets, int32_t layer,
+                          const termezo_layer_trace* trace, double* loss, double* per_seq) {
+  if (!c || !d_tokens || !d_targets || !trace) return TERMEZO_EINVAL;
+  if (c->sh.op || !c->built) return TERMEZO_ESTATE;
+  if (layer < 0 || layer > c->sh.L) return TERMEZO_EINVAL;
+  c->trace = trace;
+  c->trace_layer = layer;
+  int rc = run_forward(c, d_tokens, d_targets, c->code_sw, 0);
+  c->trace = nullptr;
+  c->trace_layer = -1;
+  if (rc) return rc;
+  double l = 0;
+  cudaMemcpyAsync(&l, c->loss, sizeof(double), cudaMemcpyDeviceToHost, c->stream);
+  if (per_seq)
+    cudaMemcpyAsync(per_seq, c->per_seq, c->sh.B * sizeof(double), cudaMemcpyDeviceToHost, c->stream);
+  rc = sync_status(c);
+  if (rc) return rc;
+  if (loss) *loss = l;
+  return TERMEZO_OK;
+}
+
 namespace {
 
 // Algorithm 1's loop body with K directions: shrink (t >= 1); for each
@@ -817,6 +870,7 @@ int step_impl(termezo_ctx* c, const uint64_t* seeds, int K, float eps, float lr,
   const int warn = (density != c->density) ? TERMEZO_WMASKFIXED : TERMEZO_OK;
   cudaStream_t st = c->stream;
   cudaMemsetAsync(c->ma.counters, 0, 3 * sizeof(unsigned long long), st);
+  cudaMemsetAsync(c->ma.counters + 4, 0, sizeof(unsigned long long), st);
   int rc;
   if (c->updated) {
     rc = do_shrink(c);
@@ -830,25 +884,25 @@ int step_impl(termezo_ctx* c, const uint64_t* seeds, int K, float eps, float lr,
     const uint64_t seed = seeds[k];
     dirs.seed[k] = seed;
     {
-      ProfScope ps(c, 2, k8);
+      ProfScope ps(c, 2 + PASS_PM, k8);
       ensure_pm(c, seed, eps);
     }
     {
-      ProfScope ps(c, 2, k8);
+      ProfScope ps(c, 2 + PASS_REQUANT, k8);
       tmz::sparse_requant(c->ma, c->cur, seed, eps, +1, st);
     }
     if (theta) {
-      ProfScope ps(c, 2, theta8);
+      ProfScope ps(c, 2 + PASS_THETA, theta8);
       tmz::theta_pm(th, seed, eps, 0, st);
     }
     rc = run_forward(c, d_tokens, d_targets, c->ma.sw_plus, 0);
     if (rc) return rc;
     {
-      ProfScope ps(c, 2, k8);
+      ProfScope ps(c, 2 + PASS_REQUANT, k8);
       tmz::sparse_requant(c->ma, c->cur, seed, eps, -1, st);
     }
     if (theta) {
-      ProfScope ps(c, 2, theta8);
+      ProfScope ps(c, 2 + PASS_THETA, theta8);
       tmz::theta_pm(th, seed, eps, 1, st);
     }
     rc = run_forward(c, d_tokens, d_targets, c->ma.sw_minus, 1);
@@ -857,7 +911,7 @@ int step_impl(termezo_ctx* c, const uint64_t* seeds, int K, float eps, float lr,
     tmz::launch_grad(c->loss, eps, c->g + k, st);
     if (K > 1) cudaMemcpyAsync(c->lossk + 2 * k, c->loss, 2 * sizeof(double), cudaMemcpyDeviceToDevice, st);
     if (k + 1 < K) {
-      ProfScope ps(c, 2, 1.5 * k8);
+      ProfScope ps(c, 2 + PASS_UPDATE, 1.5 * k8);
       tmz::sparse_restore(c->ma, c->cur, seed, eps, st);
       c->pm_valid = false;
       if (theta) tmz::theta_pm(th, seed, eps, 0, st);
@@ -865,23 +919,23 @@ int step_impl(termezo_ctx* c, const uint64_t* seeds, int K, float eps, float lr,
   }
   dirs.last = seeds[K - 1];
   {
-    ProfScope ps(c, 2, 1.5 * k8);
+    ProfScope ps(c, 2 + PASS_UPDATE, 1.5 * k8);
     tmz::sparse_update_dirs(c->ma, c->cur, dirs, eps, lr, c->g, st);
   }
   if (theta) {
-    ProfScope ps(c, 2, theta8);
+    ProfScope ps(c, 2 + PASS_THETA, theta8);
     tmz::theta_update(th, dirs, eps, lr, c->g, st);
   }
   c->pm_valid = false;
   struct {
     double loss[2 * tmz::KMAX];
     double g[tmz::KMAX];
-    unsigned long long cnt[4];
+    unsigned long long cnt[5];
     uint32_t k;
   } h{};
   cudaMemcpyAsync(h.loss, K > 1 ? c->lossk : c->loss, 2 * K * sizeof(double), cudaMemcpyDeviceToHost, st);
   cudaMemcpyAsync(h.g, c->g, K * sizeof(double), cudaMemcpyDeviceToHost, st);
-  cudaMemcpyAsync(h.cnt, c->ma.counters, 4 * sizeof(unsigned long long), cudaMemcpyDeviceToHost, st);
+  cudaMemcpyAsync(h.cnt, c->ma.counters, 5 * sizeof(unsigned long long), cudaMemcpyDeviceToHost, st);
   cudaMemcpyAsync(&h.k, c->ma.off[c->cur] + c->sh.P, sizeof(uint32_t), cudaMemcpyDeviceToHost, st);
   if (per_seq_plus)
     cudaMemcpyAsync(per_seq_plus, c->per_seq, c->sh.B * sizeof(double), cudaMemcpyDeviceToHost, st);
@@ -899,6 +953,7 @@ int step_impl(termezo_ctx* c, const uint64_t* seeds, int K, float eps, float lr,
   out->n_flipped = h.cnt[0];
   out->n_jumps = h.cnt[1];
   out->n_dropped = h.cnt[2];
+  out->n_near_threshold = h.cnt[4];
   if (losses)
     for (int i = 0; i < 2 * K; ++i) losses[i] = h.loss[i];
   if (gs)
@@ -1048,7 +1103,7 @@ int termezo_profile(termezo_ctx* c, int enable, termezo_profile_out* out) {
     c->prof.clear();
     c->ev_used = 0;
     c->prof_stride = enable;
-    c->prof_seq[0] = c->prof_seq[1] = c->prof_seq[2] = 0;
+    for (auto& q : c->prof_seq) q = 0;
     c->launch_base = tmz::kernel_launches();
     cudaMemsetAsync(c->ma.counters + 3, 0, sizeof(unsigned long long), c->stream);
     c->prof_on = true;
@@ -1072,19 +1127,28 @@ int termezo_profile(termezo_ctx* c, int enable, termezo_profile_out* out) {
         out->attn_ms += ms;
         out->attn_flops += r.work;
       } else {
-        out->sparse_launches++;
-        out->sparse_ms += ms;
-        out->sparse_bytes += r.work;
+        const int k = r.cat - 2;
+        out->pass_launches[k]++;
+        out->pass_ms[k] += ms;
+        out->pass_bytes[k] += r.work;
       }
     }
     out->gemm_seen = c->prof_seq[0];
     out->attn_seen = c->prof_seq[1];
-    out->sparse_seen = c->prof_seq[2];
-    // packed words rewritten by all passes, in the proportion of the timed ones
-    unsigned long long words = 0;
-    cudaMemcpy(&words, c->ma.counters + 3, sizeof(words), cudaMemcpyDeviceToHost);
-    if (out->sparse_seen)
-      out->sparse_bytes += 8.0 * (double)words * (double)out->sparse_launches / (double)out->sparse_seen;
+    for (int k = 0; k < TERMEZO_PASS_KINDS; ++k) out->pass_seen[k] = c->prof_seq[2 + k];
+    // the 32-byte sectors of the packed store that the requantisations
+    // rewrote (read and written), in the proportion of the timed passes
+    unsigned long long sectors = 0;
+    cudaMemcpy(&sectors, c->ma.counters + 3, sizeof(sectors), cudaMemcpyDeviceToHost);
+    if (out->pass_seen[PASS_REQUANT])
+      out->pass_bytes[PASS_REQUANT] += 64.0 * (double)sectors * (double)out->pass_launches[PASS_REQUANT] /
+                                       (double)out->pass_seen[PASS_REQUANT];
+    for (int k = 0; k < TERMEZO_PASS_KINDS; ++k) {
+      out->sparse_launches += out->pass_launches[k];
+      out->sparse_seen += out->pass_seen[k];
+      out->sparse_ms += out->pass_ms[k];
+      out->sparse_bytes += out->pass_bytes[k];
+    }
   }
   return TERMEZO_OK;
 }

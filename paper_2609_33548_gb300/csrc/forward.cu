@@ -248,6 +248,21 @@ __device__ __forceinline__ void expand_word(uint32_t w, uint8_t* dst) {
   *reinterpret_cast<uint4*>(dst) = make_uint4(v[0], v[1], v[2], v[3]);
 }
 
+// Value of an e4m3 byte (1 sign, 4 exponent bits with bias 7, 3 mantissa
+// bits); the codes' halves are integers in [-128, 112] and [0, 15].
+__device__ __forceinline__ float e4m3_value(uint32_t b) {
+  const int e = (int)((b >> 3) & 15u), m = (int)(b & 7u);
+  const float v = e ? ldexpf((float)(8 + m), e - 10) : ldexpf((float)m, -9);
+  return (b & 0x80u) ? -v : v;
+}
+
+__global__ void k_codes_i8(const uint8_t* __restrict__ q, int M, int K, int8_t* __restrict__ out) {
+  const uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const uint64_t n = (uint64_t)M * K;
+  if (i >= n) return;
+  out[i] = (int8_t)(int)__fadd_rn(e4m3_value(q[i]), e4m3_value(q[n + i]));
+}
+
 // One thread per packed word.
 __global__ void k_expand_codes(const uint32_t* __restrict__ words, uint64_t n_words, uint8_t* __restrict__ out) {
   const uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -703,6 +718,13 @@ void launch_norm_quant(const float* x, const float* gain, int M, int D, uint8_t*
 void launch_norm_quant_bf16(const uint16_t* x, int M, int D, uint8_t* q, float* deq, cudaStream_t s) {
   kernel_launches() += 1;
   k_norm_quant<Bf16In><<<M, 256, 0, s>>>(reinterpret_cast<const Bf16In*>(x), nullptr, D, q, deq);
+}
+
+void launch_codes_i8(const uint8_t* q, int M, int K, int8_t* out, cudaStream_t s) {
+  const uint64_t n = (uint64_t)M * K;
+  if (!n) return;
+  ++kernel_launches();
+  k_codes_i8<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(q, M, K, out);
 }
 
 void launch_expand_codes(const uint32_t* words, uint64_t rows, int K, uint8_t* out, cudaStream_t s) {

@@ -114,6 +114,9 @@ cudaError_t gemm_launch(const GemmPlan& plan, GemmArgs args, cudaStream_t stream
 // the hi matrix then the lo matrix (ld = D).
 void launch_norm_quant(const float* x, const float* gain, int M, int D, uint8_t* q, float* deq,
                        cudaStream_t s);
+// The int8 activation codes held as e4m3 (hi, lo) pairs in q [2, M, K] (the
+// layout launch_norm_quant writes) -> int8 out [M, K] (hi + lo).
+void launch_codes_i8(const uint8_t* q, int M, int K, int8_t* out, cudaStream_t s);
 // Packed 2-bit codes [rows, K/16] -> e4m3 {-1, 0, +1} [rows, K] bytes.
 void launch_expand_codes(const uint32_t* words, uint64_t rows, int K, uint8_t* out, cudaStream_t s);
 // gate, up codes (two [F, K/16] word matrices) -> e4m3 [256 * ceil(F/128), K]

@@ -53,7 +53,10 @@ std::mutex g_mu;
 tmz::ExactSum* g_addr[kMaxDevices] = {};
 
 // Device address of g_partials for the current device (looked up once per
-// device; host code cannot use the symbol itself as a device pointer).
+// device; host code cannot use the symbol itself as a device pointer).  A
+// cudaDeviceReset destroys the context that holds the array, so the cached
+// address is void afterwards: callers must not reset a device they keep
+// using with this entry point.
 tmz::ExactSum* scratch_for_current_device(int* status) {
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
@@ -87,9 +90,16 @@ extern "C" int termezo_absmean_noalloc(const float* d_w, uint64_t n, float* d_ou
   int status = TERMEZO_OK;
   tmz::ExactSum* parts = scratch_for_current_device(&status);
   if (!parts) return status;
-  const uint32_t nb = (uint32_t)((n + kChunk - 1) / kChunk);
+  uint32_t nb = (uint32_t)((n + kChunk - 1) / kChunk);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  k_noalloc_partial<<<nb, kThreads, 0, st>>>(d_w, n, parts);
-  k_noalloc_final<<<1, kThreads, 0, st>>>(parts, nb, n, d_out);
-  return cudaGetLastError() == cudaSuccess ? TERMEZO_OK : TERMEZO_ECUDA;
+  // cudaLaunchKernel reports the error of this launch only: an earlier,
+  // unrelated error pending on the thread is neither taken as this call's
+  // failure nor cleared from the caller's view.
+  void* a1[] = {(void*)&d_w, (void*)&n, (void*)&parts};
+  if (cudaLaunchKernel((const void*)k_noalloc_partial, dim3(nb), dim3(kThreads), a1, 0, st) != cudaSuccess)
+    return TERMEZO_ECUDA;
+  void* a2[] = {(void*)&parts, (void*)&nb, (void*)&n, (void*)&d_out};
+  if (cudaLaunchKernel((const void*)k_noalloc_final, dim3(1), dim3(kThreads), a2, 0, st) != cudaSuccess)
+    return TERMEZO_ECUDA;
+  return TERMEZO_OK;
 }

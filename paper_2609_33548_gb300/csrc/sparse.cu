@@ -421,35 +421,43 @@ __global__ void __launch_bounds__(TPB) k_sparse_pm_sum(MaskArgs a, int cur, uint
 // write that word, so no two threads write the same word.
 constexpr uint32_t RQ_MAX = 4096;  // elements per sparse block (see the host's block plan)
 
-__device__ __forceinline__ void requant_codes(const MaskArgs& a, int sign, uint64_t seed, float eps, float tau,
-                                              float taup, uint32_t i, float w, uint32_t* code, uint32_t* code_p) {
+__device__ __forceinline__ float requant_codes(const MaskArgs& a, int sign, uint64_t seed, float eps, float tau,
+                                               float taup, uint32_t i, float w, uint32_t* code, uint32_t* code_p) {
   if (sign == 0) {
     *code = ternary_code(w, tau);
     *code_p = *code;
-    return;
+    return w;
   }
   float wp, wm, ee;
   perturbed(w, normal_at(seed, i), eps, &wp, &wm, &ee);
-  *code = ternary_code(sign > 0 ? wp : wm, tau);
+  const float ws = sign > 0 ? wp : wm;
+  *code = ternary_code(ws, tau);
   *code_p = ternary_code(wp, taup);
+  return ws;  // the latent this pass quantises
 }
 
 __global__ void __launch_bounds__(TPB) k_sparse_requant(MaskArgs a, int cur, uint64_t seed, float eps, int sign) {
   __shared__ uint8_t sc[RQ_MAX];
-  __shared__ unsigned long long cnt[3];
-  if (threadIdx.x < 3) cnt[threadIdx.x] = 0;
+  __shared__ unsigned long long cnt[4];
+  if (threadIdx.x < 4) cnt[threadIdx.x] = 0;
   const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
   const uint32_t* idx = a.idx[cur];
   const float* lat = a.lat[cur];
   const float* tau_sel = sign > 0 ? a.tau_plus : (sign < 0 ? a.tau_minus : a.tau_cur);
   const float tau = tau_sel[r.proj];
   const float taup = a.tau_plus[r.proj];
+  // Near-threshold test of the oracle's report, | |w| - tau | < 1e-5 s_w in
+  // float64: near the threshold |w| - tau is exact in fp32 (Sterbenz), and
+  // for an fp32 distance "d < t" with t a float64 equals "d < t rounded up to
+  // fp32", so one float64 product per block suffices.
+  const float sw_sel = sign > 0 ? a.sw_plus[r.proj] : a.sw_minus[r.proj];
+  const float near_thr = sign != 0 ? __double2float_ru(1e-5 * (double)sw_sel) : 0.f;
   const uint32_t n = r.end - r.beg;
   if (n > RQ_MAX) {  // cannot happen with the host's block plan; recorded, never silent
     if (threadIdx.x == 0) atomicOr(a.err, ERR_BOUNDS);
     return;
   }
-  uint32_t flips = 0, jumps = 0, words = 0;
+  uint32_t flips = 0, jumps = 0, words = 0, near = 0;  // words: 32-byte sectors rewritten
   // phase 1: codes of the block's own elements (bits 0-1: this pass, 2-3: + pass)
   for (uint32_t j0 = threadIdx.x; j0 < n; j0 += 4 * TPB) {
 #pragma unroll
@@ -457,7 +465,8 @@ __global__ void __launch_bounds__(TPB) k_sparse_requant(MaskArgs a, int cur, uin
       const uint32_t j = j0 + u * TPB;
       if (j < n) {
         uint32_t c, cp;
-        requant_codes(a, sign, seed, eps, tau, taup, idx[r.beg + j], lat[r.beg + j], &c, &cp);
+        const float ws = requant_codes(a, sign, seed, eps, tau, taup, idx[r.beg + j], lat[r.beg + j], &c, &cp);
+        near += boundary_distance(ws, tau) < near_thr;
         sc[j] = (uint8_t)(c | (cp << 2));
         if (a.wbyte) a.wbyte[idx[r.beg + j]] = code_e4m3(c);
       }
@@ -469,7 +478,8 @@ __global__ void __launch_bounds__(TPB) k_sparse_requant(MaskArgs a, int cur, uin
     const uint32_t i = idx[e];
     if (e != r.seg_beg && (idx[e - 1] >> 4) == (i >> 4)) continue;  // not the leader
     const uint32_t wi = i >> 4;
-    ++words;
+    // the first rewritten word of a 32-byte sector (8 words) counts the sector
+    if (e == r.seg_beg || (idx[e - 1] >> 7) != (i >> 7)) ++words;
     uint32_t word = a.packed[wi];
     for (uint32_t e2 = e; e2 < r.seg_end; ++e2) {
       const uint32_t i2 = idx[e2];
@@ -494,11 +504,13 @@ __global__ void __launch_bounds__(TPB) k_sparse_requant(MaskArgs a, int cur, uin
   if (flips) atomicAdd(&cnt[0], (unsigned long long)flips);
   if (jumps) atomicAdd(&cnt[1], (unsigned long long)jumps);
   if (words) atomicAdd(&cnt[2], (unsigned long long)words);
+  if (near) atomicAdd(&cnt[3], (unsigned long long)near);
   __syncthreads();
   if (threadIdx.x == 0) {
     if (cnt[0]) atomicAdd(&a.counters[0], cnt[0]);
     if (cnt[1]) atomicAdd(&a.counters[1], cnt[1]);
     if (cnt[2]) atomicAdd(&a.counters[3], cnt[2]);
+    if (cnt[3]) atomicAdd(&a.counters[4], cnt[3]);
   }
 }
 

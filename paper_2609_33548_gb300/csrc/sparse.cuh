@@ -44,7 +44,8 @@ struct MaskArgs {
   unsigned long long* grp_tie0; // [P] ties before the first dense block of each group
   float* xi0p;                  // [P] xi_0 of each projection (Eq. 5)
   uint32_t *blk_a, *blk_b, *blk_c, *blk_d;   // per-block scratch
-  unsigned long long* counters; // [0] flipped, [1] jumps, [2] dropped, [3] packed words rewritten
+  unsigned long long* counters; // [0] flipped, [1] jumps, [2] dropped, [3] 32-byte sectors of the packed store rewritten,
+                                // [4] active latents within 1e-5 s_w of +-tau in the +/- passes
   unsigned* err;
 };
 

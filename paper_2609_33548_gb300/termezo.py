@@ -20,7 +20,7 @@ OK, WMASKFIXED, EINVAL, ESTATE, ENOMEM, ECUDA, ETIMEOUT = 0, 1, -1, -2, -3, -4, 
 # Every function declared in include/termezo.h.
 EXPORTS = (
     "termezo_workspace_bytes", "termezo_memory", "termezo_create", "termezo_load_params", "termezo_build_mask",
-    "termezo_build_mask_rule", "termezo_forward_loss", "termezo_step", "termezo_step_k", "termezo_step_joint", "termezo_shrink", "termezo_requantize", "termezo_update",
+    "termezo_build_mask_rule", "termezo_forward_loss", "termezo_forward_trace", "termezo_step", "termezo_step_k", "termezo_step_joint", "termezo_shrink", "termezo_requantize", "termezo_update",
     "termezo_bitlinear", "termezo_state_sizes", "termezo_export_state", "termezo_normal",
     "termezo_absmean_noalloc", "termezo_attention", "termezo_profile", "termezo_destroy", "termezo_strerror",
 )
@@ -36,7 +36,7 @@ class StepOut(ctypes.Structure):
     _fields_ = [("loss_plus", ctypes.c_double), ("loss_minus", ctypes.c_double),
                 ("g", ctypes.c_double), ("k_active", ctypes.c_uint64),
                 ("n_flipped", ctypes.c_uint64), ("n_jumps", ctypes.c_uint64),
-                ("n_dropped", ctypes.c_uint64)]
+                ("n_dropped", ctypes.c_uint64), ("n_near_threshold", ctypes.c_uint64)]
 
     def as_dict(self):
         return {n: getattr(self, n) for n, _ in self._fields_}
@@ -57,11 +57,25 @@ class ProfileOut(ctypes.Structure):
                 ("attn_launches", ctypes.c_uint64), ("attn_ms", ctypes.c_double),
                 ("attn_flops", ctypes.c_double), ("sparse_launches", ctypes.c_uint64),
                 ("sparse_ms", ctypes.c_double), ("sparse_bytes", ctypes.c_double),
-                ("gemm_seen", ctypes.c_uint64), ("attn_seen", ctypes.c_uint64), ("sparse_seen", ctypes.c_uint64)]
+                ("gemm_seen", ctypes.c_uint64), ("attn_seen", ctypes.c_uint64), ("sparse_seen", ctypes.c_uint64),
+                ("pass_launches", ctypes.c_uint64 * 5), ("pass_seen", ctypes.c_uint64 * 5),
+                ("pass_ms", ctypes.c_double * 5), ("pass_bytes", ctypes.c_double * 5)]
 
     def as_dict(self):
-        return {n: getattr(self, n) for n, _ in self._fields_}
+        return {n: (list(getattr(self, n)) if n.startswith("pass_") else getattr(self, n)) for n, _ in self._fields_}
 
+
+# sparse pass kinds of ProfileOut.pass_* (include/termezo.h)
+PASS_KINDS = ("pm_sum", "requant", "update", "shrink", "theta")
+
+
+TRACE_FIELDS = ("x_in", "codes_attn", "deq_attn", "q", "k", "vt", "attn", "codes_o", "deq_o", "x_mid",
+                "codes_mlp", "deq_mlp", "hid", "codes_down", "deq_down", "x_out")
+
+
+class LayerTrace(ctypes.Structure):
+    """termezo_layer_trace: device pointers of the buffers to fill (NULL: skip)."""
+    _fields_ = [(n, ctypes.c_void_p) for n in TRACE_FIELDS]
 
 MASK_GLOBAL, MASK_PER_TENSOR = 0, 1
 
@@ -99,6 +113,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         "termezo_build_mask": (I32, [P, F64, ctypes.POINTER(U64), ctypes.POINTER(F32)]),
         "termezo_build_mask_rule": (I32, [P, F64, I32, ctypes.POINTER(U64), P]),
         "termezo_forward_loss": (I32, [P, P, P, ctypes.POINTER(F64), P]),
+        "termezo_forward_trace": (I32, [P, P, P, I32, ctypes.POINTER(LayerTrace), ctypes.POINTER(F64), P]),
         "termezo_step": (I32, [P, U64, F32, F32, F64, P, P, ctypes.POINTER(StepOut), P, P]),
         "termezo_step_k": (I32, [P, P, I32, F32, F32, F64, P, P, ctypes.POINTER(StepOut), P, P]),
         "termezo_step_joint": (I32, [P, P, I32, F32, F32, F64, P, P, ctypes.POINTER(StepOut), P, P]),
@@ -224,6 +239,32 @@ class Context:
             self.handle, _ptr(tokens), _ptr(targets), ctypes.byref(loss),
             per.ctypes.data_as(ctypes.c_void_p)))
         return loss.value, per
+
+    def termezo_forward_trace(self, tokens, targets, layer: int, fields=TRACE_FIELDS):
+        """Forward at the codes now in the packed store; returns (loss,
+        per-sequence losses, dict of device tensors with the intermediates
+        of `layer` named in `fields`; layer == layers: only x_in, the
+        residual stream after the last layer)."""
+        c = self.cfg
+        T, D, F = c.seq * c.batch, c.hidden, c.ffn
+        hd = c.hidden // c.heads
+        shapes = dict(x_in=((T, D), torch.float32), codes_attn=((T, D), torch.int8), deq_attn=((T,), torch.float32),
+                      q=((c.batch, c.heads, c.seq, hd), torch.int16), k=((c.batch, c.kv_heads, c.seq, hd), torch.int16),
+                      vt=((c.batch, c.kv_heads, hd, c.seq), torch.int16), attn=((T, c.heads * hd), torch.float32),
+                      codes_o=((T, c.heads * hd), torch.int8), deq_o=((T,), torch.float32),
+                      x_mid=((T, D), torch.float32), codes_mlp=((T, D), torch.int8), deq_mlp=((T,), torch.float32),
+                      hid=((T, F), torch.float32), codes_down=((T, F), torch.int8), deq_down=((T,), torch.float32),
+                      x_out=((T, D), torch.float32))
+        if layer == c.layers:
+            fields = ("x_in",)
+        bufs = {n: torch.empty(shapes[n][0], dtype=shapes[n][1], device=self.workspace.device) for n in fields}
+        tr = LayerTrace(**{n: t.data_ptr() for n, t in bufs.items()})
+        loss = ctypes.c_double(0)
+        per = np.zeros(c.batch, dtype=np.float64)
+        _check("termezo_forward_trace", load().termezo_forward_trace(
+            self.handle, _ptr(tokens), _ptr(targets), layer, ctypes.byref(tr), ctypes.byref(loss),
+            per.ctypes.data_as(ctypes.c_void_p)))
+        return loss.value, per, bufs
 
     def termezo_step(self, seed: int, eps: float, lr: float, density: float, tokens, targets):
         out = StepOut()

@@ -18,3 +18,17 @@ def rel_err(a, b):
     a = float(a)
     b = float(b)
     return abs(a - b) / max(abs(b), 1e-300)
+
+
+def record(kind: str, **fields):
+    """Parity evidence: prints one JSON line and appends it to the file named
+    by TERMEZO_PARITY_LOG when that variable is set."""
+    import json
+    import os
+
+    line = json.dumps(dict(kind=kind, **fields), default=float)
+    print(line)
+    path = os.environ.get("TERMEZO_PARITY_LOG")
+    if path:
+        with open(path, "a") as f:
+            f.write(line + "\n")

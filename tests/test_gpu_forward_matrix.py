@@ -13,6 +13,7 @@ from oracle import bitnet, rounding, termezo as otz
 from paper_2609_33548_gb300 import synth
 from paper_2609_33548_gb300 import termezo as tz
 
+from helpers import record
 
 pytestmark = pytest.mark.gpu
 
@@ -54,5 +55,6 @@ def test_forward_loss_matrix(name, cache):
     per_o, _ = bitnet.batch_loss(cfg, split, sw, *th, rows=rows)
     ens = rounding.loss_ensemble(cfg, (split, sw), th, n=8, rows=rows)
     for b in rows:
-        # 1e-3, or inside the spread of valid fp32 roundings of the oracle
+        # 1e-3, or no further from the oracle than its valid fp32 re-roundings
+        record("forward_matrix", workload=name, cache=cache, sequence=b, **rounding.summary(per[b], per_o[b], ens[:, b]))
         assert rounding.within(per[b], per_o[b], ens[:, b]), (name, b, per[b], per_o[b], ens[:, b])

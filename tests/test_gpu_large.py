@@ -10,9 +10,15 @@ configuration bench.py times.
   latents within 1e-5 s_w of a threshold.
 * BitLinear GEMM at the 2B shapes (M 8192 tokens): int32 accumulators of
   sampled rows bit-exact.
-* One step on the 0.7B model: the loss of each sequence depends only on that
-  sequence, so sampled sequences are evaluated by the oracle at +eps z and
-  -eps z (1e-3, or inside the spread of valid fp32 roundings).
+* One step on the 0.7B and 2B models (2B at densities 1 % and 0.1 %): the loss
+  of each sequence depends only on that sequence, so sampled sequences are
+  evaluated by the oracle at +eps z and -eps z.  The per-sequence F+-, and g,
+  must agree to 1e-3 or lie no further from the oracle than the furthest of
+  8 valid fp32 re-roundings of the oracle (oracle/rounding.py); at 24-30
+  layers those move F by several percent, because one flipped activation code
+  changes every later layer, so this comparison is statistical and every
+  value is recorded.  The exact, per-operation parity of these forwards is
+  test_gpu_layerwise.py's.  tau+ and tau- of every projection are bit-exact.
 Inputs are drawn on the host by the seeded generator (so the oracle can
 redraw them anywhere) and copied to the device."""
 import numpy as np
@@ -22,6 +28,8 @@ import torch
 from oracle import bitnet, philox, rounding, ternary, termezo as otz
 from paper_2609_33548_gb300 import synth
 from paper_2609_33548_gb300 import termezo as tz
+
+from helpers import record
 
 pytestmark = pytest.mark.gpu
 
@@ -121,36 +129,52 @@ def test_full_size_per_tensor_mask():
     np.testing.assert_array_equal(st["latents"], w[sel])
 
 
-def test_step_sampled_sequences_0_7b():
-    cfg, density = synth.BITNET_07B, 0.01
+def _step_sampled_sequences(cfg, density, rows, name):
     ctx, dev, (w, emb, gains, head, tok, tgt) = _setup(cfg, density)
     reg = otz.registry(cfg)
-    act = _mask_exact(ctx, w, reg, density)
+    k0, xi0 = ctx.termezo_build_mask(density)
+    act, xi0_o, k0_o, _ = otz.initial_mask(w, reg, density)
+    assert k0 == k0_o and np.float32(xi0).view(np.uint32) == np.float32(xi0_o).view(np.uint32)
     seed = synth.step_seed(0)
     out = ctx.termezo_step(seed, EPS, LR, density, dev[4], dev[5])
     z = philox.normal(seed, act)
     e = (np.float32(EPS) * z).astype(np.float32)
+    del dev[0]
     wp = w.copy()
     wp[act] = (w[act] + e).astype(np.float32)
-    wm = wp.copy()
-    wm[act] = (wp[act] - np.float32(2) * e).astype(np.float32)
     cp, tp, swp = otz.requantize(wp, reg)
+    wp[act] = (wp[act] - np.float32(2) * e).astype(np.float32)
+    wm = wp
+    del w
     cm, tm, swm = otz.requantize(wm, reg)
     st = ctx.termezo_export_state(packed=False)
     np.testing.assert_array_equal(st["tau_plus"].view(np.uint32), tp.view(np.uint32))
     np.testing.assert_array_equal(st["tau_minus"].view(np.uint32), tm.view(np.uint32))
     split = lambda c: [c[p.base:p.base + p.n].reshape(p.N, p.K) for p in reg]
     th = (emb, gains, head, tok, tgt)
-    rows = [0, 1]
     per_p, _ = bitnet.batch_loss(cfg, split(cp), swp, *th, rows=rows)
     per_m, _ = bitnet.batch_loss(cfg, split(cm), swm, *th, rows=rows)
-    ens_p = rounding.loss_ensemble(cfg, (split(cp), swp), th, n=6, rows=rows)
-    ens_m = rounding.loss_ensemble(cfg, (split(cm), swm), th, n=6, rows=rows)
+    ens_p = rounding.loss_ensemble(cfg, (split(cp), swp), th, n=8, rows=rows)
+    ens_m = rounding.loss_ensemble(cfg, (split(cm), swm), th, n=8, rows=rows)
     two_eps = 2 * float(np.float32(EPS))
     for i, b in enumerate(rows):
-        assert rounding.within(out["per_seq_plus"][b], per_p[i], ens_p[:, i]), (b, out["per_seq_plus"][b], per_p[i])
-        assert rounding.within(out["per_seq_minus"][b], per_m[i], ens_m[:, i])
         g_gpu = (out["per_seq_plus"][b] - out["per_seq_minus"][b]) / two_eps
         g_ref = (per_p[i] - per_m[i]) / two_eps
-        assert rounding.within(g_gpu, g_ref, (ens_p[:, i] - ens_m[:, i]) / two_eps), (b, g_gpu, g_ref)
+        g_ens = (ens_p[:, i] - ens_m[:, i]) / two_eps
+        record("sampled_step", workload=name, sequence=b, F_plus=rounding.summary(out["per_seq_plus"][b], per_p[i],
+                                                                                 ens_p[:, i]),
+               F_minus=rounding.summary(out["per_seq_minus"][b], per_m[i], ens_m[:, i]),
+               g=rounding.summary(g_gpu, g_ref, g_ens))
+        assert rounding.within(out["per_seq_plus"][b], per_p[i], ens_p[:, i]), (b, out["per_seq_plus"][b], per_p[i])
+        assert rounding.within(out["per_seq_minus"][b], per_m[i], ens_m[:, i])
+        assert rounding.within(g_gpu, g_ref, g_ens), (b, g_gpu, g_ref)
     assert out["n_jumps"] == 0 and out["k_active"] == act.size
+
+
+def test_step_sampled_sequences_0_7b():
+    _step_sampled_sequences(synth.BITNET_07B, 0.01, [0, 1], "0.7b")
+
+
+@pytest.mark.parametrize("density", [0.01, 0.001])
+def test_step_sampled_sequences_2b(density):
+    _step_sampled_sequences(synth.BITNET_2B, density, [3], f"2b density {density}")
