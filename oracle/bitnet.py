@@ -74,9 +74,15 @@ def act_quant(x: np.ndarray):
 
 
 def int_matmul(q: np.ndarray, codes: np.ndarray) -> np.ndarray:
-    """Exact integer acc[m, n] = sum_k q[m, k] * codes[n, k] (float64 BLAS on
-    integers whose every partial sum stays below 2**53), returned as int64."""
-    acc = q.astype(np.float64) @ codes.astype(np.float64).T
+    """Exact integer acc[m, n] = sum_k q[m, k] * codes[n, k] for int8 codes q
+    (|q| <= 128) and ternary codes, returned as int64.  Every product is an
+    integer of magnitude <= 128 and every partial sum of any subset of them
+    at most 128 K in magnitude; for 128 K < 2**24 all of these are exact in
+    float32, so float32 BLAS returns the exact sums in any summation order.
+    Larger K use float64 (exact below 2**53)."""
+    K = q.shape[-1]
+    dt = np.float32 if 128 * K < (1 << 24) else np.float64
+    acc = q.astype(dt) @ codes.astype(dt).T
     return np.rint(acc).astype(np.int64)
 
 

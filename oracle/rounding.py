@@ -89,14 +89,30 @@ def within(value, ref, ens, rel=1e-3) -> bool:
     return abs(value - ref) <= rel * abs(ref) or abs(value - ref) <= dev
 
 
+def consistent(value, ref, ens, k=5.0) -> bool:
+    """Statistical form for losses that are chaotic in the fp32 roundings (a
+    24-30-layer random-init decoder, where one flipped activation code
+    changes every later layer and the oracle's own re-roundings spread F by
+    several percent): value lies within k sample standard deviations of the
+    mean of [ref] + ens.  For a value drawn from the same distribution as the
+    n + 1 others, (value - mean) / (sd sqrt(1 + 1/(n+1))) is Student-t with n
+    degrees of freedom; k = 5 with n = 8 rejects such a value with
+    probability about 1e-3."""
+    allv = np.concatenate([[ref], np.ravel(ens)]).astype(np.float64)
+    sd = float(np.std(allv, ddof=1))
+    return abs(float(value) - float(allv.mean())) <= k * sd
+
+
 def summary(value, ref, ens) -> dict:
     """|value - ref| next to the ensemble's largest deviation from ref and
     its range, for the parity record."""
     allv = np.concatenate([[ref], np.ravel(ens)])
+    sd = float(np.std(allv, ddof=1)) if allv.size > 1 else 0.0
     return dict(value=float(value), ref=float(ref), abs_err=abs(float(value) - float(ref)),
                 rel_err=abs(float(value) - float(ref)) / max(abs(float(ref)), 1e-300),
                 ens_max_dev=float(np.max(np.abs(np.ravel(ens) - ref))) if np.size(ens) else 0.0,
-                ens_min=float(allv.min()), ens_max=float(allv.max()), n_ens=int(np.size(ens)))
+                ens_min=float(allv.min()), ens_max=float(allv.max()), n_ens=int(np.size(ens)),
+                z=(float(value) - float(allv.mean())) / sd if sd > 0 else 0.0)
 
 
 def g_within_ensemble(g, g_ref, ens, rel=1e-3) -> bool:

@@ -12,13 +12,17 @@ configuration bench.py times.
   sampled rows bit-exact.
 * One step on the 0.7B and 2B models (2B at densities 1 % and 0.1 %): the loss
   of each sequence depends only on that sequence, so sampled sequences are
-  evaluated by the oracle at +eps z and -eps z.  The per-sequence F+-, and g,
-  must agree to 1e-3 or lie no further from the oracle than the furthest of
-  8 valid fp32 re-roundings of the oracle (oracle/rounding.py); at 24-30
-  layers those move F by several percent, because one flipped activation code
-  changes every later layer, so this comparison is statistical and every
-  value is recorded.  The exact, per-operation parity of these forwards is
-  test_gpu_layerwise.py's.  tau+ and tau- of every projection are bit-exact.
+  evaluated by the oracle at +eps z and -eps z, next to 8 valid fp32
+  re-roundings of the oracle (oracle/rounding.py).  At 24-30 layers these
+  move a sequence's F by several percent and its g by tens of percent: one
+  flipped activation code changes every later layer, so the loss of such a
+  random-init decoder is determined by its definition only to that spread.
+  The comparison is therefore statistical: F+-, g lie within 5 sample
+  standard deviations of the mean of the oracle and its re-roundings
+  (rounding.consistent; a false alarm about once in 1000), and every value is
+  recorded.  The exact, per-operation parity of these forwards is
+  test_gpu_layerwise.py's (bit-exact given the same inputs).  tau+ and tau- of
+  every projection are bit-exact.
 Inputs are drawn on the host by the seeded generator (so the oracle can
 redraw them anywhere) and copied to the device."""
 import numpy as np
@@ -165,9 +169,9 @@ def _step_sampled_sequences(cfg, density, rows, name):
                                                                                  ens_p[:, i]),
                F_minus=rounding.summary(out["per_seq_minus"][b], per_m[i], ens_m[:, i]),
                g=rounding.summary(g_gpu, g_ref, g_ens))
-        assert rounding.within(out["per_seq_plus"][b], per_p[i], ens_p[:, i]), (b, out["per_seq_plus"][b], per_p[i])
-        assert rounding.within(out["per_seq_minus"][b], per_m[i], ens_m[:, i])
-        assert rounding.within(g_gpu, g_ref, g_ens), (b, g_gpu, g_ref)
+        assert rounding.consistent(out["per_seq_plus"][b], per_p[i], ens_p[:, i]), (b, out["per_seq_plus"][b], per_p[i])
+        assert rounding.consistent(out["per_seq_minus"][b], per_m[i], ens_m[:, i])
+        assert rounding.consistent(g_gpu, g_ref, g_ens), (b, g_gpu, g_ref)
     assert out["n_jumps"] == 0 and out["k_active"] == act.size
 
 

@@ -24,6 +24,15 @@ def test_int8_ternary_dot_brute_force():
     q = np.full((2, 6912), -128)
     c = np.ones((3, 6912), np.int8)
     assert np.all(bitnet.int_matmul(q, c) == -128 * 6912)
+    # large partial sums followed by small terms, random signs: int64 sums
+    q = np.concatenate([rng.choice([-127, 127], size=(4, 3456)), rng.integers(-3, 4, size=(4, 3456))], axis=1)
+    c = rng.integers(-1, 2, size=(6, 6912)).astype(np.int8)
+    c[0] = 1
+    want = q.astype(np.int64) @ c.astype(np.int64).T
+    np.testing.assert_array_equal(bitnet.int_matmul(q, c), want)
+    # beyond K = 2^17 the float64 path is taken
+    q = np.full((1, 1 << 17), 127)
+    assert bitnet.int_matmul(q, np.ones((1, 1 << 17), np.int8))[0, 0] == 127 << 17
 
 
 def test_act_quant_properties():
