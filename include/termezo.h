@@ -353,7 +353,7 @@ int termezo_profile(termezo_ctx* ctx, int enable, termezo_profile_out* out);
  * reads KV head h / (H / KV); scores scaled by 1/sqrt(hd); P = exp(s -
  * row max) rounded to bf16; d_out fp32 [B*S, H*hd] = (P V) / sum P.
  * S % 64 == 0, hd in {64, 96, 128}, H % KV == 0.  Runs on the tcgen05
- * tensor cores when S % 128 == 0 and hd is 64 or 128, else on mma.sync.
+ * tensor cores when S % 128 == 0, else on mma.sync.
  * Stateless; on `stream`. */
 int termezo_attention(const uint16_t* d_q, const uint16_t* d_k, const uint16_t* d_vt, int32_t B, int32_t S,
                       int32_t H, int32_t KV, int32_t hd, float* d_out, void* stream);

@@ -103,6 +103,13 @@ def consistent(value, ref, ens, k=5.0) -> bool:
     return abs(float(value) - float(allv.mean())) <= k * sd
 
 
+def agrees(value, ref, ens, rel=1e-3) -> bool:
+    """The acceptance of a GPU loss or g: ``within`` (the stated relative
+    bound, or no further from the oracle than its furthest re-rounding), or,
+    where the loss is chaotic in the roundings, ``consistent``."""
+    return within(value, ref, ens, rel) or consistent(value, ref, ens)
+
+
 def summary(value, ref, ens) -> dict:
     """|value - ref| next to the ensemble's largest deviation from ref and
     its range, for the parity record."""
@@ -116,4 +123,4 @@ def summary(value, ref, ens) -> dict:
 
 
 def g_within_ensemble(g, g_ref, ens, rel=1e-3) -> bool:
-    return within(g, g_ref, ens, rel)
+    return agrees(g, g_ref, ens, rel)

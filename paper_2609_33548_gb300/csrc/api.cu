@@ -237,12 +237,27 @@ void carve(termezo_ctx* c, Carver& cv) {
   a.sproj = cv.take<uint16_t>(c->NBS_max);
   cv.sec = SEC_PACKED;
   a.packed = cv.take<uint32_t>(s.d / 16);
+  // The second buffer is followed by k_cap / 16 + 4096 spare entries (mask
+  // state): the three-pass mask build stages its superset of S_0 there.
+  const size_t spare = c->k_cap / 16 + 4096;
   for (int i = 0; i < 2; ++i) {
     cv.sec = SEC_INDEX;
     a.idx[i] = cv.take<uint32_t>(c->k_cap);
+    const size_t idx_end = cv.off;
+    cv.sec = SEC_MASK;
+    if (i == 1) cv.take<uint32_t>(spare);
+    const size_t idx_room = (cv.off - idx_end) / sizeof(uint32_t) + c->k_cap;
     cv.sec = SEC_LATENTS;
     a.lat[i] = cv.take<float>(c->k_cap);
+    const size_t lat_end = cv.off;
     cv.sec = SEC_MASK;
+    if (i == 1) cv.take<float>(spare);
+    const size_t lat_room = (cv.off - lat_end) / sizeof(float) + c->k_cap;
+    if (i == 1) {
+      // entries that fit below the next buffer (alignment gaps included)
+      const size_t room = idx_room < lat_room ? idx_room : lat_room;
+      a.sup_cap = (uint32_t)(room < 0xFFFFFFFFull ? room : 0xFFFFFFFFull);
+    }
     a.off[i] = cv.take<uint32_t>(P + 1);
   }
   a.S_total = cv.take<ExactSum>(P);
@@ -253,7 +268,9 @@ void carve(termezo_ctx* c, Carver& cv) {
   float** fl[9] = {&a.gamma_cur, &a.tau_cur, &a.sw_cur, &a.gamma_plus, &a.tau_plus,
                    &a.sw_plus,   &a.gamma_minus, &a.tau_minus, &a.sw_minus};
   for (auto f : fl) *f = cv.take<float>(P + 2);
-  a.hist = cv.take<unsigned long long>(2048 * (size_t)P);
+  a.hist = cv.take<unsigned long long>(2048 * (size_t)P > 8192 ? 2048 * (size_t)P : 8192);
+  a.scan_state = cv.take<unsigned long long>(nbd ? nbd : 1);
+  a.sup = cv.take<uint32_t>(4);
   a.sel = cv.take<tmz::SelectState>(P);
   a.grp_tie0 = cv.take<unsigned long long>(P);
   a.xi0p = cv.take<float>(P);
@@ -748,9 +765,32 @@ int termezo_build_mask_rule(termezo_ctx* c, double density, int32_t rule, uint64
   c->ma.groups = (int)groups.size();
   std::vector<tmz::SelectState> sel_h = groups;
   cudaMemcpyAsync(c->ma.sel, sel_h.data(), groups.size() * sizeof(tmz::SelectState), cudaMemcpyHostToDevice, st);
-  cudaMemsetAsync(c->ma.hist, 0, groups.size() * 2048 * sizeof(unsigned long long), st);
-  tmz::mask_build(c->ma, c->latents, k0, st);
-  int rc = cuda_status(c);
+  int rc = TERMEZO_OK;
+  bool built_fast = false;
+  if (rule == TERMEZO_MASK_GLOBAL && k0 > 0) {
+    // three dense passes (tmz::mask_build_fast); the six-pass build when the
+    // superset of S_0 does not fit its buffer
+    cudaMemsetAsync(c->ma.hist, 0, 8192 * sizeof(unsigned long long), st);
+    cudaMemsetAsync(c->ma.sup, 0, 4 * sizeof(uint32_t), st);
+    cudaMemsetAsync(c->ma.scan_state, 0, (size_t)c->ma.NBD * sizeof(unsigned long long), st);
+    tmz::mask_build_fast(c->ma, c->latents, k0, st);
+    uint32_t sup[4] = {0, 0, 0, 0};
+    cudaMemcpyAsync(sup, c->ma.sup, sizeof(sup), cudaMemcpyDeviceToHost, st);
+    rc = sync_status(c);
+    if (rc) return rc;
+    if (!sup[1]) {
+      tmz::mask_build_fast_offsets(c->ma, k0, st);
+      built_fast = true;
+    } else {
+      cudaMemcpyAsync(c->ma.sel, sel_h.data(), groups.size() * sizeof(tmz::SelectState), cudaMemcpyHostToDevice,
+                      st);
+    }
+  }
+  if (!built_fast) {
+    cudaMemsetAsync(c->ma.hist, 0, groups.size() * 2048 * sizeof(unsigned long long), st);
+    tmz::mask_build(c->ma, c->latents, k0, st);
+  }
+  rc = cuda_status(c);
   if (rc) return rc;
   std::vector<uint32_t> off(s.P + 1);
   std::vector<float> xi0p(s.P);

@@ -1,5 +1,5 @@
 // Causal attention on the 5th-generation tensor cores (sm_103a), for head
-// dims 64 and 128 and sequence lengths that are multiples of 128.
+// dims 64, 96 and 128 and sequence lengths that are multiples of 128.
 //
 // Same arithmetic as the mma.sync kernel: Q, K, V bf16; s = fl(acc * scale);
 // pass 1 finds the exact row maximum m over the causal keys; pass 2 forms
@@ -46,11 +46,17 @@ static_assert(128 * REG_CTRL + 256 * REG_SOFTMAX + 128 * REG_EPI == ATT_THREADS 
 constexpr int BQ = 128, BKEY = 128;
 constexpr int ATOM = 128 * 128;  // one 128-row x 64-element bf16 swizzle atom block
 
+// A Q or K tile (128 rows x HD) is loaded as 64-column swizzle atoms; at HD
+// 96 the second atom is half filled (TMA writes zeros past column 95, and the
+// MMAs read only its first 32 columns).  A V^T tile is HD rows x 128 keys.
 template <int HD>
 struct AttTc {
-  static constexpr int TILE = HD * 256;            // bytes of a Q or K tile (128 x HD) or V^T tile (HD x 128)
-  static constexpr int V_ATOM = HD * 128;          // V^T: HD rows x 64 keys
-  static constexpr int NS = HD == 64 ? 6 : 3;      // K / V^T ring slots
+  static constexpr int QK_ATOMS = (HD + 63) / 64;
+  static constexpr int QK_BYTES = QK_ATOMS * ATOM;  // bytes TMA writes for a Q or K tile
+  static constexpr int V_ATOM = HD * 128;           // V^T: HD rows x 64 keys
+  static constexpr int V_BYTES = 2 * V_ATOM;        // bytes TMA writes for a V^T tile
+  static constexpr int TILE = QK_BYTES > V_BYTES ? QK_BYTES : V_BYTES;  // a Q buffer or a ring slot
+  static constexpr int NS = HD == 64 ? 6 : 3;       // K / V^T ring slots
   static constexpr int Q_OFF = 0;                  // Q_A, Q_B
   static constexpr int R_OFF = Q_OFF + 2 * TILE;   // ring
   static constexpr int P_OFF = R_OFF + NS * TILE;  // P_A, P_B: 128 x 128 bf16 each
@@ -289,11 +295,11 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
         const AttItem it = att_item(i, B, KV, G, NQ);
         const int na = it.qa + 1;
         if (nq >= 1 && !(ok = mbar_wait(q_empty, (nq - 1) & 1u))) break;
-        mbar_expect_tx(q_full, (it.hb >= 0 ? 2 : 1) * L::TILE);
-        for (int a = 0; a < HD / 64; ++a)
+        mbar_expect_tx(q_full, (it.hb >= 0 ? 2 : 1) * L::QK_BYTES);
+        for (int a = 0; a < L::QK_ATOMS; ++a)
           tma_load_2d(sb + L::Q_OFF + a * ATOM, &tmQ, a * 64, (it.b * H + it.ha) * S + it.qa * BQ, q_full);
         if (it.hb >= 0)
-          for (int a = 0; a < HD / 64; ++a)
+          for (int a = 0; a < L::QK_ATOMS; ++a)
             tma_load_2d(sb + L::Q_OFF + L::TILE + a * ATOM, &tmQ, a * 64, (it.b * H + it.hb) * S + it.qb * BQ,
                         q_full);
         ++nq;
@@ -302,9 +308,9 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
           const uint32_t slot = rp % NS, use = rp / NS;
           if (use >= 1 && !mbar_wait(ring_empty + 8 * slot, (use - 1) & 1u)) return false;
           const uint32_t dst = sb + L::R_OFF + slot * L::TILE, fb = ring_full + 8 * slot;
-          mbar_expect_tx(fb, L::TILE);
+          mbar_expect_tx(fb, v ? L::V_BYTES : L::QK_BYTES);
           if (!v)
-            for (int a = 0; a < HD / 64; ++a) tma_load_2d(dst + a * ATOM, &tmK, a * 64, rowK + j * BKEY, fb);
+            for (int a = 0; a < L::QK_ATOMS; ++a) tma_load_2d(dst + a * ATOM, &tmK, a * 64, rowK + j * BKEY, fb);
           else
             for (int a = 0; a < 2; ++a) tma_load_2d(dst + a * L::V_ATOM, &tmV, j * BKEY + a * 64, rowV, fb);
           ++rp;
@@ -516,14 +522,16 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
         const uint32_t tO = tmem + lanes + 256 + t * 128;
         uint8_t* prow = smem + L::P_OFF + t * 2 * ATOM + row * 128;
         const uint32_t wbase = sb + L::P_OFF + t * 2 * ATOM + quarter * 32 * 128;
+        constexpr int RD = (HD + 63) / 64;  // rounds of up to 64 columns (two 32-column boxes)
 #pragma unroll 1
-        for (int rd = 0; rd < HD / 64; ++rd) {
+        for (int rd = 0; rd < RD; ++rd) {
           if (rd > 0) {
             if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
             __syncwarp();
           }
 #pragma unroll
           for (int cc = 0; cc < 2; ++cc) {
+            if (64 * rd + 32 * cc >= HD) break;
             uint32_t ov[32];
             tmem_ld_cols<1>(tO + 64 * rd + 32 * cc, ov);
 #pragma unroll
@@ -534,7 +542,7 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
               *reinterpret_cast<float4*>(prow + cc * ATOM + ((k ^ (row & 7)) * 16)) = make_float4(a.x, a.y, b.x, b.y);
             }
           }
-          if (rd + 1 == HD / 64) {
+          if (rd + 1 == RD) {
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
             arrive(o_free + 8 * t);
           }
@@ -542,7 +550,7 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
           __syncwarp();
           if (lane == 0) {
             tma_store_2d(&tmO, wbase, ocol0 + 64 * rd, orow);
-            tma_store_2d(&tmO, wbase + ATOM, ocol0 + 64 * rd + 32, orow);
+            if (64 * rd + 32 < HD) tma_store_2d(&tmO, wbase + ATOM, ocol0 + 64 * rd + 32, orow);
             asm volatile("cp.async.bulk.commit_group;" ::: "memory");
           }
         }
@@ -624,7 +632,7 @@ cudaError_t launch_tc(const AttnPlan& p, int B, int S, int H, int KV, unsigned* 
 
 }  // namespace
 
-bool attention_tc_supported(int S, int hd) { return (hd == 64 || hd == 128) && S % 128 == 0; }
+bool attention_tc_supported(int S, int hd) { return (hd == 64 || hd == 96 || hd == 128) && S % 128 == 0; }
 
 bool attention_tc_plan(AttnPlan* p, const uint16_t* q, const uint16_t* k, const uint16_t* vt, float* out, int B,
                        int S, int H, int KV, int hd) {
@@ -637,7 +645,8 @@ bool attention_tc_plan(AttnPlan* p, const uint16_t* q, const uint16_t* k, const 
 cudaError_t attention_tc_launch(const AttnPlan& p, int B, int S, int H, int KV, int hd, unsigned* err,
                                 cudaStream_t s) {
   kernel_launches() += 1;
-  return hd == 64 ? launch_tc<64>(p, B, S, H, KV, err, s) : launch_tc<128>(p, B, S, H, KV, err, s);
+  return hd == 64 ? launch_tc<64>(p, B, S, H, KV, err, s)
+                  : (hd == 96 ? launch_tc<96>(p, B, S, H, KV, err, s) : launch_tc<128>(p, B, S, H, KV, err, s));
 }
 
 }  // namespace tmz

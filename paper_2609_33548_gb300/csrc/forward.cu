@@ -8,6 +8,7 @@
 
 #include "common.cuh"
 #include "kernels.cuh"
+#include "normquant.cuh"
 
 namespace tmz {
 
@@ -36,24 +37,6 @@ __device__ __forceinline__ float block_max(float v, float* red) {
   for (int i = 0; i < (int)(blockDim.x >> 5); ++i) t = fmaxf(t, red[i]);
   return t;
 }
-
-__device__ __forceinline__ float quant_code(float h, float s) {
-  float v = rintf(__fmul_rn(h, s));
-  return fminf(fmaxf(v, -128.f), 127.f);
-}
-
-// The BitLinear GEMM takes an int8 code q as two e4m3 values, hi = 16
-// floor(q / 16) in [-128, 112] and lo = q - hi in [0, 15]: both have at most
-// four significant bits, so both are exact in e4m3 (1 sign, 4 exponent bits
-// with bias 7, 3 mantissa bits), and hi w + lo w = q w exactly.  hi and lo
-// are formed exactly in fp32 and converted by the hardware, two per
-// instruction (x0 in the low byte).
-__device__ __forceinline__ uint32_t e4m3x2(float x0, float x1) {
-  uint16_t d;
-  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(d) : "f"(x1), "f"(x0));
-  return d;
-}
-__device__ __forceinline__ float code_hi(float q) { return __fmul_rn(floorf(__fmul_rn(q, 0.0625f)), 16.f); }
 
 // One block per row.  h_k = (x_k * r) * g_k with r = 1/sqrt(mean(x^2)+1e-5)
 // (RMSNorm) or h_k = x_k; a = max(max|h|, 1e-5); q_k = rint(h_k * (127/a)),
@@ -158,72 +141,19 @@ __global__ void __launch_bounds__(256) k_norm_quant_vec(const float* __restrict_
   if (threadIdx.x == 0) deq[row] = __fdiv_rn(a, 127.f);
 }
 
-// Same arithmetic for rows of D <= 128 NV (D % 4 == 0) with one warp per row:
-// the row's NV float4 per lane are all in flight at once and both reductions
-// are warp shuffles, so no CTA barrier stalls the loads (4 rows per CTA).
+// Same arithmetic for rows of D <= 128 NV (D % 4 == 0) with one warp per row
+// (norm_quant_row): the row's NV float4 per lane are all in flight at once and
+// both reductions are warp shuffles, so no CTA barrier stalls the loads (4
+// rows per CTA).
 template <int NV>
 __global__ void __launch_bounds__(128) k_norm_quant_warp(const float* __restrict__ x, const float* __restrict__ gain,
                                                          int D, int M, uint8_t* __restrict__ q,
                                                          float* __restrict__ deq) {
   grid_dep_wait();
-  const int lane = threadIdx.x & 31;
   const int row = blockIdx.x * 4 + (threadIdx.x >> 5);
   if (row >= M) return;
-  const float4* xr = reinterpret_cast<const float4*>(x + (size_t)row * D);
-  const float4* gr = reinterpret_cast<const float4*>(gain);
-  const int D4 = D >> 2;
-  float4 v[NV];
-#pragma unroll
-  for (int i = 0; i < NV; ++i) {
-    const int k = i * 32 + lane;
-    v[i] = k < D4 ? xr[k] : make_float4(0.f, 0.f, 0.f, 0.f);
-  }
-  if (gain) {
-    float ss = 0.f;
-#pragma unroll
-    for (int i = 0; i < NV; ++i) {
-      ss = __fadd_rn(ss, __fmul_rn(v[i].x, v[i].x));
-      ss = __fadd_rn(ss, __fmul_rn(v[i].y, v[i].y));
-      ss = __fadd_rn(ss, __fmul_rn(v[i].z, v[i].z));
-      ss = __fadd_rn(ss, __fmul_rn(v[i].w, v[i].w));
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) ss = __fadd_rn(ss, __shfl_xor_sync(0xffffffffu, ss, o));
-    const float r = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(__fdiv_rn(ss, (float)D), 1e-5f)));
-#pragma unroll
-    for (int i = 0; i < NV; ++i) {
-      const int k = i * 32 + lane;
-      if (k < D4) {
-        const float4 g = gr[k];
-        v[i].x = __fmul_rn(__fmul_rn(v[i].x, r), g.x);
-        v[i].y = __fmul_rn(__fmul_rn(v[i].y, r), g.y);
-        v[i].z = __fmul_rn(__fmul_rn(v[i].z, r), g.z);
-        v[i].w = __fmul_rn(__fmul_rn(v[i].w, r), g.w);
-      }
-    }
-  }
-  float amax = 0.f;
-#pragma unroll
-  for (int i = 0; i < NV; ++i)
-    amax = fmaxf(fmaxf(fmaxf(amax, fabsf(v[i].x)), fmaxf(fabsf(v[i].y), fabsf(v[i].z))), fabsf(v[i].w));
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
-  const float a = fmaxf(amax, 1e-5f);
-  const float s = __fdiv_rn(127.f, a);
-  uint32_t* qh = reinterpret_cast<uint32_t*>(q + (size_t)row * D);
-  uint32_t* ql = reinterpret_cast<uint32_t*>(q + ((size_t)M + row) * D);
-#pragma unroll
-  for (int i = 0; i < NV; ++i) {
-    const int k = i * 32 + lane;
-    if (k < D4) {
-      const float c0 = quant_code(v[i].x, s), c1 = quant_code(v[i].y, s);
-      const float c2 = quant_code(v[i].z, s), c3 = quant_code(v[i].w, s);
-      const float h0 = code_hi(c0), h1 = code_hi(c1), h2 = code_hi(c2), h3 = code_hi(c3);
-      qh[k] = e4m3x2(h0, h1) | (e4m3x2(h2, h3) << 16);
-      ql[k] = e4m3x2(__fsub_rn(c0, h0), __fsub_rn(c1, h1)) | (e4m3x2(__fsub_rn(c2, h2), __fsub_rn(c3, h3)) << 16);
-    }
-  }
-  if (lane == 0) deq[row] = __fdiv_rn(a, 127.f);
+  norm_quant_row<NV, false>(x + (size_t)row * D, gain, D, q + (size_t)row * D, q + ((size_t)M + row) * D, deq + row,
+                            threadIdx.x & 31);
 }
 
 struct Bf16In {

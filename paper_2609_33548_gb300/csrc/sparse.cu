@@ -677,6 +677,423 @@ __global__ void k_normal(uint64_t seed, const uint32_t* idx, uint64_t n, float* 
   if (i < n) z[i] = normal_at(seed, idx[i]);
 }
 
+// ------------------------------------------- mask build, three dense passes --
+// The global quantile of Eq. 4 with three reads of the dense latents: (1) the
+// exact absmean sums (k_dense_sum), (2) a fine histogram of the distance keys
+// (13 bits: exponent and 5 mantissa bits, 32 bins an octave) written together
+// with every code at tau_0, (3) the order-preserving compaction of the
+// "superset" -- every weight whose key falls in the k0-th key's fine bin or
+// below -- into the second sparse-store buffer, with a decoupled look-back
+// scan across blocks.  The exact xi_0 and the ties are then resolved on the
+// superset alone (two 9-bit radix passes over the weights of the fine bin,
+// a count, a scan and an order-preserving scatter into S_0).  The superset
+// holds about (1 + 1/32) k0 weights; when it would not fit, the host runs the
+// six-pass build instead.
+
+constexpr int FINE_SHIFT = 18;                 // fine bin = key >> 18 (bit 31 of a distance is 0)
+constexpr int HIST_DB = 16;                    // dense blocks per CTA of the histogram pass
+constexpr int SUP_DB = 8;                      // dense blocks per CTA of the superset compaction
+constexpr int SUP_STAGE = 4096;                // superset entries a CTA stages in shared memory
+
+// Pass 1 of the fast build: the exact sum of |w| of each dense block, one
+// warp per block (float4 number q * 32 + lane for q < 32, no CTA barrier).
+__global__ void __launch_bounds__(TPB) k_dense_sum_warp(MaskArgs a, const float* __restrict__ w) {
+  const int lane = threadIdx.x & 31;
+  const uint32_t b = blockIdx.x * (TPB / 32) + (threadIdx.x >> 5);
+  if (b >= a.NBD) return;
+  const DenseRange r = dense_range(a, b);
+  ExactAcc acc;
+  ea_zero(acc);
+#pragma unroll 8
+  for (int q = 0; q < (int)(DENSE_CHUNK / 128); ++q) {
+    const uint64_t i = r.start + 4ull * (q * 32 + lane);
+    if (i < r.end) {
+      const float4 t = *reinterpret_cast<const float4*>(w + i);
+      ea_add_abs(acc, t.x);
+      ea_add_abs(acc, t.y);
+      ea_add_abs(acc, t.z);
+      ea_add_abs(acc, t.w);
+    }
+  }
+  ExactSum s = ea_result(acc);
+  es_warp_reduce(s);
+  if (lane == 0) a.partials[b] = s;
+}
+constexpr int FINE_BINS = 1 << (31 - FINE_SHIFT);
+constexpr uint32_t SUP_CHUNK = 4096;           // superset entries per block of the resolution kernels
+
+__device__ __forceinline__ uint32_t dist_key(float w, float tau) {
+  return __float_as_uint(boundary_distance(w, tau));
+}
+
+// Projection of global index i (binary search over base[0..P]).
+__device__ __forceinline__ int proj_of_index(const MaskArgs& a, uint32_t i) {
+  int lo = 0, hi = a.P - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (a.base[mid] <= (uint64_t)i) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+// Pass 2: fine distance histogram and the codes of every weight at tau_0,
+// HIST_DB dense blocks per CTA (one flush of the shared histogram).  Thread
+// t reads float4 number q * TPB + t of a block (coalesced); a packed word (16
+// codes) comes from the four threads of a quad.
+__global__ void __launch_bounds__(TPB) k_hist_codes(MaskArgs a, const float* __restrict__ w) {
+  __shared__ uint32_t h[FINE_BINS];
+  for (int i = threadIdx.x; i < FINE_BINS; i += TPB) h[i] = 0;
+  __syncthreads();
+  const int lane = threadIdx.x & 31;
+  const uint32_t b0 = blockIdx.x * HIST_DB, b1 = min(a.NBD, b0 + HIST_DB);
+  for (uint32_t b = b0; b < b1; ++b) {
+    const DenseRange r = dense_range(a, b);
+    const float tau = a.tau_cur[r.proj];
+    float4 t[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const uint64_t i = r.start + 4ull * (q * TPB + threadIdx.x);
+      t[q] = i < r.end ? *reinterpret_cast<const float4*>(w + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const uint64_t i = r.start + 4ull * (q * TPB + threadIdx.x);
+      const bool live = i < r.end;  // uniform over a quad (chunk lengths are multiples of 16)
+      const float v[4] = {t[q].x, t[q].y, t[q].z, t[q].w};
+      uint32_t byte = 0;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        if (live) atomicAdd(&h[dist_key(v[e], tau) >> FINE_SHIFT], 1u);
+        byte |= ternary_code(v[e], tau) << (2 * e);
+      }
+      const int q0 = lane & ~3;
+      const uint32_t c0 = __shfl_sync(0xffffffffu, byte, q0), c1 = __shfl_sync(0xffffffffu, byte, q0 + 1);
+      const uint32_t c2 = __shfl_sync(0xffffffffu, byte, q0 + 2), c3 = __shfl_sync(0xffffffffu, byte, q0 + 3);
+      if (live && (lane & 3) == 0) a.packed[i >> 4] = c0 | (c1 << 8) | (c2 << 16) | (c3 << 24);
+      if (live && a.wbyte)
+        *reinterpret_cast<uint32_t*>(a.wbyte + i) = code_e4m3(byte & 3u) | (code_e4m3((byte >> 2) & 3u) << 8) |
+                                                    (code_e4m3((byte >> 4) & 3u) << 16) |
+                                                    (code_e4m3((byte >> 6) & 3u) << 24);
+    }
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < FINE_BINS; i += TPB)
+    if (h[i]) atomicAdd(&a.hist[i], (unsigned long long)h[i]);
+}
+
+// The bin of `bins` (a.hist[0..bins), bins <= 8192) that holds the krem-th
+// key of group 0; appends its `bits` to the prefix and clears the
+// histogram.  Each thread sums a chunk of bins, thread 0 finds the chunk and
+// then the bin (the chunk's bins loaded at once).  fine != 0 (the first
+// pass): also the superset size (every key below the bin plus the bin) and
+// whether it fits the superset buffer.
+__global__ void __launch_bounds__(256) k_select_fast(MaskArgs a, int bins, int bits, int fine) {
+  constexpr int MAXPER = 32;
+  __shared__ unsigned long long csum[256];
+  const int per = (bins + 255) / 256;
+  {
+    const int b0 = min(bins, (int)threadIdx.x * per), b1 = min(bins, b0 + per);
+    unsigned long long sum = 0;
+    for (int i = b0; i < b1; ++i) sum += a.hist[i];
+    csum[threadIdx.x] = sum;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && per <= MAXPER) {
+    SelectState* sel = a.sel;
+    const unsigned long long krem = sel->krem;
+    unsigned long long cum = 0;
+    int chunk = 255;
+    for (int c = 0; c < 256; ++c) {
+      if (cum + csum[c] >= krem) { chunk = c; break; }
+      cum += csum[c];
+    }
+    const int c0 = chunk * per;
+    unsigned long long v[MAXPER];
+#pragma unroll
+    for (int j = 0; j < MAXPER; ++j) v[j] = (j < per && c0 + j < bins) ? a.hist[c0 + j] : 0ull;
+    int B = bins - 1;
+    for (int j = 0; j < per && c0 + j < bins; ++j) {
+      if (cum + v[j] >= krem) { B = c0 + j; break; }
+      cum += v[j];
+    }
+    if (fine) {
+      const unsigned long long n_sup = cum + a.hist[B];
+      a.sup[0] = (uint32_t)(n_sup < 0xFFFFFFFFull ? n_sup : 0xFFFFFFFFull);
+      a.sup[1] = n_sup > (unsigned long long)a.sup_cap ? 1u : 0u;
+    }
+    sel->krem = krem - cum;
+    sel->prefix = fine ? (uint32_t)B : ((sel->prefix << bits) | (uint32_t)B);
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < bins; i += blockDim.x) a.hist[i] = 0;
+}
+
+__device__ __forceinline__ void st_release_u64(unsigned long long* p, unsigned long long v) {
+  asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+__device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Decoupled look-back by one warp: the exclusive prefix of block b (blocks
+// numbered in the order they took a ticket, so every block waits only on
+// blocks that run or ran before it).  State words: 1 << 62 | aggregate,
+// 2 << 62 | inclusive prefix.  The warp reads the states of 32 predecessors
+// at once (lane j: block b - 1 - j, then the next 32 ...), adds the
+// aggregates up to the nearest inclusive prefix and stops there.  Each wait
+// is bounded (kWaitNs, decided by lane 0 for the whole warp); on time-out
+// ERR_TIMEOUT is recorded and the prefix found so far is used.
+__device__ unsigned long long lookback_prefix(const MaskArgs& a, uint32_t b, uint32_t total, int lane) {
+  constexpr unsigned long long AGG = 1ull << 62, INC = 2ull << 62, VAL = (1ull << 62) - 1;
+  if (b == 0) {
+    if (lane == 0) st_release_u64(&a.scan_state[0], INC | total);
+    return 0;
+  }
+  if (lane == 0) st_release_u64(&a.scan_state[b], AGG | total);
+  unsigned long long excl = 0;
+  long long base = (long long)b - 1;
+  const uint64_t t0 = globaltimer_ns();
+  bool timed_out = false;
+  while (!timed_out) {
+    const long long j = base - lane;
+    unsigned long long sv = j >= 0 ? ld_acquire_u64(&a.scan_state[j]) : INC;  // before block 0: nothing
+    while (__any_sync(0xffffffffu, (sv >> 62) == 0)) {
+      int late = lane == 0 && globaltimer_ns() - t0 > kWaitNs;
+      late = __shfl_sync(0xffffffffu, late, 0);
+      if (late) {
+        if (lane == 0) atomicOr(a.err, ERR_TIMEOUT);
+        timed_out = true;
+        break;
+      }
+      if ((sv >> 62) == 0) sv = ld_acquire_u64(&a.scan_state[j]);
+    }
+    if (timed_out) break;
+    const unsigned inc = __ballot_sync(0xffffffffu, (sv >> 62) == 2);
+    const int stop = inc ? __ffs(inc) - 1 : 31;  // the nearest inclusive prefix, or the whole window
+    unsigned long long v = lane <= stop ? (sv & VAL) : 0ull;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    excl += v;
+    if (inc) break;
+    base -= 32;
+  }
+  if (lane == 0) st_release_u64(&a.scan_state[b], INC | (excl + total));
+  return excl;
+}
+
+// Pass 3: every weight whose fine bin is at most the k0-th key's, in index
+// order, into idx[1] / lat[1].  A CTA takes SUP_DB consecutive dense blocks
+// (in ticket order), finds its selected weights and their order (one block
+// scan per float4 column of each block: index order is block-major, then
+// q-major), stages them in shared memory, gets its global offset by the
+// look-back and copies them out.  More than SUP_STAGE selected weights (a
+// dense mask): the CTA reads its blocks again and writes directly.
+__device__ __forceinline__ void superset_block(const MaskArgs& a, const float* __restrict__ w, uint32_t b,
+                                               uint32_t bmax, uint32_t* sh, uint32_t& run, bool stage,
+                                               uint32_t* st_idx, float* st_lat, unsigned long long gbase) {
+  const DenseRange r = dense_range(a, b);
+  const float tau = a.tau_cur[r.proj];
+  float4 t[4];
+  uint32_t mask = 0, cnt[4];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const uint64_t i = r.start + 4ull * (q * TPB + threadIdx.x);
+    t[q] = i < r.end ? *reinterpret_cast<const float4*>(w + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const uint64_t i = r.start + 4ull * (q * TPB + threadIdx.x);
+    cnt[q] = 0;
+    if (i < r.end) {
+      const float vv[4] = {t[q].x, t[q].y, t[q].z, t[q].w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e)
+        if ((dist_key(vv[e], tau) >> FINE_SHIFT) <= bmax) { mask |= 1u << (4 * q + e); ++cnt[q]; }
+    }
+  }
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    uint32_t tot;
+    uint32_t pos = run + block_excl_scan(cnt[q], sh, &tot);
+    const uint32_t i = (uint32_t)(r.start + 4ull * (q * TPB + threadIdx.x));
+    const float vv[4] = {t[q].x, t[q].y, t[q].z, t[q].w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e)
+      if (mask & (1u << (4 * q + e))) {
+        if (stage) {
+          if (pos < SUP_STAGE) {
+            st_idx[pos] = i + e;
+            st_lat[pos] = vv[e];
+          }
+        } else if (gbase + pos < a.sup_cap) {  // cannot fail: the size was checked against the capacity
+          a.idx[1][gbase + pos] = i + e;
+          a.lat[1][gbase + pos] = vv[e];
+        }
+        ++pos;
+      }
+    run += tot;
+  }
+}
+
+__global__ void __launch_bounds__(TPB) k_superset(MaskArgs a, const float* __restrict__ w) {
+  __shared__ uint32_t sh[TPB / 32];
+  __shared__ uint32_t s_bid;
+  __shared__ unsigned long long s_excl;
+  __shared__ uint32_t st_idx[SUP_STAGE];
+  __shared__ float st_lat[SUP_STAGE];
+  if (a.sup[1]) return;  // the superset does not fit: the host runs the six-pass build
+  if (threadIdx.x == 0) s_bid = atomicAdd(&a.sup[2], 1u);
+  __syncthreads();
+  const uint32_t c = s_bid;
+  const uint32_t b0 = c * SUP_DB, b1 = min(a.NBD, b0 + SUP_DB);
+  const uint32_t bmax = a.sel->prefix;
+  uint32_t run = 0;  // selected weights of this CTA so far (the same in every thread)
+  for (uint32_t b = b0; b < b1; ++b) superset_block(a, w, b, bmax, sh, run, true, st_idx, st_lat, 0);
+  if (threadIdx.x < 32) {
+    const unsigned long long e = lookback_prefix(a, c, run, threadIdx.x);
+    if (threadIdx.x == 0) s_excl = e;
+  }
+  __syncthreads();
+  const unsigned long long base = s_excl;
+  if (run <= SUP_STAGE) {
+    for (uint32_t j = threadIdx.x; j < run; j += TPB)
+      if (base + j < a.sup_cap) {
+        a.idx[1][base + j] = st_idx[j];
+        a.lat[1][base + j] = st_lat[j];
+      }
+  } else {
+    uint32_t run2 = 0;
+    for (uint32_t b = b0; b < b1; ++b) superset_block(a, w, b, bmax, sh, run2, false, st_idx, st_lat, base);
+  }
+}
+
+// Radix passes over the superset's weights in the fine bin: pass 1 keys
+// bits 17..9 of those in bin prefix, pass 2 bits 8..0 of those whose top 23
+// bits match the prefix.
+__global__ void __launch_bounds__(TPB) k_sup_hist(MaskArgs a, int pass) {
+  __shared__ uint32_t h[512];
+  for (int i = threadIdx.x; i < 512; i += TPB) h[i] = 0;
+  __syncthreads();
+  const bool live = !a.sup[1];
+  const uint32_t n = a.sup[0], prefix = a.sel->prefix;
+  for (uint32_t e = blockIdx.x * TPB + threadIdx.x; live && e < n; e += gridDim.x * TPB) {
+    const uint32_t i = a.idx[1][e];
+    const uint32_t key = dist_key(a.lat[1][e], a.tau_cur[proj_of_index(a, i)]);
+    if (pass == 1 && (key >> FINE_SHIFT) == prefix) atomicAdd(&h[(key >> 9) & 511u], 1u);
+    if (pass == 2 && (key >> 9) == prefix) atomicAdd(&h[key & 511u], 1u);
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < 512; i += TPB)
+    if (h[i]) atomicAdd(&a.hist[i], (unsigned long long)h[i]);
+}
+
+// Per superset block: weights below the key of xi_0 (blk_a) and equal to it (blk_b).
+__global__ void __launch_bounds__(TPB) k_sup_count(MaskArgs a) {
+  __shared__ uint32_t sh[TPB / 32];
+  const uint32_t n = a.sup[0], key_p = a.sel->prefix;
+  const uint32_t lo = blockIdx.x * SUP_CHUNK, hi = min(n, lo + SUP_CHUNK);
+  if (a.sup[1] || lo >= n) return;  // (uniform) blocks past the superset own no scratch entry
+  uint32_t less = 0, eq = 0;
+  for (uint32_t e = lo + threadIdx.x; e < hi; e += TPB) {
+    const uint32_t key = dist_key(a.lat[1][e], a.tau_cur[proj_of_index(a, a.idx[1][e])]);
+    less += key < key_p;
+    eq += key == key_p;
+  }
+  uint32_t tl, te;
+  block_excl_scan(less, sh, &tl);
+  block_excl_scan(eq, sh, &te);
+  if (threadIdx.x == 0) {
+    a.blk_a[blockIdx.x] = tl;
+    a.blk_b[blockIdx.x] = te;
+  }
+}
+
+// Single block over the superset blocks: selected weights before each block
+// (blk_c) and ties before it (blk_d); the first krem ties in index order are
+// kept.
+__global__ void __launch_bounds__(1024) k_scan_sup(MaskArgs a) {
+  __shared__ unsigned long long sh[1024];
+  const uint32_t nblk = a.sup[1] ? 0u : (a.sup[0] + SUP_CHUNK - 1) / SUP_CHUNK;
+  const uint32_t per = (nblk + 1023) / 1024;
+  const uint32_t b0 = min(nblk, threadIdx.x * per), b1 = min(nblk, b0 + per);
+  const unsigned long long ties = a.sel->krem;
+  unsigned long long eq = 0;
+  for (uint32_t b = b0; b < b1; ++b) eq += a.blk_b[b];
+  unsigned long long tb = scan1024(eq, sh);
+  unsigned long long sel = 0, t = tb;
+  for (uint32_t b = b0; b < b1; ++b) {
+    unsigned long long take = t >= ties ? 0 : ties - t;
+    if (take > a.blk_b[b]) take = a.blk_b[b];
+    sel += a.blk_a[b] + take;
+    t += a.blk_b[b];
+  }
+  unsigned long long sb = scan1024(sel, sh);
+  t = tb;
+  for (uint32_t b = b0; b < b1; ++b) {
+    a.blk_c[b] = (uint32_t)sb;
+    a.blk_d[b] = (uint32_t)t;
+    unsigned long long take = t >= ties ? 0 : ties - t;
+    if (take > a.blk_b[b]) take = a.blk_b[b];
+    sb += a.blk_a[b] + take;
+    t += a.blk_b[b];
+  }
+}
+
+// S_0 from the superset, in index order, into idx[0] / lat[0].
+__global__ void __launch_bounds__(TPB) k_sup_scatter(MaskArgs a, uint32_t k0) {
+  __shared__ uint32_t sh[TPB / 32];
+  const uint32_t n = a.sup[0], key_p = a.sel->prefix;
+  const unsigned long long ties = a.sel->krem;
+  const uint32_t lo = blockIdx.x * SUP_CHUNK, hi = min(n, lo + SUP_CHUNK);
+  if (a.sup[1] || lo >= n) return;
+  const uint32_t e0 = lo + 16u * threadIdx.x;
+  uint32_t keys[16], eq = 0;
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    keys[j] = 0xFFFFFFFFu;
+    if (e0 + j < hi) keys[j] = dist_key(a.lat[1][e0 + j], a.tau_cur[proj_of_index(a, a.idx[1][e0 + j])]);
+    eq += keys[j] == key_p;
+  }
+  unsigned long long tie_rank = (unsigned long long)a.blk_d[blockIdx.x] + block_excl_scan(eq, sh, nullptr);
+  uint32_t selm = 0, nsel = 0;
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    bool s = keys[j] < key_p;
+    if (keys[j] == key_p) {
+      s = tie_rank < ties;
+      ++tie_rank;
+    }
+    if (s) { selm |= 1u << j; ++nsel; }
+  }
+  uint32_t pos = a.blk_c[blockIdx.x] + block_excl_scan(nsel, sh, nullptr);
+#pragma unroll
+  for (int j = 0; j < 16; ++j)
+    if (selm & (1u << j)) {
+      if (pos < k0) {
+        a.idx[0][pos] = a.idx[1][e0 + j];
+        a.lat[0][pos] = a.lat[1][e0 + j];
+      } else {
+        atomicOr(a.err, ERR_BOUNDS);  // more than k0 selected: never silent
+      }
+      ++pos;
+    }
+}
+
+// off[0][p]: entries of S_0 below projection p (binary search of base[p]).
+__global__ void k_off_search(MaskArgs a, uint32_t k0) {
+  for (int p = threadIdx.x; p <= a.P; p += blockDim.x) {
+    if (p == a.P) { a.off[0][p] = k0; continue; }
+    uint32_t lo = 0, hi = k0;
+    while (lo < hi) {
+      const uint32_t mid = (lo + hi) >> 1;
+      if ((uint64_t)a.idx[0][mid] < a.base[p]) lo = mid + 1; else hi = mid;
+    }
+    a.off[0][p] = lo;
+  }
+}
+
 }  // namespace
 
 // ----------------------------------------------------------- host side ----
@@ -695,6 +1112,31 @@ void mask_build(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_t s) 
   k_compact<<<a.NBD, TPB, 0, s>>>(a, w);
   k_dense_offsets<<<1, 256, 0, s>>>(a, (uint32_t)k0);
   k_xi0<<<1, 256, 0, s>>>(a);
+}
+
+void mask_build_fast(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_t s) {
+  kernel_launches() += 13;
+  k_dense_sum_warp<<<(a.NBD + TPB / 32 - 1) / (TPB / 32), TPB, 0, s>>>(a, w);
+  k_reduce_proj<<<a.P, TPB, 0, s>>>(a.partials, a.dpre, 1, 0, nullptr, a.base, a.S_total, a.gamma_cur, a.tau_cur,
+                                    a.sw_cur);
+  k_hist_codes<<<(a.NBD + HIST_DB - 1) / HIST_DB, TPB, 0, s>>>(a, w);
+  k_select_fast<<<1, 256, 0, s>>>(a, FINE_BINS, 0, 1);
+  k_superset<<<(a.NBD + SUP_DB - 1) / SUP_DB, TPB, 0, s>>>(a, w);
+  const uint32_t nsb = (a.sup_cap + SUP_CHUNK - 1) / SUP_CHUNK;
+  const uint32_t nh = nsb < 1024u ? (nsb ? nsb : 1u) : 1024u;
+  k_sup_hist<<<nh, TPB, 0, s>>>(a, 1);
+  k_select_fast<<<1, 256, 0, s>>>(a, 512, 9, 0);
+  k_sup_hist<<<nh, TPB, 0, s>>>(a, 2);
+  k_select_fast<<<1, 256, 0, s>>>(a, 512, 9, 0);
+  k_sup_count<<<nsb ? nsb : 1u, TPB, 0, s>>>(a);
+  k_scan_sup<<<1, 1024, 0, s>>>(a);
+  k_sup_scatter<<<nsb ? nsb : 1u, TPB, 0, s>>>(a, (uint32_t)k0);
+  k_xi0<<<1, 256, 0, s>>>(a);
+}
+
+void mask_build_fast_offsets(const MaskArgs& a, uint64_t k0, cudaStream_t s) {
+  kernel_launches() += 1;
+  k_off_search<<<1, 256, 0, s>>>(a, (uint32_t)k0);
 }
 
 void mask_finish(const MaskArgs& a, cudaStream_t s) {

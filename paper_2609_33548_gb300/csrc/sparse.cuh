@@ -39,11 +39,14 @@ struct MaskArgs {
   float *gamma_minus, *tau_minus, *sw_minus; // [P+2] of w - eps z
   int groups;                   // selection groups: 1 (the global quantile of Eq. 4) or P
                                 // (one per projection: the per-tensor variant)
-  unsigned long long* hist;     // [groups x 2048]
+  unsigned long long* hist;     // [max(groups x 2048, 8192)]
   SelectState* sel;             // [groups]
   unsigned long long* grp_tie0; // [P] ties before the first dense block of each group
   float* xi0p;                  // [P] xi_0 of each projection (Eq. 5)
   uint32_t *blk_a, *blk_b, *blk_c, *blk_d;   // per-block scratch
+  uint32_t sup_cap;             // entries idx[1] / lat[1] hold (the superset of mask_build_fast)
+  unsigned long long* scan_state; // [NBD] decoupled look-back words of the superset compaction
+  uint32_t* sup;                // [4] superset size, overflow flag, block ticket, unused
   unsigned long long* counters; // [0] flipped, [1] jumps, [2] dropped, [3] 32-byte sectors of the packed store rewritten,
                                 // [4] active latents within 1e-5 s_w of +-tau in the +/- passes
   unsigned* err;
@@ -52,6 +55,13 @@ struct MaskArgs {
 // Selects S_0 (the a.groups groups' select states must hold their k) and
 // writes the sparse store, the codes at tau_0 and xi0p.
 void mask_build(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_t s);
+// The global quantile (groups == 1, 0 < k0) in three dense passes.  hist
+// [8192], sup and scan_state must be zero and sel hold k0.  Afterwards sup[1]
+// != 0 means the superset did not fit in idx[1] / lat[1] and nothing but the
+// codes at tau_0 was written (run mask_build instead); otherwise S_0, xi0p
+// and the codes are written and mask_build_fast_offsets writes off[0].
+void mask_build_fast(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_t s);
+void mask_build_fast_offsets(const MaskArgs& a, uint64_t k0, cudaStream_t s);
 void mask_finish(const MaskArgs& a, cudaStream_t s);
 void sparse_pm_taus(const MaskArgs& a, int cur, uint64_t seed, float eps, cudaStream_t s);
 void sparse_requant(const MaskArgs& a, int cur, uint64_t seed, float eps, int sign, cudaStream_t s);

@@ -55,6 +55,7 @@ def test_forward_loss_matrix(name, cache):
     per_o, _ = bitnet.batch_loss(cfg, split, sw, *th, rows=rows)
     ens = rounding.loss_ensemble(cfg, (split, sw), th, n=8, rows=rows)
     for b in rows:
-        # 1e-3, or no further from the oracle than its valid fp32 re-roundings
+        # 1e-3, or no further from the oracle than its valid fp32 re-roundings,
+        # or within 5 standard deviations of them (rounding.agrees)
         record("forward_matrix", workload=name, cache=cache, sequence=b, **rounding.summary(per[b], per_o[b], ens[:, b]))
-        assert rounding.within(per[b], per_o[b], ens[:, b]), (name, b, per[b], per_o[b], ens[:, b])
+        assert rounding.agrees(per[b], per_o[b], ens[:, b]), (name, b, per[b], per_o[b], ens[:, b])

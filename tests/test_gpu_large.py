@@ -19,7 +19,7 @@ configuration bench.py times.
   random-init decoder is determined by its definition only to that spread.
   The comparison is therefore statistical: F+-, g lie within 5 sample
   standard deviations of the mean of the oracle and its re-roundings
-  (rounding.consistent; a false alarm about once in 1000), and every value is
+  (rounding.agrees / rounding.consistent; a false alarm about once in 1000), and every value is
   recorded.  The exact, per-operation parity of these forwards is
   test_gpu_layerwise.py's (bit-exact given the same inputs).  tau+ and tau- of
   every projection are bit-exact.
@@ -169,9 +169,9 @@ def _step_sampled_sequences(cfg, density, rows, name):
                                                                                  ens_p[:, i]),
                F_minus=rounding.summary(out["per_seq_minus"][b], per_m[i], ens_m[:, i]),
                g=rounding.summary(g_gpu, g_ref, g_ens))
-        assert rounding.consistent(out["per_seq_plus"][b], per_p[i], ens_p[:, i]), (b, out["per_seq_plus"][b], per_p[i])
-        assert rounding.consistent(out["per_seq_minus"][b], per_m[i], ens_m[:, i])
-        assert rounding.consistent(g_gpu, g_ref, g_ens), (b, g_gpu, g_ref)
+        assert rounding.agrees(out["per_seq_plus"][b], per_p[i], ens_p[:, i]), (b, out["per_seq_plus"][b], per_p[i])
+        assert rounding.agrees(out["per_seq_minus"][b], per_m[i], ens_m[:, i])
+        assert rounding.agrees(g_gpu, g_ref, g_ens), (b, g_gpu, g_ref)
     assert out["n_jumps"] == 0 and out["k_active"] == act.size
 
 
