@@ -399,12 +399,27 @@ __global__ void __launch_bounds__(TPB) k_sparse_pm_sum(MaskArgs a, int cur, uint
   ExactAcc ap, am;
   ea_zero(ap);
   ea_zero(am);
-  for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) {
-    const float z = normal_at(seed, a.idx[cur][e]);
-    float wp, wm, ee;
-    perturbed(a.lat[cur][e], z, eps, &wp, &wm, &ee);
-    ea_add_abs(ap, wp);
-    ea_add_abs(am, wm);
+  // four weights per iteration: their Philox chains are independent, so they
+  // interleave (the exact sums do not depend on the order of the adds)
+  for (uint32_t e0 = r.beg + threadIdx.x; e0 < r.end; e0 += 4 * TPB) {
+    uint32_t id[4];
+    float wv[4], z[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const uint32_t e = e0 + u * TPB;
+      id[u] = e < r.end ? a.idx[cur][e] : 0u;
+      wv[u] = e < r.end ? a.lat[cur][e] : 0.f;
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) z[u] = normal_at(seed, id[u]);
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+      if (e0 + u * TPB < r.end) {
+        float wp, wm, ee;
+        perturbed(wv[u], z[u], eps, &wp, &wm, &ee);
+        ea_add_abs(ap, wp);
+        ea_add_abs(am, wm);
+      }
   }
   ExactSum sp = ea_result(ap), sm = ea_result(am);
   es_block_reduce(sp, red);
@@ -532,20 +547,47 @@ __global__ void __launch_bounds__(TPB) k_sparse_update(MaskArgs a, int cur, Upda
   const uint64_t last = KM == 1 ? d.seed[0] : d.last;
   ExactAcc acc;
   ea_zero(acc);
-  for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) {
-    const uint32_t i = a.idx[cur][e];
-    const float zl = normal_at(last, i);
-    float wp, wm, ee;
-    perturbed(a.lat[cur][e], zl, eps, &wp, &wm, &ee);
-    float wn = __fadd_rn(wm, ee);
+  if (KM == 1) {
+    // four weights per iteration (independent Philox chains interleave)
+    for (uint32_t e0 = r.beg + threadIdx.x; e0 < r.end; e0 += 4 * TPB) {
+      uint32_t id[4];
+      float wv[4], zl[4];
 #pragma unroll
-    for (int k = 0; k < KM; ++k)
-      if (k < d.K) {
-        const float z = (KM == 1 || k == d.K - 1) ? zl : normal_at(d.seed[k], i);
-        wn = __fsub_rn(wn, __fmul_rn(c[k], z));
+      for (int u = 0; u < 4; ++u) {
+        const uint32_t e = e0 + u * TPB;
+        id[u] = e < r.end ? a.idx[cur][e] : 0u;
+        wv[u] = e < r.end ? a.lat[cur][e] : 0.f;
       }
-    a.lat[cur][e] = wn;
-    ea_add_abs(acc, wn);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) zl[u] = normal_at(last, id[u]);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const uint32_t e = e0 + u * TPB;
+        if (e < r.end) {
+          float wp, wm, ee;
+          perturbed(wv[u], zl[u], eps, &wp, &wm, &ee);
+          const float wn = __fsub_rn(__fadd_rn(wm, ee), __fmul_rn(c[0], zl[u]));
+          a.lat[cur][e] = wn;
+          ea_add_abs(acc, wn);
+        }
+      }
+    }
+  } else {
+    for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) {
+      const uint32_t i = a.idx[cur][e];
+      const float zl = normal_at(last, i);
+      float wp, wm, ee;
+      perturbed(a.lat[cur][e], zl, eps, &wp, &wm, &ee);
+      float wn = __fadd_rn(wm, ee);
+#pragma unroll
+      for (int k = 0; k < KM; ++k)
+        if (k < d.K) {
+          const float z = (k == d.K - 1) ? zl : normal_at(d.seed[k], i);
+          wn = __fsub_rn(wn, __fmul_rn(c[k], z));
+        }
+      a.lat[cur][e] = wn;
+      ea_add_abs(acc, wn);
+    }
   }
   ExactSum s = ea_result(acc);
   es_block_reduce(s, red);
@@ -697,6 +739,11 @@ constexpr int SUP_STAGE = 4096;                // superset entries a CTA stages 
 
 // Pass 1 of the fast build: the exact sum of |w| of each dense block, one
 // warp per block (float4 number q * 32 + lane for q < 32, no CTA barrier).
+// For |w| in [2^-31, 2) (biased exponent e in [96, 128)) m << (e - 96) < 2^56
+// is accumulated in one uint64 (128 values per lane: < 2^63); it is bucket 1
+// of the ExactSum shifted by 32 (bucket 1 holds m << (e - 64) for e in
+// [64, 128)), so the buckets hold the same integers as es_add_abs would put
+// there.  Other values take ea_add_abs.
 __global__ void __launch_bounds__(TPB) k_dense_sum_warp(MaskArgs a, const float* __restrict__ w) {
   const int lane = threadIdx.x & 31;
   const uint32_t b = blockIdx.x * (TPB / 32) + (threadIdx.x >> 5);
@@ -704,21 +751,32 @@ __global__ void __launch_bounds__(TPB) k_dense_sum_warp(MaskArgs a, const float*
   const DenseRange r = dense_range(a, b);
   ExactAcc acc;
   ea_zero(acc);
+  uint64_t fx = 0;
+  auto add = [&](float v) {
+    const uint32_t bits = __float_as_uint(v) & 0x7FFFFFFFu;
+    const uint32_t sh = (bits >> 23) - 96u;
+    if (sh < 32u)
+      fx += (uint64_t)((bits & 0x7FFFFFu) | 0x800000u) << sh;
+    else
+      ea_add_abs(acc, v);
+  };
 #pragma unroll 8
   for (int q = 0; q < (int)(DENSE_CHUNK / 128); ++q) {
     const uint64_t i = r.start + 4ull * (q * 32 + lane);
     if (i < r.end) {
       const float4 t = *reinterpret_cast<const float4*>(w + i);
-      ea_add_abs(acc, t.x);
-      ea_add_abs(acc, t.y);
-      ea_add_abs(acc, t.z);
-      ea_add_abs(acc, t.w);
+      add(t.x);
+      add(t.y);
+      add(t.z);
+      add(t.w);
     }
   }
   ExactSum s = ea_result(acc);
+  s.b[1] += (u128)fx << 32;
   es_warp_reduce(s);
   if (lane == 0) a.partials[b] = s;
 }
+
 constexpr int FINE_BINS = 1 << (31 - FINE_SHIFT);
 constexpr uint32_t SUP_CHUNK = 4096;           // superset entries per block of the resolution kernels
 
@@ -885,87 +943,105 @@ __device__ unsigned long long lookback_prefix(const MaskArgs& a, uint32_t b, uin
 
 // Pass 3: every weight whose fine bin is at most the k0-th key's, in index
 // order, into idx[1] / lat[1].  A CTA takes SUP_DB consecutive dense blocks
-// (in ticket order), finds its selected weights and their order (one block
-// scan per float4 column of each block: index order is block-major, then
-// q-major), stages them in shared memory, gets its global offset by the
-// look-back and copies them out.  More than SUP_STAGE selected weights (a
-// dense mask): the CTA reads its blocks again and writes directly.
-__device__ __forceinline__ void superset_block(const MaskArgs& a, const float* __restrict__ w, uint32_t b,
-                                               uint32_t bmax, uint32_t* sh, uint32_t& run, bool stage,
-                                               uint32_t* st_idx, float* st_lat, unsigned long long gbase) {
+// (in ticket order), one per warp.  A warp walks its block in index order
+// (float4 number q * 32 + lane, q-major), ranks its selected weights with warp
+// scans and stages them in its share of shared memory; one barrier gives the
+// warps their offsets, the look-back the CTA's global offset, and the warps
+// copy their weights out.  A warp with more than its share (a dense mask)
+// makes the CTA read its blocks again and write directly.
+constexpr int SUP_WSTAGE = SUP_STAGE / (TPB / 32);  // staged entries per warp
+
+// One warp's dense block b: the selected weights in index order, staged
+// (stage) or written at out0 + their rank (!stage).  Returns the count.
+__device__ __forceinline__ uint32_t superset_warp(const MaskArgs& a, const float* __restrict__ w, uint32_t b,
+                                                  uint32_t bmax, int lane, bool stage, uint32_t* st_idx,
+                                                  float* st_lat, unsigned long long out0) {
   const DenseRange r = dense_range(a, b);
   const float tau = a.tau_cur[r.proj];
-  float4 t[4];
-  uint32_t mask = 0, cnt[4];
+  uint32_t run = 0;
+  for (int q0 = 0; q0 < (int)(DENSE_CHUNK / 128); q0 += 8) {
+    float4 t[8];
 #pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const uint64_t i = r.start + 4ull * (q * TPB + threadIdx.x);
-    t[q] = i < r.end ? *reinterpret_cast<const float4*>(w + i) : make_float4(0.f, 0.f, 0.f, 0.f);
-  }
+    for (int u = 0; u < 8; ++u) {
+      const uint64_t i = r.start + 4ull * ((q0 + u) * 32 + lane);
+      t[u] = i < r.end ? *reinterpret_cast<const float4*>(w + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
 #pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const uint64_t i = r.start + 4ull * (q * TPB + threadIdx.x);
-    cnt[q] = 0;
-    if (i < r.end) {
-      const float vv[4] = {t[q].x, t[q].y, t[q].z, t[q].w};
+    for (int u = 0; u < 8; ++u) {
+      const uint64_t i = r.start + 4ull * ((q0 + u) * 32 + lane);
+      const float vv[4] = {t[u].x, t[u].y, t[u].z, t[u].w};
+      uint32_t m = 0;
+      if (i < r.end) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) m |= ((dist_key(vv[e], tau) >> FINE_SHIFT) <= bmax ? 1u : 0u) << e;
+      }
+      const uint32_t cnt = __popc(m);
+      uint32_t incl = cnt;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      uint32_t pos = run + incl - cnt;
 #pragma unroll
       for (int e = 0; e < 4; ++e)
-        if ((dist_key(vv[e], tau) >> FINE_SHIFT) <= bmax) { mask |= 1u << (4 * q + e); ++cnt[q]; }
+        if (m & (1u << e)) {
+          if (stage) {
+            if (pos < SUP_WSTAGE) {
+              st_idx[pos] = (uint32_t)i + e;
+              st_lat[pos] = vv[e];
+            }
+          } else if (out0 + pos < a.sup_cap) {  // cannot fail: the size was checked against the capacity
+            a.idx[1][out0 + pos] = (uint32_t)i + e;
+            a.lat[1][out0 + pos] = vv[e];
+          }
+          ++pos;
+        }
+      run += __shfl_sync(0xffffffffu, incl, 31);
     }
   }
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    uint32_t tot;
-    uint32_t pos = run + block_excl_scan(cnt[q], sh, &tot);
-    const uint32_t i = (uint32_t)(r.start + 4ull * (q * TPB + threadIdx.x));
-    const float vv[4] = {t[q].x, t[q].y, t[q].z, t[q].w};
-#pragma unroll
-    for (int e = 0; e < 4; ++e)
-      if (mask & (1u << (4 * q + e))) {
-        if (stage) {
-          if (pos < SUP_STAGE) {
-            st_idx[pos] = i + e;
-            st_lat[pos] = vv[e];
-          }
-        } else if (gbase + pos < a.sup_cap) {  // cannot fail: the size was checked against the capacity
-          a.idx[1][gbase + pos] = i + e;
-          a.lat[1][gbase + pos] = vv[e];
-        }
-        ++pos;
-      }
-    run += tot;
-  }
+  return run;
 }
 
 __global__ void __launch_bounds__(TPB) k_superset(MaskArgs a, const float* __restrict__ w) {
-  __shared__ uint32_t sh[TPB / 32];
   __shared__ uint32_t s_bid;
   __shared__ unsigned long long s_excl;
+  __shared__ uint32_t s_wcnt[TPB / 32];
   __shared__ uint32_t st_idx[SUP_STAGE];
   __shared__ float st_lat[SUP_STAGE];
   if (a.sup[1]) return;  // the superset does not fit: the host runs the six-pass build
   if (threadIdx.x == 0) s_bid = atomicAdd(&a.sup[2], 1u);
   __syncthreads();
   const uint32_t c = s_bid;
-  const uint32_t b0 = c * SUP_DB, b1 = min(a.NBD, b0 + SUP_DB);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t b = c * SUP_DB + warp;
   const uint32_t bmax = a.sel->prefix;
-  uint32_t run = 0;  // selected weights of this CTA so far (the same in every thread)
-  for (uint32_t b = b0; b < b1; ++b) superset_block(a, w, b, bmax, sh, run, true, st_idx, st_lat, 0);
-  if (threadIdx.x < 32) {
-    const unsigned long long e = lookback_prefix(a, c, run, threadIdx.x);
-    if (threadIdx.x == 0) s_excl = e;
+  uint32_t* my_idx = st_idx + warp * SUP_WSTAGE;
+  float* my_lat = st_lat + warp * SUP_WSTAGE;
+  const uint32_t n = b < a.NBD ? superset_warp(a, w, b, bmax, lane, true, my_idx, my_lat, 0) : 0u;
+  if (lane == 0) s_wcnt[warp] = n;
+  __syncthreads();
+  uint32_t woff = 0, total = 0;
+  bool fits = true;
+  for (int k = 0; k < TPB / 32; ++k) {
+    if (k < warp) woff += s_wcnt[k];
+    total += s_wcnt[k];
+    fits = fits && s_wcnt[k] <= SUP_WSTAGE;
+  }
+  if (warp == 0) {
+    const unsigned long long e = lookback_prefix(a, c, total, lane);
+    if (lane == 0) s_excl = e;
   }
   __syncthreads();
-  const unsigned long long base = s_excl;
-  if (run <= SUP_STAGE) {
-    for (uint32_t j = threadIdx.x; j < run; j += TPB)
+  const unsigned long long base = s_excl + woff;
+  if (fits) {
+    for (uint32_t j = lane; j < n; j += 32)
       if (base + j < a.sup_cap) {
-        a.idx[1][base + j] = st_idx[j];
-        a.lat[1][base + j] = st_lat[j];
+        a.idx[1][base + j] = my_idx[j];
+        a.lat[1][base + j] = my_lat[j];
       }
-  } else {
-    uint32_t run2 = 0;
-    for (uint32_t b = b0; b < b1; ++b) superset_block(a, w, b, bmax, sh, run2, false, st_idx, st_lat, base);
+  } else if (b < a.NBD) {
+    superset_warp(a, w, b, bmax, lane, false, my_idx, my_lat, base);
   }
 }
 
