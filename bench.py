@@ -51,12 +51,13 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # dense passes over the latents that termezo_build_mask's kernels make
 # (absmean, three radix-histogram passes, count, compaction)
 MASK_BUILD_DENSE_PASSES = 6
-# DRAM bytes (read + write) per k_bitlinear_gemm launch, the mean over the 240
-# GEMM launches of one 2B-shaped step, from the one-pass ncu launch list in
-# profiles/step_2b_launch_list.md.  It describes the kernel source with this
-# SHA-1 only; any other source, or another workload, reports null.
+# DRAM bytes (read + write) per k_bitlinear_gemm launch, the mean over eight
+# consecutive GEMM launches (two layers, every shape twice) of the 2B-shaped
+# step, from a one-pass ncu capture (profiles/k_bitlinear_gemm_2b_step_dram.md).
+# It describes the kernel source with this SHA-1 only; any other source, or
+# another workload, reports null.
 GEMM_TRAFFIC = {"workload": "2b", "source": "paper_2609_33548_gb300/csrc/gemm.cu",
-                "sha1": "4c962ad660ddb05afece1b02f6bceecda002c227", "bytes_per_launch": 206.5e6}
+                "sha1": "4c962ad660ddb05afece1b02f6bceecda002c227", "bytes_per_launch": 208.0e6}
 
 
 def gemm_traffic(workload):
