@@ -215,21 +215,21 @@ class OracleSample:
         return est, t_rq, t_fw
 
 
-def memory_report(cfg, density, peak_bytes, weight_cache=False):
+def memory_report(cfg, density, peak_bytes, weight_cache=False, z_cache=False):
     """Device bytes by part (termezo_memory) next to the memory equation of
     Sec. 5 evaluated with this build's precisions (B = 4 fp32 latents,
     B_Q = 1/4, 32-bit active indices), and the peak torch allocation over the
     timed steps (workspace + theta + batches).  The e4m3 weight cache, when
     on, is its own part (d bytes, outside the equation)."""
     from paper_2609_33548_gb300 import termezo as tz
-    m = tz.termezo_memory(tz.make_cfg(cfg, weight_cache), density)
+    m = tz.termezo_memory(tz.make_cfg(cfg, weight_cache, z_cache), density)
     d, k0 = m["d"], m["k_cap"]
     B, BQ = 4, 0.25
     eq_latent = d * B - math.ceil(d * (1 - density) * (B - BQ)) + math.ceil(density * d * BQ) + math.ceil(k0 * 4)
     gb = 1e9
     return {"workspace_gb": m["workspace"] / gb, "packed_codes_gb": m["packed"] / gb,
             "sparse_store_gb": (m["sparse_index"] + m["sparse_latents"]) / gb, "forward_gb": m["forward"] / gb,
-            "theta_gb": m["theta"] / gb, "weight_cache_gb": m["weight_cache"] / gb,
+            "theta_gb": m["theta"] / gb, "weight_cache_gb": m["weight_cache"] / gb, "z_cache_gb": m["z_cache"] / gb,
             "peak_allocated_gb": peak_bytes / gb,
             "latents": {"mezo_fp32_gb": d * B / gb, "equation_gb": eq_latent / gb,
                         "build_gb": (m["packed"] + m["sparse_index"] + m["sparse_latents"]) / gb,
@@ -291,7 +291,7 @@ def run_mine(args):
     emb, gains, head = synth.theta(cfg, device=dev)
     nb = args.warmup + args.steps
     batches = [synth.batch(cfg, device=dev, step=i) for i in range(nb)]
-    ctx = tz.Context(tz.make_cfg(cfg, args.weight_cache), density, device=dev)
+    ctx = tz.Context(tz.make_cfg(cfg, args.weight_cache, args.z_cache), density, device=dev)
     ctx.termezo_load_params(w, emb, gains, head)
     stream = torch.cuda.current_stream()
 
@@ -413,7 +413,7 @@ def run_mine(args):
                    "parallelism": f"replicas{world}", "layers": cfg.layers, "hidden": cfg.hidden,
                    "density": density, "k_active": int(outs[-1]["k_active"]), "eps": EPS, "lr": LR,
                    "directions": K, "theta_trained": bool(args.theta),
-                   "weight_cache": bool(args.weight_cache),
+                   "weight_cache": bool(args.weight_cache), "z_cache": bool(args.z_cache),
                    "l2": "no flush: per-step working set (521 MB packed codes, >1 GB activations) exceeds L2"},
         "steps_per_s": world * args.steps / (ms_max / 1e3),
         "roofline": {"bound": "tensor",
@@ -439,7 +439,7 @@ def run_mine(args):
                                    "(index + latent per active weight, 64 B per rewritten 32-byte sector of the "
                                    "packed store, 4 B per updated latent); mask build 3 dense reads + codes + S_0")},
         "e2e": {"value": tokens / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-        "memory": memory_report(cfg, density, torch.cuda.max_memory_allocated(dev), args.weight_cache),
+        "memory": memory_report(cfg, density, torch.cuda.max_memory_allocated(dev), args.weight_cache, args.z_cache),
         "gpu_launches": int(prof["launches"]),
         "clocks": clocks,
         "last_step": {k: outs[-1][k] for k in ("loss_plus", "loss_minus", "g", "k_active", "n_flipped", "n_jumps",
@@ -471,7 +471,7 @@ def run_op(args):
     w = synth.op_latents(N, K, device=dev).reshape(-1)
     x = synth.op_activations(M, K, device=dev)
     y = torch.empty(M, N, dtype=torch.float32, device=dev)
-    ctx = tz.Context(tz.op_cfg(N, K, M), density, device=dev)
+    ctx = tz.Context(tz.op_cfg(N, K, M, args.z_cache), density, device=dev)
     ctx.termezo_load_params(w)
     k0, _ = ctx.termezo_build_mask(density)
 
@@ -575,6 +575,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--weight-cache", action="store_true",
                     help="keep an e4m3 copy of the codes (d bytes) instead of expanding them before every GEMM")
+    ap.add_argument("--z-cache", action="store_true",
+                    help="keep z of the active weights (4 B each) between the passes of a direction instead of "
+                         "regenerating it")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -56,12 +56,19 @@ typedef struct termezo_ctx termezo_ctx;
  * 2-bit store by every call that rewrites codes, and the forward's GEMMs read
  * it directly instead of expanding the packed codes of each projection
  * before its GEMM.  It trades d bytes of device memory (not part of the
- * paper's memory equation) for the expansion work.  Ignored for layers == 0. */
+ * paper's memory equation) for the expansion work.  Ignored for layers == 0.
+ * z_cache != 0: the workspace also holds one float per active weight (the
+ * sparse store's capacity, 4 k bytes, not part of the paper's memory
+ * equation): the perturbation sums of a direction write z there in store
+ * order and the requantisations, the restore and the update of the same
+ * direction read it instead of regenerating z by Philox (the values are the
+ * same).  0: every pass regenerates z (Algorithm 1 draws z from the seed). */
 typedef struct {
   int32_t layers, hidden, heads, kv_heads, ffn, vocab, seq, batch;
   int32_t loss_mode;
   int32_t n_labels;
   int32_t weight_cache;
+  int32_t z_cache;
 } termezo_model_cfg;
 
 /* Per-step report (Algorithm 1 with K = 1; counters of Eq. 11). */
@@ -103,6 +110,7 @@ typedef struct {
   uint64_t mask_bitmask;    /* the paper's dense bit-mask option, ceil(d / 8) */
   uint64_t mask_index_list; /* the paper's index-list option, ceil(rho_0 d ceil(log2 d) / 8) */
   uint64_t weight_cache;    /* e4m3 copy of the codes (weight_cache != 0), d bytes; else 0 */
+  uint64_t z_cache;         /* z of the active weights (z_cache != 0), 4 k_cap bytes; else 0 */
 } termezo_memory_out;
 
 int termezo_memory(const termezo_model_cfg* cfg, double density, termezo_memory_out* out);

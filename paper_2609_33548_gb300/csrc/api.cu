@@ -23,6 +23,7 @@ constexpr uint32_t SPARSE_CHUNK = 4096;
 struct Shape {
   bool op;
   bool wcache;  // e4m3 weight cache (decoder contexts)
+  bool zcache;  // z of the active weights kept between the passes of a direction
   int L, D, H, KV, hd, F, V, S, B, T, C, mode;
   int P;
   std::vector<uint64_t> base;  // [P+1]
@@ -34,6 +35,7 @@ int make_shape(const termezo_model_cfg* c, Shape* s) {
   if (!c) return TERMEZO_EINVAL;
   s->op = c->layers == 0;
   s->wcache = !s->op && c->weight_cache != 0;
+  s->zcache = c->z_cache != 0;
   s->L = c->layers;
   s->D = c->hidden;
   s->F = c->ffn;
@@ -87,7 +89,7 @@ uint64_t keep_count(double density, uint64_t d) { return (uint64_t)std::floor(de
 enum { PASS_PM = 0, PASS_REQUANT = 1, PASS_UPDATE = 2, PASS_SHRINK = 3, PASS_THETA = 4 };
 static_assert(PASS_THETA + 1 == TERMEZO_PASS_KINDS, "pass kinds");
 
-enum Section { SEC_PACKED, SEC_INDEX, SEC_LATENTS, SEC_MASK, SEC_FORWARD, SEC_WCACHE, SEC_COUNT };
+enum Section { SEC_PACKED, SEC_INDEX, SEC_LATENTS, SEC_MASK, SEC_FORWARD, SEC_WCACHE, SEC_ZCACHE, SEC_COUNT };
 
 struct Carver {
   uint8_t* base;
@@ -259,6 +261,11 @@ void carve(termezo_ctx* c, Carver& cv) {
       a.sup_cap = (uint32_t)(room < 0xFFFFFFFFull ? room : 0xFFFFFFFFull);
     }
     a.off[i] = cv.take<uint32_t>(P + 1);
+  }
+  if (s.zcache) {
+    cv.sec = SEC_ZCACHE;
+    a.zbuf = cv.take<float>(c->k_cap);
+    cv.sec = SEC_MASK;
   }
   a.S_total = cv.take<ExactSum>(P);
   a.A_frozen = cv.take<ExactSum>(P);
@@ -563,6 +570,12 @@ int run_forward(termezo_ctx* c, const int32_t* tokens, const int32_t* targets, c
   return cuda_status(c);
 }
 
+// The z buffer holds the z of `seed` in the current store order (written by
+// the perturbation sums of that seed since the last shrink or update).
+bool z_ready(const termezo_ctx* c, uint64_t seed) {
+  return c->ma.zbuf && c->pm_valid && c->pm_seed == seed;
+}
+
 void ensure_pm(termezo_ctx* c, uint64_t seed, float eps) {
   if (c->pm_valid && c->pm_seed == seed && c->pm_eps == eps) return;
   tmz::sparse_pm_taus(c->ma, c->cur, seed, eps, c->stream);
@@ -612,6 +625,7 @@ int termezo_memory(const termezo_model_cfg* cfg, double density, termezo_memory_
   out->mask_state = cv.bytes[SEC_MASK];
   out->forward = cv.bytes[SEC_FORWARD];
   out->weight_cache = cv.bytes[SEC_WCACHE];
+  out->z_cache = cv.bytes[SEC_ZCACHE];
   out->workspace = cv.off + 256;
   out->theta = s.op ? 0
                     : (uint64_t)s.V * s.D * 4 + (uint64_t)(2 * s.L + 1) * s.D * 4 + (uint64_t)s.V * s.D * 2;
@@ -843,7 +857,7 @@ int termezo_forward_loss(termezo_ctx* c, const int32_t* d_tokens, const int32_t*
                          double* per_seq) {
   if (!c || !d_tokens || !d_targets) return TERMEZO_EINVAL;
   if (c->sh.op || !c->built) return TERMEZO_ESTATE;
-  tmz::sparse_requant(c->ma, c->cur, 0, 0.f, 0, c->stream);
+  tmz::sparse_requant(c->ma, c->cur, 0, 0.f, 0, false, c->stream);
   c->code_sw = c->ma.sw_cur;
   int rc = run_forward(c, d_tokens, d_targets, c->ma.sw_cur, 0);
   if (rc) return rc;
@@ -929,7 +943,7 @@ int step_impl(termezo_ctx* c, const uint64_t* seeds, int K, float eps, float lr,
     }
     {
       ProfScope ps(c, 2 + PASS_REQUANT, k8);
-      tmz::sparse_requant(c->ma, c->cur, seed, eps, +1, st);
+      tmz::sparse_requant(c->ma, c->cur, seed, eps, +1, z_ready(c, seed), st);
     }
     if (theta) {
       ProfScope ps(c, 2 + PASS_THETA, theta8);
@@ -939,7 +953,7 @@ int step_impl(termezo_ctx* c, const uint64_t* seeds, int K, float eps, float lr,
     if (rc) return rc;
     {
       ProfScope ps(c, 2 + PASS_REQUANT, k8);
-      tmz::sparse_requant(c->ma, c->cur, seed, eps, -1, st);
+      tmz::sparse_requant(c->ma, c->cur, seed, eps, -1, z_ready(c, seed), st);
     }
     if (theta) {
       ProfScope ps(c, 2 + PASS_THETA, theta8);
@@ -952,7 +966,7 @@ int step_impl(termezo_ctx* c, const uint64_t* seeds, int K, float eps, float lr,
     if (K > 1) cudaMemcpyAsync(c->lossk + 2 * k, c->loss, 2 * sizeof(double), cudaMemcpyDeviceToDevice, st);
     if (k + 1 < K) {
       ProfScope ps(c, 2 + PASS_UPDATE, 1.5 * k8);
-      tmz::sparse_restore(c->ma, c->cur, seed, eps, st);
+      tmz::sparse_restore(c->ma, c->cur, seed, eps, z_ready(c, seed), st);
       c->pm_valid = false;
       if (theta) tmz::theta_pm(th, seed, eps, 0, st);
     }
@@ -960,7 +974,7 @@ int step_impl(termezo_ctx* c, const uint64_t* seeds, int K, float eps, float lr,
   dirs.last = seeds[K - 1];
   {
     ProfScope ps(c, 2 + PASS_UPDATE, 1.5 * k8);
-    tmz::sparse_update_dirs(c->ma, c->cur, dirs, eps, lr, c->g, st);
+    tmz::sparse_update_dirs(c->ma, c->cur, dirs, eps, lr, c->g, z_ready(c, dirs.last), st);
   }
   if (theta) {
     ProfScope ps(c, 2 + PASS_THETA, theta8);
@@ -1052,7 +1066,7 @@ int termezo_requantize(termezo_ctx* c, uint64_t seed, float eps, int sign) {
     if (!(eps > 0.f)) return TERMEZO_EINVAL;
     ensure_pm(c, seed, eps);
   }
-  tmz::sparse_requant(c->ma, c->cur, seed, eps, sign, c->stream);
+  tmz::sparse_requant(c->ma, c->cur, seed, eps, sign, sign != 0 && z_ready(c, seed), c->stream);
   c->code_sw = sign > 0 ? c->ma.sw_plus : (sign < 0 ? c->ma.sw_minus : c->ma.sw_cur);
   return cuda_status(c);
 }
@@ -1061,7 +1075,7 @@ int termezo_update(termezo_ctx* c, uint64_t seed, float eps, float lr, double g)
   if (!c) return TERMEZO_EINVAL;
   if (!c->built) return TERMEZO_ESTATE;
   if (!(eps > 0.f) || !std::isfinite(lr) || !std::isfinite(g)) return TERMEZO_EINVAL;
-  tmz::sparse_update(c->ma, c->cur, seed, eps, lr, nullptr, g, 1, c->stream);
+  tmz::sparse_update(c->ma, c->cur, seed, eps, lr, nullptr, g, 1, z_ready(c, seed), c->stream);
   c->updated = true;
   c->pm_valid = false;
   c->t += 1;

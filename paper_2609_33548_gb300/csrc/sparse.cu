@@ -415,6 +415,7 @@ __global__ void __launch_bounds__(TPB) k_sparse_pm_sum(MaskArgs a, int cur, uint
 #pragma unroll
     for (int u = 0; u < 4; ++u)
       if (e0 + u * TPB < r.end) {
+        if (a.zbuf) a.zbuf[e0 + u * TPB] = z[u];
         float wp, wm, ee;
         perturbed(wv[u], z[u], eps, &wp, &wm, &ee);
         ea_add_abs(ap, wp);
@@ -436,22 +437,29 @@ __global__ void __launch_bounds__(TPB) k_sparse_pm_sum(MaskArgs a, int cur, uint
 // write that word, so no two threads write the same word.
 constexpr uint32_t RQ_MAX = 4096;  // elements per sparse block (see the host's block plan)
 
+// z of active weight e (global index i): from the z buffer (use_z) or regenerated.
+__device__ __forceinline__ float z_of(const MaskArgs& a, bool use_z, uint64_t seed, uint32_t e, uint32_t i) {
+  return use_z ? a.zbuf[e] : normal_at(seed, i);
+}
+
 __device__ __forceinline__ float requant_codes(const MaskArgs& a, int sign, uint64_t seed, float eps, float tau,
-                                               float taup, uint32_t i, float w, uint32_t* code, uint32_t* code_p) {
+                                               float taup, uint32_t i, uint32_t e, bool use_z, float w,
+                                               uint32_t* code, uint32_t* code_p) {
   if (sign == 0) {
     *code = ternary_code(w, tau);
     *code_p = *code;
     return w;
   }
   float wp, wm, ee;
-  perturbed(w, normal_at(seed, i), eps, &wp, &wm, &ee);
+  perturbed(w, z_of(a, use_z, seed, e, i), eps, &wp, &wm, &ee);
   const float ws = sign > 0 ? wp : wm;
   *code = ternary_code(ws, tau);
   *code_p = ternary_code(wp, taup);
   return ws;  // the latent this pass quantises
 }
 
-__global__ void __launch_bounds__(TPB) k_sparse_requant(MaskArgs a, int cur, uint64_t seed, float eps, int sign) {
+__global__ void __launch_bounds__(TPB) k_sparse_requant(MaskArgs a, int cur, uint64_t seed, float eps, int sign,
+                                                        bool use_z) {
   __shared__ uint8_t sc[RQ_MAX];
   __shared__ unsigned long long cnt[4];
   if (threadIdx.x < 4) cnt[threadIdx.x] = 0;
@@ -480,7 +488,8 @@ __global__ void __launch_bounds__(TPB) k_sparse_requant(MaskArgs a, int cur, uin
       const uint32_t j = j0 + u * TPB;
       if (j < n) {
         uint32_t c, cp;
-        const float ws = requant_codes(a, sign, seed, eps, tau, taup, idx[r.beg + j], lat[r.beg + j], &c, &cp);
+        const float ws =
+            requant_codes(a, sign, seed, eps, tau, taup, idx[r.beg + j], r.beg + j, use_z, lat[r.beg + j], &c, &cp);
         near += boundary_distance(ws, tau) < near_thr;
         sc[j] = (uint8_t)(c | (cp << 2));
         if (a.wbyte) a.wbyte[idx[r.beg + j]] = code_e4m3(c);
@@ -505,7 +514,7 @@ __global__ void __launch_bounds__(TPB) k_sparse_requant(MaskArgs a, int cur, uin
         code = v & 3u;
         cp = v >> 2;
       } else {  // follower in the next block's range
-        requant_codes(a, sign, seed, eps, tau, taup, i2, lat[e2], &code, &cp);
+        requant_codes(a, sign, seed, eps, tau, taup, i2, e2, use_z, lat[e2], &code, &cp);
       }
       if (sign < 0) {
         flips += cp != code;
@@ -537,7 +546,7 @@ __global__ void __launch_bounds__(TPB) k_sparse_requant(MaskArgs a, int cur, uin
 // exact per-block sums of |w| of the result (the next tau).
 template <int KM>
 __global__ void __launch_bounds__(TPB) k_sparse_update(MaskArgs a, int cur, UpdateDirs d, float eps, float lr,
-                                                       const double* g_dev, double g_host, int use_host) {
+                                                       const double* g_dev, double g_host, int use_host, bool use_z) {
   __shared__ ExactSum red[TPB / 32];
   const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
   const double lr_k = (double)lr / (double)d.K;
@@ -559,7 +568,7 @@ __global__ void __launch_bounds__(TPB) k_sparse_update(MaskArgs a, int cur, Upda
         wv[u] = e < r.end ? a.lat[cur][e] : 0.f;
       }
 #pragma unroll
-      for (int u = 0; u < 4; ++u) zl[u] = normal_at(last, id[u]);
+      for (int u = 0; u < 4; ++u) zl[u] = (use_z && e0 + u * TPB < r.end) ? a.zbuf[e0 + u * TPB] : normal_at(last, id[u]);
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
         const uint32_t e = e0 + u * TPB;
@@ -575,7 +584,7 @@ __global__ void __launch_bounds__(TPB) k_sparse_update(MaskArgs a, int cur, Upda
   } else {
     for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) {
       const uint32_t i = a.idx[cur][e];
-      const float zl = normal_at(last, i);
+      const float zl = z_of(a, use_z, last, e, i);
       float wp, wm, ee;
       perturbed(a.lat[cur][e], zl, eps, &wp, &wm, &ee);
       float wn = __fadd_rn(wm, ee);
@@ -595,11 +604,11 @@ __global__ void __launch_bounds__(TPB) k_sparse_update(MaskArgs a, int cur, Upda
 }
 
 // Algorithm 1's restore after a direction that is not the last one.
-__global__ void __launch_bounds__(TPB) k_sparse_restore(MaskArgs a, int cur, uint64_t seed, float eps) {
+__global__ void __launch_bounds__(TPB) k_sparse_restore(MaskArgs a, int cur, uint64_t seed, float eps, bool use_z) {
   const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
   for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) {
     float wp, wm, ee;
-    perturbed(a.lat[cur][e], normal_at(seed, a.idx[cur][e]), eps, &wp, &wm, &ee);
+    perturbed(a.lat[cur][e], use_z ? a.zbuf[e] : normal_at(seed, a.idx[cur][e]), eps, &wp, &wm, &ee);
     a.lat[cur][e] = __fadd_rn(wm, ee);
   }
 }
@@ -1230,36 +1239,37 @@ void sparse_pm_taus(const MaskArgs& a, int cur, uint64_t seed, float eps, cudaSt
                                     a.tau_minus, a.sw_minus);
 }
 
-void sparse_requant(const MaskArgs& a, int cur, uint64_t seed, float eps, int sign, cudaStream_t s) {
+void sparse_requant(const MaskArgs& a, int cur, uint64_t seed, float eps, int sign, bool use_z, cudaStream_t s) {
   kernel_launches() += 1;
-  k_sparse_requant<<<a.NBS, TPB, 0, s>>>(a, cur, seed, eps, sign);
+  k_sparse_requant<<<a.NBS, TPB, 0, s>>>(a, cur, seed, eps, sign, use_z && a.zbuf);
 }
 
 void sparse_update(const MaskArgs& a, int cur, uint64_t seed, float eps, float lr, const double* g_dev, double g_host,
-                   int use_host, cudaStream_t s) {
+                   int use_host, bool use_z, cudaStream_t s) {
   kernel_launches() += 2;
   UpdateDirs d{};
   d.seed[0] = d.last = seed;
   d.K = 1;
-  k_sparse_update<1><<<a.NBS, TPB, 0, s>>>(a, cur, d, eps, lr, g_dev, g_host, use_host);
+  k_sparse_update<1><<<a.NBS, TPB, 0, s>>>(a, cur, d, eps, lr, g_dev, g_host, use_host, use_z && a.zbuf);
   k_reduce_proj<<<a.P, TPB, 0, s>>>(a.partials, a.spre, 1, 0, a.A_frozen, a.base, nullptr, a.gamma_cur, a.tau_cur,
                                     a.sw_cur);
 }
 
 void sparse_update_dirs(const MaskArgs& a, int cur, const UpdateDirs& d, float eps, float lr, const double* g_dev,
-                        cudaStream_t s) {
+                        bool use_z, cudaStream_t s) {
+  use_z = use_z && a.zbuf;
   kernel_launches() += 2;
   if (d.K == 1)
-    k_sparse_update<1><<<a.NBS, TPB, 0, s>>>(a, cur, d, eps, lr, g_dev, 0.0, 0);
+    k_sparse_update<1><<<a.NBS, TPB, 0, s>>>(a, cur, d, eps, lr, g_dev, 0.0, 0, use_z);
   else
-    k_sparse_update<KMAX><<<a.NBS, TPB, 0, s>>>(a, cur, d, eps, lr, g_dev, 0.0, 0);
+    k_sparse_update<KMAX><<<a.NBS, TPB, 0, s>>>(a, cur, d, eps, lr, g_dev, 0.0, 0, use_z);
   k_reduce_proj<<<a.P, TPB, 0, s>>>(a.partials, a.spre, 1, 0, a.A_frozen, a.base, nullptr, a.gamma_cur, a.tau_cur,
                                     a.sw_cur);
 }
 
-void sparse_restore(const MaskArgs& a, int cur, uint64_t seed, float eps, cudaStream_t s) {
+void sparse_restore(const MaskArgs& a, int cur, uint64_t seed, float eps, bool use_z, cudaStream_t s) {
   kernel_launches() += 1;
-  k_sparse_restore<<<a.NBS, TPB, 0, s>>>(a, cur, seed, eps);
+  k_sparse_restore<<<a.NBS, TPB, 0, s>>>(a, cur, seed, eps, use_z && a.zbuf);
 }
 
 void sparse_shrink(const MaskArgs& a, int cur, uint32_t* d_total, cudaStream_t s) {

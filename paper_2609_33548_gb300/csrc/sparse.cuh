@@ -44,6 +44,9 @@ struct MaskArgs {
   unsigned long long* grp_tie0; // [P] ties before the first dense block of each group
   float* xi0p;                  // [P] xi_0 of each projection (Eq. 5)
   uint32_t *blk_a, *blk_b, *blk_c, *blk_d;   // per-block scratch
+  float* zbuf;                  // [k_cap] z of the active weights of the current direction, in
+                                // store order (written by the perturbation sums), or null: every
+                                // pass regenerates z
   uint32_t sup_cap;             // entries idx[1] / lat[1] hold (the superset of mask_build_fast)
   unsigned long long* scan_state; // [NBD] decoupled look-back words of the superset compaction
   uint32_t* sup;                // [4] superset size, overflow flag, block ticket, unused
@@ -64,7 +67,9 @@ void mask_build_fast(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_
 void mask_build_fast_offsets(const MaskArgs& a, uint64_t k0, cudaStream_t s);
 void mask_finish(const MaskArgs& a, cudaStream_t s);
 void sparse_pm_taus(const MaskArgs& a, int cur, uint64_t seed, float eps, cudaStream_t s);
-void sparse_requant(const MaskArgs& a, int cur, uint64_t seed, float eps, int sign, cudaStream_t s);
+// use_z: read z from zbuf (filled by sparse_pm_taus for this seed and store
+// order) instead of regenerating it.
+void sparse_requant(const MaskArgs& a, int cur, uint64_t seed, float eps, int sign, bool use_z, cudaStream_t s);
 // Directions of one step (Algorithm 1 with K <= KMAX perturbations).
 constexpr int KMAX = 8;
 struct UpdateDirs {
@@ -91,13 +96,13 @@ void theta_pm(const ThetaArgs& t, uint64_t seed, float eps, int mode, cudaStream
 void theta_update(const ThetaArgs& t, const UpdateDirs& d, float eps, float lr, const double* g_dev, cudaStream_t s);
 
 // Restore after direction seed: w = fl(fl(fl(w + e) - 2 e) + e), e = fl(eps z).
-void sparse_restore(const MaskArgs& a, int cur, uint64_t seed, float eps, cudaStream_t s);
+void sparse_restore(const MaskArgs& a, int cur, uint64_t seed, float eps, bool use_z, cudaStream_t s);
 // Restore after the last direction, then w = fl(w - fl(c_k z_k)) for k = 0..K-1
 // with c_k = (float)((lr / K) g_k), g_k = g_dev[k]; exact sums of the result.
 void sparse_update_dirs(const MaskArgs& a, int cur, const UpdateDirs& d, float eps, float lr, const double* g_dev,
-                        cudaStream_t s);
+                        bool use_z, cudaStream_t s);
 void sparse_update(const MaskArgs& a, int cur, uint64_t seed, float eps, float lr, const double* g_dev,
-                   double g_host, int use_host, cudaStream_t s);
+                   double g_host, int use_host, bool use_z, cudaStream_t s);
 void sparse_shrink(const MaskArgs& a, int cur, uint32_t* d_total, cudaStream_t s);
 void launch_grad(const double* loss, float eps, double* g, cudaStream_t s);
 void launch_normal(uint64_t seed, const uint32_t* idx, uint64_t n, float* z, cudaStream_t s);

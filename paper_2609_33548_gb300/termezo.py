@@ -29,7 +29,7 @@ EXPORTS = (
 class ModelCfg(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in
                 ("layers", "hidden", "heads", "kv_heads", "ffn", "vocab", "seq", "batch",
-                 "loss_mode", "n_labels", "weight_cache")]
+                 "loss_mode", "n_labels", "weight_cache", "z_cache")]
 
 
 class StepOut(ctypes.Structure):
@@ -45,7 +45,7 @@ class StepOut(ctypes.Structure):
 class MemoryOut(ctypes.Structure):
     _fields_ = [(n, ctypes.c_uint64) for n in
                 ("d", "k_cap", "packed", "sparse_index", "sparse_latents", "mask_state", "forward", "workspace",
-                 "theta", "mask_bitmask", "mask_index_list", "weight_cache")]
+                 "theta", "mask_bitmask", "mask_index_list", "weight_cache", "z_cache")]
 
     def as_dict(self):
         return {n: getattr(self, n) for n, _ in self._fields_}
@@ -154,16 +154,17 @@ def _stream(stream=None):
     return ctypes.c_void_p(s.cuda_stream)
 
 
-def make_cfg(cfg, weight_cache: bool = False) -> ModelCfg:
+def make_cfg(cfg, weight_cache: bool = False, z_cache: bool = False) -> ModelCfg:
     """ModelCfg from any object with the ModelConfig attribute names;
-    weight_cache keeps an e4m3 byte per weight for the forward's GEMMs."""
+    weight_cache keeps an e4m3 byte per weight for the forward's GEMMs,
+    z_cache a float per active weight for z between the passes of a step."""
     return ModelCfg(cfg.layers, cfg.hidden, cfg.heads, cfg.kv_heads, cfg.ffn, cfg.vocab, cfg.seq,
-                    cfg.batch, cfg.loss_mode, cfg.n_labels, 1 if weight_cache else 0)
+                    cfg.batch, cfg.loss_mode, cfg.n_labels, 1 if weight_cache else 0, 1 if z_cache else 0)
 
 
-def op_cfg(N: int, K: int, M: int) -> ModelCfg:
+def op_cfg(N: int, K: int, M: int, z_cache: bool = False) -> ModelCfg:
     """Single-projection context: one [N, K] ternary projection, M rows."""
-    return ModelCfg(0, K, 0, 0, N, 0, M, 1, 0, 0)
+    return ModelCfg(0, K, 0, 0, N, 0, M, 1, 0, 0, 0, 1 if z_cache else 0)
 
 
 def termezo_workspace_bytes(cfg: ModelCfg, density: float) -> int:

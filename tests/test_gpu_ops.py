@@ -58,10 +58,12 @@ def test_mask_build_bit_exact(op_latents, density):
     np.testing.assert_array_equal(st["packed"], ternary.pack_codes(ternary.quantize(w, tau_o[0])))
 
 
-def test_perturb_requantize_update(op_latents):
+@pytest.mark.parametrize("zbuf", [False, True], ids=["regenerate-z", "z-buffer"])
+def test_perturb_requantize_update(op_latents, zbuf):
     density, seed, eps, lr, g = 0.01, 1000, np.float32(1e-3), np.float32(1e-3), -5.25
     w = op_latents
-    ctx, _ = _ctx(w, density)
+    ctx = tz.Context(tz.op_cfg(N, K, M, zbuf), density)
+    ctx.termezo_load_params(torch.from_numpy(w).cuda())
     ctx.termezo_build_mask(density)
     reg = otz.single_registry(N, K)
     state = otz.build(w, reg, density)

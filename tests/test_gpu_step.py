@@ -46,20 +46,23 @@ DENSITY, EPS, LR = 0.01, 1e-3, 1e-6
 
 
 # every step test runs with the GEMMs reading packed codes expanded before each
-# GEMM and with the e4m3 weight cache that the sparse kernels keep in step
-@pytest.fixture(scope="module", params=[(synth.TINY, False), (TINY_SFT, False), (synth.TINY, True), (TINY_SFT, True)],
-                ids=["last-token", "token-level", "last-token-cache", "token-level-cache"])
+# GEMM, with the e4m3 weight cache that the sparse kernels keep in step, and
+# with the z buffer that carries z between the passes of a direction
+@pytest.fixture(scope="module", params=[(synth.TINY, False, False), (TINY_SFT, False, False), (synth.TINY, True, False),
+                                        (TINY_SFT, True, False), (synth.TINY, False, True), (TINY_SFT, False, True)],
+                ids=["last-token", "token-level", "last-token-cache", "token-level-cache", "last-token-zbuf",
+                     "token-level-zbuf"])
 def inputs(request):
-    cfg, cache = request.param
+    cfg, cache, zbuf = request.param
     w = synth.latents(cfg)
     emb, gains, head = synth.theta(cfg)
     tok, tgt = synth.batch(cfg)
-    return w, emb, gains, head, tok, tgt, cfg, cache
+    return w, emb, gains, head, tok, tgt, cfg, cache, zbuf
 
 
 def _gpu_ctx(inputs):
-    w, emb, gains, head, tok, tgt, CFG, cache = inputs
-    ctx = tz.Context(tz.make_cfg(CFG, cache), DENSITY)
+    w, emb, gains, head, tok, tgt, CFG, cache, zbuf = inputs
+    ctx = tz.Context(tz.make_cfg(CFG, cache, zbuf), DENSITY)
     dev = [t.cuda() for t in (w, emb, gains, head, tok, tgt)]
     ctx.termezo_load_params(dev[0], dev[1], dev[2], dev[3])
     return ctx, dev
@@ -118,7 +121,7 @@ def test_one_step_matches_oracle(inputs):
     lp = rounding.loss_ensemble(_cfg(inputs), (_split(cp, reg), swp), _theta_np(inputs), n=8).mean(axis=1)
     lm = rounding.loss_ensemble(_cfg(inputs), (_split(cm, reg), swm), _theta_np(inputs), n=8).mean(axis=1)
     ens = (lp - lm) / (2 * float(np.float32(EPS)))
-    name = _cfg(inputs).name + ("-cache" if inputs[7] else "")
+    name = _cfg(inputs).name + ("-cache" if inputs[7] else "") + ("-zbuf" if inputs[8] else "")
     record("step_loss_plus", workload=name, **rounding.summary(out["loss_plus"], rec["loss_plus"], lp))
     record("step_loss_minus", workload=name, **rounding.summary(out["loss_minus"], rec["loss_minus"], lm))
     record("step_g", workload=name, **rounding.summary(out["g"], rec["g"], ens))
@@ -284,7 +287,7 @@ def test_joint_theta_step_matches_oracle(inputs):
     rounding and the bf16 head in all but a rare element that rounds to a
     neighbouring bf16 value."""
     K = 2
-    w0, emb0, gains0, head0, tok, tgt, cfg, _ = inputs
+    w0, emb0, gains0, head0, tok, tgt, cfg, _, _ = inputs
     ctx, dev = _gpu_ctx(inputs)
     ctx.termezo_build_mask(DENSITY)
     reg = otz.registry(cfg)

@@ -66,3 +66,17 @@ def test_weight_cache_part(cfg, density):
     assert m1["workspace"] - m0["workspace"] == m1["weight_cache"] - (m0["forward"] - m1["forward"])
     for k in ("packed", "sparse_index", "sparse_latents", "mask_state", "theta"):
         assert m1[k] == m0[k]
+
+
+@pytest.mark.parametrize("cfg,density", CASES, ids=[f"{c.name}-{d}" for c, d in CASES])
+def test_z_cache_part(cfg, density):
+    """The optional z buffer is one float per active weight of the store's
+    capacity, its own part outside the memory equation."""
+    m0 = tz.termezo_memory(tz.make_cfg(cfg), density)
+    m1 = tz.termezo_memory(tz.make_cfg(cfg, z_cache=True), density)
+    k0 = math.floor(density * cfg.d_lat)
+    assert m0["z_cache"] == 0
+    assert 4 * k0 <= m1["z_cache"] < 4 * k0 + 256
+    assert abs((m1["workspace"] - m0["workspace"]) - m1["z_cache"]) <= 256
+    for k in ("packed", "sparse_index", "sparse_latents", "forward", "theta", "weight_cache"):
+        assert m1[k] == m0[k]
