@@ -614,43 +614,64 @@ __global__ void __launch_bounds__(TPB) k_sparse_restore(MaskArgs a, int cur, uin
 }
 
 // Eq. 5 at tau_cur: marks dropped weights, writes their code at tau_cur,
-// sums their |w| and counts the kept ones per block.
+// sums their |w| and counts the kept ones per block.  The block's indices
+// and latents are staged in shared memory; thread t then owns entries
+// t + TPB u, and the leader of a packed word (its first entry in the
+// segment) rewrites the word when any of its entries was dropped.
 __global__ void __launch_bounds__(TPB) k_shrink_mark(MaskArgs a, int cur) {
+  constexpr int PER = RQ_MAX / TPB;
   __shared__ ExactSum red[TPB / 32];
   __shared__ uint32_t sh[TPB / 32];
+  __shared__ uint32_t si[RQ_MAX];
+  __shared__ float sl[RQ_MAX];
+  __shared__ uint32_t s_prev;
   const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
   const uint32_t* idx = a.idx[cur];
   const float* lat = a.lat[cur];
   const float tau = a.tau_cur[r.proj];
   const float xi0 = a.xi0p[r.proj];
+  const uint32_t n = r.end - r.beg;
+  if (n > RQ_MAX) {  // cannot happen with the host's block plan; recorded, never silent
+    if (threadIdx.x == 0) atomicOr(a.err, ERR_BOUNDS);
+    return;
+  }
   ExactAcc acc;
   ea_zero(acc);
   uint32_t kept = 0, dropped = 0;
-  for (uint32_t e = r.beg + threadIdx.x; e < r.end; e += TPB) {
-    const float w = lat[e];
+  if (threadIdx.x == 0) s_prev = r.beg > r.seg_beg ? idx[r.beg - 1] : 0xFFFFFFFFu;
+  for (uint32_t j = threadIdx.x; j < n; j += TPB) {
+    const float w = lat[r.beg + j];
+    si[j] = idx[r.beg + j];
+    sl[j] = w;
     if (boundary_distance(w, tau) <= xi0) {
       ++kept;
     } else {
       ++dropped;
       ea_add_abs(acc, w);
     }
-    const uint32_t i = idx[e];
-    if (e != r.seg_beg && (idx[e - 1] >> 4) == (i >> 4)) continue;
+  }
+  __syncthreads();
+#pragma unroll 4
+  for (int u = 0; u < PER; ++u) {
+    const uint32_t j = threadIdx.x + u * TPB;  // consecutive threads, consecutive entries
+    if (j >= n) break;
+    const uint32_t i = si[j], prev = j ? si[j - 1] : s_prev;
+    if (prev != 0xFFFFFFFFu && (prev >> 4) == (i >> 4)) continue;  // not the leader
     const uint32_t wi = i >> 4;
-    uint32_t word = a.packed[wi];
-    bool touched = false;
-    for (uint32_t e2 = e; e2 < r.seg_end; ++e2) {
-      const uint32_t i2 = idx[e2];
+    uint32_t set = 0, mask = 0;
+    for (uint32_t e2 = r.beg + j; e2 < r.seg_end; ++e2) {
+      const bool in_block = e2 < r.end;
+      const uint32_t i2 = in_block ? si[e2 - r.beg] : idx[e2];
       if ((i2 >> 4) != wi) break;
-      const float w2 = lat[e2];
+      const float w2 = in_block ? sl[e2 - r.beg] : lat[e2];
       if (boundary_distance(w2, tau) > xi0) {
         const uint32_t shf = 2 * (i2 & 15u), code = ternary_code(w2, tau);
-        word = (word & ~(3u << shf)) | (code << shf);
+        mask |= 3u << shf;
+        set |= code << shf;
         if (a.wbyte) a.wbyte[i2] = code_e4m3(code);
-        touched = true;
       }
     }
-    if (touched) a.packed[wi] = word;
+    if (mask) a.packed[wi] = (a.packed[wi] & ~mask) | set;
   }
   ExactSum s = ea_result(acc);
   es_block_reduce(s, red);
@@ -689,29 +710,51 @@ __global__ void __launch_bounds__(1024) k_scan_simple(MaskArgs a, uint32_t n, ui
   }
 }
 
+// The kept weights of the block, in order, to the other buffer.  Warp w owns
+// entries 512 w .. 512 w + 511 (lane l: 512 w + 32 u + l, coalesced); a
+// ballot per u ranks the kept entries of 32 consecutive ones, one block scan
+// gives the warps their offsets.
 __global__ void __launch_bounds__(TPB) k_shrink_scatter(MaskArgs a, int cur) {
+  constexpr int PER = RQ_MAX / TPB;
   __shared__ uint32_t sh[TPB / 32];
   const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
   const float tau = a.tau_cur[r.proj];
   const float xi0 = a.xi0p[r.proj];
-  uint32_t pos = a.blk_c[blockIdx.x];
-  for (uint32_t base = r.beg; base < r.end; base += TPB) {
-    const uint32_t e = base + threadIdx.x;
-    bool keep = false;
-    float w = 0.f;
-    uint32_t i = 0;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const uint32_t e0 = r.beg + (uint32_t)warp * 32 * PER + lane;
+  uint32_t iv[PER], keep = 0, cnt = 0;
+  float wv[PER];
+#pragma unroll
+  for (int u = 0; u < PER; ++u) {
+    const uint32_t e = e0 + 32 * u;
+    iv[u] = 0;
+    wv[u] = 0.f;
+    bool k = false;
     if (e < r.end) {
-      w = a.lat[cur][e];
-      i = a.idx[cur][e];
-      keep = boundary_distance(w, tau) <= xi0;
+      wv[u] = a.lat[cur][e];
+      iv[u] = a.idx[cur][e];
+      k = boundary_distance(wv[u], tau) <= xi0;
     }
-    uint32_t tot;
-    const uint32_t rank = block_excl_scan(keep ? 1u : 0u, sh, &tot);
-    if (keep) {
-      a.idx[cur ^ 1][pos + rank] = i;
-      a.lat[cur ^ 1][pos + rank] = w;
+    const uint32_t b = __ballot_sync(0xffffffffu, k);
+    keep |= (k ? 1u : 0u) << u;
+    cnt += __popc(b);  // the warp's kept entries (the same in every lane)
+  }
+  // warp offsets: an exclusive scan of the warps' counts (lane 0's value)
+  uint32_t wcnt = lane == 0 ? cnt : 0u;
+  uint32_t woff = block_excl_scan(wcnt, sh, nullptr);
+  woff = __shfl_sync(0xffffffffu, woff, 0);
+  uint32_t pos = a.blk_c[blockIdx.x] + woff;
+  const uint32_t lt = (1u << lane) - 1u;
+#pragma unroll
+  for (int u = 0; u < PER; ++u) {
+    const bool k = keep & (1u << u);
+    const uint32_t b = __ballot_sync(0xffffffffu, k);
+    if (k) {
+      const uint32_t p = pos + __popc(b & lt);
+      a.idx[cur ^ 1][p] = iv[u];
+      a.lat[cur ^ 1][p] = wv[u];
     }
-    pos += tot;
+    pos += __popc(b);
   }
 }
 
