@@ -13,7 +13,7 @@ last-token loss over 4 label tokens) at mask density 1%.
                   [--workload NAME] [--k-dirs K]
 
 With N > 1 (torchrun) every rank runs an independent replica (the step has
-no cross-GPU exchange in this build); value = tokens of all ranks / max
+no cross-GPU exchange in this library); value = tokens of all ranks / max
 time.  --impl reference times the CPU oracle on a bounded sample of the same
 workload on the host cores.
 """
@@ -217,7 +217,7 @@ class OracleSample:
 
 def memory_report(cfg, density, peak_bytes, weight_cache=False, z_cache=False):
     """Device bytes by part (termezo_memory) next to the memory equation of
-    Sec. 5 evaluated with this build's precisions (B = 4 fp32 latents,
+    Sec. 5 evaluated with this library's precisions (B = 4 fp32 latents,
     B_Q = 1/4, 32-bit active indices), and the peak torch allocation over the
     timed steps (workspace + theta + batches).  The e4m3 weight cache, when
     on, is its own part (d bytes, outside the equation)."""

@@ -93,7 +93,7 @@ int termezo_workspace_bytes(const termezo_model_cfg* cfg, double density, size_t
 /* Device memory of a context, by part (Sec. 5's memory equation): the
  * paper gives the TerMeZO footprint as the MeZO footprint minus
  * d (1 - rho_0)(B - B_Q) plus rho_0 d B_Q plus the mask, M_mask =
- * min(ceil(d / 8), ceil(rho_0 d ceil(log2 d) / 8)).  This build stores the
+ * min(ceil(d / 8), ceil(rho_0 d ceil(log2 d) / 8)).  This library stores the
  * active latents in float32 (B = 4) with 32-bit indices, both in two buffers
  * (the order-preserving shrink writes the second), and every code packed at
  * B_Q = 2/8.  All sizes in bytes; host only, no device call. */

@@ -38,7 +38,7 @@ def test_memory_report_parts(cfg, density):
 
 
 def test_latent_storage_against_the_memory_equation():
-    """Latent-related bytes of the equation with this build's precisions
+    """Latent-related bytes of the equation with this library's precisions
     (B = 4: fp32 latents, B_Q = 1/4, the index list at 32 bits) equal the
     build's packed codes plus one buffer of the sparse store; the second
     buffer (written by the order-preserving shrink) is the only addition."""
