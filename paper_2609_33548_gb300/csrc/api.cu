@@ -122,6 +122,8 @@ struct termezo_ctx {
   uint32_t NBS_max = 0;
   uint32_t* d_total = nullptr;
   std::vector<uint32_t> dpre;
+  std::vector<uint32_t> off_host, spre_host;  // sparse-store offsets read back, block plan uploaded
+  std::vector<uint16_t> sproj_host;
   int cur = 0;
   bool built = false;
   int t = 0;
@@ -584,6 +586,34 @@ void ensure_pm(termezo_ctx* c, uint64_t seed, float eps) {
   c->pm_valid = true;
 }
 
+// Splits each projection's segment of the sparse store (off[p] .. off[p+1])
+// into ceil(count / SPARSE_CHUNK) blocks, at least one, and uploads that plan
+// (spre, sproj) for the sparse kernels, which split each segment evenly over
+// its blocks from the offsets on the device.  The mask only shrinks, so a plan
+// made from earlier counts keeps every block at most SPARSE_CHUNK long; the
+// step re-plans after each read-back so that the blocks stay full as the
+// active set shrinks.  Every per-block result (exact sums, counts, the words
+// rewritten by their leaders) is independent of the partition.
+int plan_sparse_blocks(termezo_ctx* c, const uint32_t* off) {
+  const int P = c->sh.P;
+  std::vector<uint32_t>& spre = c->spre_host;
+  spre.assign(P + 1, 0);
+  for (int p = 0; p < P; ++p) {
+    const uint32_t cnt = off[p + 1] - off[p];
+    const uint32_t nb = (cnt + SPARSE_CHUNK - 1) / SPARSE_CHUNK;
+    spre[p + 1] = spre[p] + (nb ? nb : 1);
+  }
+  if (spre[P] > c->NBS_max) return TERMEZO_ECUDA;
+  c->ma.NBS = spre[P];
+  c->sproj_host.resize(spre[P]);
+  for (int p = 0; p < P; ++p)
+    for (uint32_t b = spre[p]; b < spre[p + 1]; ++b) c->sproj_host[b] = (uint16_t)p;
+  cudaMemcpyAsync((void*)c->ma.spre, spre.data(), (P + 1) * sizeof(uint32_t), cudaMemcpyHostToDevice, c->stream);
+  cudaMemcpyAsync((void*)c->ma.sproj, c->sproj_host.data(), spre[P] * sizeof(uint16_t), cudaMemcpyHostToDevice,
+                  c->stream);
+  return cuda_status(c);
+}
+
 int do_shrink(termezo_ctx* c) {
   ProfScope ps(c, 2 + PASS_SHRINK, 3.0 * 8.0 * (double)c->k_active);
   tmz::sparse_shrink(c->ma, c->cur, c->d_total, c->stream);
@@ -816,19 +846,8 @@ int termezo_build_mask_rule(termezo_ctx* c, double density, int32_t rule, uint64
     fprintf(stderr, "termezo: mask build selected %u weights, expected %llu\n", off[s.P], (unsigned long long)k0);
     return TERMEZO_ECUDA;
   }
-  std::vector<uint32_t> spre(s.P + 1, 0);
-  for (int p = 0; p < s.P; ++p) {
-    const uint32_t cnt = off[p + 1] - off[p];
-    uint32_t nb = (cnt + SPARSE_CHUNK - 1) / SPARSE_CHUNK;
-    spre[p + 1] = spre[p] + (nb ? nb : 1);
-  }
-  if (spre[s.P] > c->NBS_max) return TERMEZO_ECUDA;
-  c->ma.NBS = spre[s.P];
-  cudaMemcpyAsync((void*)c->ma.spre, spre.data(), (s.P + 1) * sizeof(uint32_t), cudaMemcpyHostToDevice, st);
-  std::vector<uint16_t> sproj(spre[s.P]);
-  for (int p = 0; p < s.P; ++p)
-    for (uint32_t b = spre[p]; b < spre[p + 1]; ++b) sproj[b] = (uint16_t)p;
-  cudaMemcpyAsync((void*)c->ma.sproj, sproj.data(), sproj.size() * sizeof(uint16_t), cudaMemcpyHostToDevice, st);
+  rc = plan_sparse_blocks(c, off.data());
+  if (rc) return rc;
   tmz::mask_finish(c->ma, st);
   c->cur = 0;
   c->k0 = k0;
@@ -990,12 +1009,17 @@ int step_impl(termezo_ctx* c, const uint64_t* seeds, int K, float eps, float lr,
   cudaMemcpyAsync(h.loss, K > 1 ? c->lossk : c->loss, 2 * K * sizeof(double), cudaMemcpyDeviceToHost, st);
   cudaMemcpyAsync(h.g, c->g, K * sizeof(double), cudaMemcpyDeviceToHost, st);
   cudaMemcpyAsync(h.cnt, c->ma.counters, 5 * sizeof(unsigned long long), cudaMemcpyDeviceToHost, st);
-  cudaMemcpyAsync(&h.k, c->ma.off[c->cur] + c->sh.P, sizeof(uint32_t), cudaMemcpyDeviceToHost, st);
+  c->off_host.resize(c->sh.P + 1);
+  cudaMemcpyAsync(c->off_host.data(), c->ma.off[c->cur], (c->sh.P + 1) * sizeof(uint32_t), cudaMemcpyDeviceToHost,
+                  st);
   if (per_seq_plus)
     cudaMemcpyAsync(per_seq_plus, c->per_seq, c->sh.B * sizeof(double), cudaMemcpyDeviceToHost, st);
   if (per_seq_minus)
     cudaMemcpyAsync(per_seq_minus, c->per_seq + c->sh.B, c->sh.B * sizeof(double), cudaMemcpyDeviceToHost, st);
   rc = sync_status(c);
+  if (rc) return rc;
+  h.k = c->off_host[c->sh.P];
+  rc = plan_sparse_blocks(c, c->off_host.data());
   if (rc) return rc;
   c->updated = true;
   c->t += 1;
