@@ -48,9 +48,13 @@ WORKLOADS = {
     "tiny": (synth.TINY, 0.01),
 }
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-# dense passes over the latents that termezo_build_mask's kernels make
-# (absmean, three radix-histogram passes, count, compaction)
-MASK_BUILD_DENSE_PASSES = 6
+
+def mask_build_dense_passes(d):
+    """Reads of the dense latents that termezo_build_mask's kernels make: the
+    exact sums, the distance histogram (over one block of 4096 in 16 when the
+    model has at least 65536 blocks) and the superset compaction."""
+    return 2 + (1 / 16 if d // 4096 >= 65536 else 1)
+
 # DRAM bytes (read + write) per k_bitlinear_gemm launch, the mean over eight
 # consecutive GEMM launches (two layers, every shape twice) of the 2B-shaped
 # step, from a one-pass ncu capture (profiles/k_bitlinear_gemm_2b_step_dram.md).
@@ -316,7 +320,7 @@ def run_mine(args):
     # the absmean, the distance histogram and the selection; the packed codes
     # and S_0 written) and the bytes of the passes the kernels make
     build_bytes = 3 * 4 * d + d / 4 + 8 * k0
-    build_bytes_kernels = MASK_BUILD_DENSE_PASSES * 4 * d + d / 4 + 8 * k0
+    build_bytes_kernels = mask_build_dense_passes(d) * 4 * d + d / 4 + 8 * k0
     # the dense latents are read only by the mask build: released here, so the
     # footprint measured over the timed steps is the method's (Sec. 5)
     del w

@@ -241,9 +241,10 @@ void carve(termezo_ctx* c, Carver& cv) {
   a.sproj = cv.take<uint16_t>(c->NBS_max);
   cv.sec = SEC_PACKED;
   a.packed = cv.take<uint32_t>(s.d / 16);
-  // The second buffer is followed by k_cap / 16 + 4096 spare entries (mask
-  // state): the three-pass mask build stages its superset of S_0 there.
-  const size_t spare = c->k_cap / 16 + 4096;
+  // The second buffer is followed by k_cap / 8 + 4096 spare entries (mask
+  // state): the fast mask build stages its superset of S_0 there (about k0
+  // (1 + 1/100 + 1/45) plus the sampling margin).
+  const size_t spare = c->k_cap / 8 + 4096;
   for (int i = 0; i < 2; ++i) {
     cv.sec = SEC_INDEX;
     a.idx[i] = cv.take<uint32_t>(c->k_cap);
@@ -812,8 +813,8 @@ int termezo_build_mask_rule(termezo_ctx* c, double density, int32_t rule, uint64
   int rc = TERMEZO_OK;
   bool built_fast = false;
   if (rule == TERMEZO_MASK_GLOBAL && k0 > 0) {
-    // three dense passes (tmz::mask_build_fast); the six-pass build when the
-    // superset of S_0 does not fit its buffer
+    // two dense passes and a sampled one (tmz::mask_build_fast); the six-pass
+    // build when the superset of S_0 misses k0 or does not fit its buffer
     cudaMemsetAsync(c->ma.hist, 0, 8192 * sizeof(unsigned long long), st);
     cudaMemsetAsync(c->ma.sup, 0, 4 * sizeof(uint32_t), st);
     cudaMemsetAsync(c->ma.scan_state, 0, (size_t)c->ma.NBD * sizeof(unsigned long long), st);

@@ -8,6 +8,8 @@
 // segment of the (sorted) active list.  Per-projection sums of |w| are exact
 // (ExactSum), so tau and therefore every ternary code is independent of
 // the order in which blocks are reduced.
+#include <cmath>
+
 #include "common.cuh"
 #include "kernels.cuh"
 #include "sparse.cuh"
@@ -772,20 +774,26 @@ __global__ void k_normal(uint64_t seed, const uint32_t* idx, uint64_t n, float* 
 }
 
 // ------------------------------------------- mask build, three dense passes --
-// The global quantile of Eq. 4 with three reads of the dense latents: (1) the
-// exact absmean sums (k_dense_sum), (2) a fine histogram of the distance keys
-// (13 bits: exponent and 5 mantissa bits, 32 bins an octave) written together
-// with every code at tau_0, (3) the order-preserving compaction of the
-// "superset" -- every weight whose key falls in the k0-th key's fine bin or
-// below -- into the second sparse-store buffer, with a decoupled look-back
-// scan across blocks.  The exact xi_0 and the ties are then resolved on the
-// superset alone (two 9-bit radix passes over the weights of the fine bin,
-// a count, a scan and an order-preserving scatter into S_0).  The superset
-// holds about (1 + 1/32) k0 weights; when it would not fit, the host runs the
+// The global quantile of Eq. 4 with two reads of the dense latents and a
+// sample of a third: (1) the exact absmean sums (k_dense_sum_warp), (2) a fine
+// histogram of the distance keys (13 bits: exponent and 5 mantissa bits, 32
+// bins an octave) over every HIST_SAMPLE-th dense block (every block of a
+// small model), which gives a bin bound holding k0 keys with a margin, (3) the
+// order-preserving compaction of the "superset" -- every weight whose key
+// falls in that bin or below -- into the second sparse-store buffer, with a
+// decoupled look-back scan across blocks, written together with every code
+// at tau_0.  The superset holds every key of those bins, so its own fine
+// histogram gives the exact bin of the k0-th key and the rank within it; the
+// exact xi_0 and the ties are then resolved on the superset alone (two 9-bit
+// radix passes over the weights of that bin, a count, a scan and an
+// order-preserving scatter into S_0).  When the superset holds fewer than k0
+// weights (the sample missed) or does not fit its buffer, the host runs the
 // six-pass build instead.
 
 constexpr int FINE_SHIFT = 18;                 // fine bin = key >> 18 (bit 31 of a distance is 0)
 constexpr int HIST_DB = 16;                    // dense blocks per CTA of the histogram pass
+constexpr uint32_t HIST_SAMPLE = 16;           // the histogram reads one dense block in HIST_SAMPLE ...
+constexpr uint32_t HIST_SAMPLE_MIN = 65536;    // ... when the model has at least this many blocks
 constexpr int SUP_DB = 8;                      // dense blocks per CTA of the superset compaction
 constexpr int SUP_STAGE = 4096;                // superset entries a CTA stages in shared memory
 
@@ -846,18 +854,38 @@ __device__ __forceinline__ int proj_of_index(const MaskArgs& a, uint32_t i) {
   return lo;
 }
 
-// Pass 2: fine distance histogram and the codes of every weight at tau_0,
-// HIST_DB dense blocks per CTA (one flush of the shared histogram).  Thread
-// t reads float4 number q * TPB + t of a block (coalesced); a packed word (16
-// codes) comes from the four threads of a quad.
-__global__ void __launch_bounds__(TPB) k_hist_codes(MaskArgs a, const float* __restrict__ w) {
+// Projections of increasing global indices (a thread's run of the sorted
+// superset): one binary search, then a step forward whenever an index
+// reaches the next projection's base (base[P] = d bounds every index).
+struct ProjWalk {
+  int p;
+  uint64_t next;
+  __device__ __forceinline__ void start(const MaskArgs& a, uint32_t i) {
+    p = proj_of_index(a, i);
+    next = a.base[p + 1];
+  }
+  __device__ __forceinline__ int at(const MaskArgs& a, uint32_t i) {
+    while ((uint64_t)i >= next) next = a.base[++p + 1];
+    return p;
+  }
+};
+
+// Dense blocks read by the histogram pass: b = stride j + stride / 2.
+__host__ __device__ __forceinline__ uint32_t sampled_blocks(uint32_t nbd, uint32_t stride) {
+  return nbd > stride / 2 ? (nbd - stride / 2 + stride - 1) / stride : 0u;
+}
+
+// Pass 2: fine distance histogram of the sampled dense blocks, HIST_DB of them
+// per CTA (one flush of the shared histogram).  Thread t reads float4 number
+// q * TPB + t of a block (coalesced).
+__global__ void __launch_bounds__(TPB) k_hist_fine(MaskArgs a, const float* __restrict__ w, uint32_t stride) {
   __shared__ uint32_t h[FINE_BINS];
   for (int i = threadIdx.x; i < FINE_BINS; i += TPB) h[i] = 0;
   __syncthreads();
-  const int lane = threadIdx.x & 31;
-  const uint32_t b0 = blockIdx.x * HIST_DB, b1 = min(a.NBD, b0 + HIST_DB);
-  for (uint32_t b = b0; b < b1; ++b) {
-    const DenseRange r = dense_range(a, b);
+  const uint32_t ns = sampled_blocks(a.NBD, stride);
+  const uint32_t j0 = blockIdx.x * HIST_DB, j1 = min(ns, j0 + HIST_DB);
+  for (uint32_t j = j0; j < j1; ++j) {
+    const DenseRange r = dense_range(a, j * stride + stride / 2);
     const float tau = a.tau_cur[r.proj];
     float4 t[4];
 #pragma unroll
@@ -868,22 +896,12 @@ __global__ void __launch_bounds__(TPB) k_hist_codes(MaskArgs a, const float* __r
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       const uint64_t i = r.start + 4ull * (q * TPB + threadIdx.x);
-      const bool live = i < r.end;  // uniform over a quad (chunk lengths are multiples of 16)
-      const float v[4] = {t[q].x, t[q].y, t[q].z, t[q].w};
-      uint32_t byte = 0;
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        if (live) atomicAdd(&h[dist_key(v[e], tau) >> FINE_SHIFT], 1u);
-        byte |= ternary_code(v[e], tau) << (2 * e);
+      if (i < r.end) {
+        atomicAdd(&h[dist_key(t[q].x, tau) >> FINE_SHIFT], 1u);
+        atomicAdd(&h[dist_key(t[q].y, tau) >> FINE_SHIFT], 1u);
+        atomicAdd(&h[dist_key(t[q].z, tau) >> FINE_SHIFT], 1u);
+        atomicAdd(&h[dist_key(t[q].w, tau) >> FINE_SHIFT], 1u);
       }
-      const int q0 = lane & ~3;
-      const uint32_t c0 = __shfl_sync(0xffffffffu, byte, q0), c1 = __shfl_sync(0xffffffffu, byte, q0 + 1);
-      const uint32_t c2 = __shfl_sync(0xffffffffu, byte, q0 + 2), c3 = __shfl_sync(0xffffffffu, byte, q0 + 3);
-      if (live && (lane & 3) == 0) a.packed[i >> 4] = c0 | (c1 << 8) | (c2 << 16) | (c3 << 24);
-      if (live && a.wbyte)
-        *reinterpret_cast<uint32_t*>(a.wbyte + i) = code_e4m3(byte & 3u) | (code_e4m3((byte >> 2) & 3u) << 8) |
-                                                    (code_e4m3((byte >> 4) & 3u) << 16) |
-                                                    (code_e4m3((byte >> 6) & 3u) << 24);
     }
   }
   __syncthreads();
@@ -891,13 +909,16 @@ __global__ void __launch_bounds__(TPB) k_hist_codes(MaskArgs a, const float* __r
     if (h[i]) atomicAdd(&a.hist[i], (unsigned long long)h[i]);
 }
 
-// The bin of `bins` (a.hist[0..bins), bins <= 8192) that holds the krem-th
-// key of group 0; appends its `bits` to the prefix and clears the
-// histogram.  Each thread sums a chunk of bins, thread 0 finds the chunk and
-// then the bin (the chunk's bins loaded at once).  fine != 0 (the first
-// pass): also the superset size (every key below the bin plus the bin) and
-// whether it fits the superset buffer.
-__global__ void __launch_bounds__(256) k_select_fast(MaskArgs a, int bins, int bits, int fine) {
+// The bin of `bins` (a.hist[0..bins), bins <= 8192) that holds the rank-th
+// key, and clears the histogram.  Each thread sums a chunk of bins, thread 0
+// finds the chunk and then the bin (the chunk's bins loaded at once).  Modes:
+// SEL_RADIX appends the bin's `bits` to the prefix and makes krem the rank
+// within it (rank = krem); SEL_FIRST sets the prefix to the bin, likewise;
+// SEL_BOUND sets the prefix to the first bin whose cumulative count reaches
+// `target` (the last bin if none does) and leaves krem.
+enum { SEL_RADIX = 0, SEL_FIRST = 1, SEL_BOUND = 2 };
+__global__ void __launch_bounds__(256) k_select_fast(MaskArgs a, int bins, int bits, int mode,
+                                                     unsigned long long target) {
   constexpr int MAXPER = 32;
   __shared__ unsigned long long csum[256];
   const int per = (bins + 255) / 256;
@@ -910,7 +931,7 @@ __global__ void __launch_bounds__(256) k_select_fast(MaskArgs a, int bins, int b
   __syncthreads();
   if (threadIdx.x == 0 && per <= MAXPER) {
     SelectState* sel = a.sel;
-    const unsigned long long krem = sel->krem;
+    const unsigned long long krem = mode == SEL_BOUND ? target : sel->krem;
     unsigned long long cum = 0;
     int chunk = 255;
     for (int c = 0; c < 256; ++c) {
@@ -926,13 +947,8 @@ __global__ void __launch_bounds__(256) k_select_fast(MaskArgs a, int bins, int b
       if (cum + v[j] >= krem) { B = c0 + j; break; }
       cum += v[j];
     }
-    if (fine) {
-      const unsigned long long n_sup = cum + a.hist[B];
-      a.sup[0] = (uint32_t)(n_sup < 0xFFFFFFFFull ? n_sup : 0xFFFFFFFFull);
-      a.sup[1] = n_sup > (unsigned long long)a.sup_cap ? 1u : 0u;
-    }
-    sel->krem = krem - cum;
-    sel->prefix = fine ? (uint32_t)B : ((sel->prefix << bits) | (uint32_t)B);
+    if (mode != SEL_BOUND) sel->krem = krem - cum;
+    sel->prefix = mode == SEL_RADIX ? ((sel->prefix << bits) | (uint32_t)B) : (uint32_t)B;
   }
   __syncthreads();
   for (int i = threadIdx.x; i < bins; i += blockDim.x) a.hist[i] = 0;
@@ -993,23 +1009,30 @@ __device__ unsigned long long lookback_prefix(const MaskArgs& a, uint32_t b, uin
   return excl;
 }
 
-// Pass 3: every weight whose fine bin is at most the k0-th key's, in index
-// order, into idx[1] / lat[1].  A CTA takes SUP_DB consecutive dense blocks
-// (in ticket order), one per warp.  A warp walks its block in index order
-// (float4 number q * 32 + lane, q-major), ranks its selected weights with warp
-// scans and stages them in its share of shared memory; one barrier gives the
-// warps their offsets, the look-back the CTA's global offset, and the warps
-// copy their weights out.  A warp with more than its share (a dense mask)
-// makes the CTA read its blocks again and write directly.
+// Pass 3: every weight whose fine bin is at most the bound, in index order,
+// into idx[1] / lat[1], and every code at tau_0.  A CTA takes SUP_DB
+// consecutive dense blocks (in ticket order), one per warp.  A warp walks its
+// block in index order (float4 number q * 32 + lane, q-major), ranks its
+// selected weights with four ballots per float4 and stages them in its share
+// of shared memory; one barrier gives the warps their offsets, the look-back
+// the CTA's global offset, and the warps copy their weights out.  A warp with
+// more than its share (a dense mask) makes the CTA read its blocks again and
+// write directly.  The CTA with the last ticket stores the superset's size in
+// sup[0]; entries past the buffer are not written (the size then exceeds
+// sup_cap and the host builds the mask the other way).
 constexpr int SUP_WSTAGE = SUP_STAGE / (TPB / 32);  // staged entries per warp
 
 // One warp's dense block b: the selected weights in index order, staged
-// (stage) or written at out0 + their rank (!stage).  Returns the count.
+// (stage) or written at out0 + their rank (!stage), and with stage the codes
+// of the block (a packed word of 16 codes from the four lanes of a quad).
+// Returns the count.
 __device__ __forceinline__ uint32_t superset_warp(const MaskArgs& a, const float* __restrict__ w, uint32_t b,
                                                   uint32_t bmax, int lane, bool stage, uint32_t* st_idx,
                                                   float* st_lat, unsigned long long out0) {
   const DenseRange r = dense_range(a, b);
   const float tau = a.tau_cur[r.proj];
+  const uint32_t lt = (1u << lane) - 1u;
+  const uint32_t klim = (bmax + 1u) << FINE_SHIFT;  // fine bin <= bmax  <=>  key < klim (bmax < 8192)
   uint32_t run = 0;
   for (int q0 = 0; q0 < (int)(DENSE_CHUNK / 128); q0 += 8) {
     float4 t[8];
@@ -1021,20 +1044,30 @@ __device__ __forceinline__ uint32_t superset_warp(const MaskArgs& a, const float
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
       const uint64_t i = r.start + 4ull * ((q0 + u) * 32 + lane);
+      const bool live = i < r.end;  // uniform over a quad (chunk lengths are multiples of 16)
       const float vv[4] = {t[u].x, t[u].y, t[u].z, t[u].w};
-      uint32_t m = 0;
-      if (i < r.end) {
+      uint32_t m = 0, byte = 0;
+      if (live) {
 #pragma unroll
-        for (int e = 0; e < 4; ++e) m |= ((dist_key(vv[e], tau) >> FINE_SHIFT) <= bmax ? 1u : 0u) << e;
+        for (int e = 0; e < 4; ++e) {
+          m |= (dist_key(vv[e], tau) < klim ? 1u : 0u) << e;
+          byte |= ternary_code(vv[e], tau) << (2 * e);
+        }
       }
-      const uint32_t cnt = __popc(m);
-      uint32_t incl = cnt;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += y;
+      if (stage) {
+        const int qd = lane & ~3;
+        const uint32_t c0 = __shfl_sync(0xffffffffu, byte, qd), c1 = __shfl_sync(0xffffffffu, byte, qd + 1);
+        const uint32_t c2 = __shfl_sync(0xffffffffu, byte, qd + 2), c3 = __shfl_sync(0xffffffffu, byte, qd + 3);
+        if (live && (lane & 3) == 0) a.packed[i >> 4] = c0 | (c1 << 8) | (c2 << 16) | (c3 << 24);
+        if (live && a.wbyte)
+          *reinterpret_cast<uint32_t*>(a.wbyte + i) = code_e4m3(byte & 3u) | (code_e4m3((byte >> 2) & 3u) << 8) |
+                                                      (code_e4m3((byte >> 4) & 3u) << 16) |
+                                                      (code_e4m3((byte >> 6) & 3u) << 24);
       }
-      uint32_t pos = run + incl - cnt;
+      // lane l's four entries follow every selected entry of lanes < l
+      const uint32_t s0 = __ballot_sync(0xffffffffu, m & 1u), s1 = __ballot_sync(0xffffffffu, m & 2u);
+      const uint32_t s2 = __ballot_sync(0xffffffffu, m & 4u), s3 = __ballot_sync(0xffffffffu, m & 8u);
+      uint32_t pos = run + __popc(s0 & lt) + __popc(s1 & lt) + __popc(s2 & lt) + __popc(s3 & lt);
 #pragma unroll
       for (int e = 0; e < 4; ++e)
         if (m & (1u << e)) {
@@ -1043,25 +1076,24 @@ __device__ __forceinline__ uint32_t superset_warp(const MaskArgs& a, const float
               st_idx[pos] = (uint32_t)i + e;
               st_lat[pos] = vv[e];
             }
-          } else if (out0 + pos < a.sup_cap) {  // cannot fail: the size was checked against the capacity
+          } else if (out0 + pos < a.sup_cap) {
             a.idx[1][out0 + pos] = (uint32_t)i + e;
             a.lat[1][out0 + pos] = vv[e];
           }
           ++pos;
         }
-      run += __shfl_sync(0xffffffffu, incl, 31);
+      run += __popc(s0) + __popc(s1) + __popc(s2) + __popc(s3);
     }
   }
   return run;
 }
 
-__global__ void __launch_bounds__(TPB) k_superset(MaskArgs a, const float* __restrict__ w) {
+__global__ void __launch_bounds__(TPB, 4) k_superset(MaskArgs a, const float* __restrict__ w) {
   __shared__ uint32_t s_bid;
   __shared__ unsigned long long s_excl;
   __shared__ uint32_t s_wcnt[TPB / 32];
   __shared__ uint32_t st_idx[SUP_STAGE];
   __shared__ float st_lat[SUP_STAGE];
-  if (a.sup[1]) return;  // the superset does not fit: the host runs the six-pass build
   if (threadIdx.x == 0) s_bid = atomicAdd(&a.sup[2], 1u);
   __syncthreads();
   const uint32_t c = s_bid;
@@ -1082,7 +1114,10 @@ __global__ void __launch_bounds__(TPB) k_superset(MaskArgs a, const float* __res
   }
   if (warp == 0) {
     const unsigned long long e = lookback_prefix(a, c, total, lane);
-    if (lane == 0) s_excl = e;
+    if (lane == 0) {
+      s_excl = e;
+      if (c + 1 == gridDim.x) a.sup[0] = (uint32_t)min(e + total, 0xFFFFFFFFull);
+    }
   }
   __syncthreads();
   const unsigned long long base = s_excl + woff;
@@ -1097,6 +1132,28 @@ __global__ void __launch_bounds__(TPB) k_superset(MaskArgs a, const float* __res
   }
 }
 
+// The fine histogram of the superset's keys (bins 0 .. the bound, all of
+// whose keys it holds), and sup[1] = 1 when the superset holds fewer than k0
+// weights or more than its buffer (nothing after this pass then runs).
+__global__ void __launch_bounds__(TPB) k_sup_hist_fine(MaskArgs a, uint32_t k0) {
+  __shared__ uint32_t h[FINE_BINS];
+  const uint32_t n = a.sup[0];
+  const bool ok = n >= k0 && n <= a.sup_cap;
+  if (blockIdx.x == 0 && threadIdx.x == 0) a.sup[1] = ok ? 0u : 1u;
+  if (!ok) return;  // (uniform)
+  for (int i = threadIdx.x; i < FINE_BINS; i += TPB) h[i] = 0;
+  __syncthreads();
+  // grid-stride over the entries (coalesced); each thread's indices increase
+  const uint32_t e0 = blockIdx.x * TPB + threadIdx.x, step = gridDim.x * TPB;
+  ProjWalk pw;
+  if (e0 < n) pw.start(a, a.idx[1][e0]);
+  for (uint32_t e = e0; e < n; e += step)
+    atomicAdd(&h[dist_key(a.lat[1][e], a.tau_cur[pw.at(a, a.idx[1][e])]) >> FINE_SHIFT], 1u);
+  __syncthreads();
+  for (int i = threadIdx.x; i < FINE_BINS; i += TPB)
+    if (h[i]) atomicAdd(&a.hist[i], (unsigned long long)h[i]);
+}
+
 // Radix passes over the superset's weights in the fine bin: pass 1 keys
 // bits 17..9 of those in bin prefix, pass 2 bits 8..0 of those whose top 23
 // bits match the prefix.
@@ -1106,9 +1163,11 @@ __global__ void __launch_bounds__(TPB) k_sup_hist(MaskArgs a, int pass) {
   __syncthreads();
   const bool live = !a.sup[1];
   const uint32_t n = a.sup[0], prefix = a.sel->prefix;
-  for (uint32_t e = blockIdx.x * TPB + threadIdx.x; live && e < n; e += gridDim.x * TPB) {
-    const uint32_t i = a.idx[1][e];
-    const uint32_t key = dist_key(a.lat[1][e], a.tau_cur[proj_of_index(a, i)]);
+  const uint32_t e0 = blockIdx.x * TPB + threadIdx.x, step = gridDim.x * TPB;
+  ProjWalk pw;
+  if (live && e0 < n) pw.start(a, a.idx[1][e0]);
+  for (uint32_t e = e0; live && e < n; e += step) {
+    const uint32_t key = dist_key(a.lat[1][e], a.tau_cur[pw.at(a, a.idx[1][e])]);
     if (pass == 1 && (key >> FINE_SHIFT) == prefix) atomicAdd(&h[(key >> 9) & 511u], 1u);
     if (pass == 2 && (key >> 9) == prefix) atomicAdd(&h[key & 511u], 1u);
   }
@@ -1124,8 +1183,10 @@ __global__ void __launch_bounds__(TPB) k_sup_count(MaskArgs a) {
   const uint32_t lo = blockIdx.x * SUP_CHUNK, hi = min(n, lo + SUP_CHUNK);
   if (a.sup[1] || lo >= n) return;  // (uniform) blocks past the superset own no scratch entry
   uint32_t less = 0, eq = 0;
+  ProjWalk pw;
+  if (lo + threadIdx.x < hi) pw.start(a, a.idx[1][lo + threadIdx.x]);
   for (uint32_t e = lo + threadIdx.x; e < hi; e += TPB) {
-    const uint32_t key = dist_key(a.lat[1][e], a.tau_cur[proj_of_index(a, a.idx[1][e])]);
+    const uint32_t key = dist_key(a.lat[1][e], a.tau_cur[pw.at(a, a.idx[1][e])]);
     less += key < key_p;
     eq += key == key_p;
   }
@@ -1169,44 +1230,61 @@ __global__ void __launch_bounds__(1024) k_scan_sup(MaskArgs a) {
   }
 }
 
-// S_0 from the superset, in index order, into idx[0] / lat[0].
+// S_0 from the superset, in index order, into idx[0] / lat[0].  Warp w of a
+// block owns its entries 512 w .. 512 w + 511 (lane l: 512 w + 32 u + l,
+// coalesced); ballots per u rank the ties and then the selected entries of
+// 32 consecutive ones, and two block scans give the warps their offsets.
 __global__ void __launch_bounds__(TPB) k_sup_scatter(MaskArgs a, uint32_t k0) {
+  constexpr int PER = SUP_CHUNK / TPB;
   __shared__ uint32_t sh[TPB / 32];
   const uint32_t n = a.sup[0], key_p = a.sel->prefix;
   const unsigned long long ties = a.sel->krem;
   const uint32_t lo = blockIdx.x * SUP_CHUNK, hi = min(n, lo + SUP_CHUNK);
-  if (a.sup[1] || lo >= n) return;
-  const uint32_t e0 = lo + 16u * threadIdx.x;
-  uint32_t keys[16], eq = 0;
+  if (a.sup[1] || lo >= n) return;  // (uniform)
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const uint32_t lt = (1u << lane) - 1u;
+  const uint32_t e0 = lo + (uint32_t)warp * 32 * PER + lane;
+  uint32_t below = 0, tie = 0, nt = 0;  // bit u: entry e0 + 32 u below / equal to xi_0's key
+  ProjWalk pw;
+  if (e0 < hi) pw.start(a, a.idx[1][e0]);
 #pragma unroll
-  for (int j = 0; j < 16; ++j) {
-    keys[j] = 0xFFFFFFFFu;
-    if (e0 + j < hi) keys[j] = dist_key(a.lat[1][e0 + j], a.tau_cur[proj_of_index(a, a.idx[1][e0 + j])]);
-    eq += keys[j] == key_p;
+  for (int u = 0; u < PER; ++u) {
+    const uint32_t e = e0 + 32u * u;
+    uint32_t key = 0xFFFFFFFFu;
+    if (e < hi) key = dist_key(a.lat[1][e], a.tau_cur[pw.at(a, a.idx[1][e])]);
+    below |= (key < key_p ? 1u : 0u) << u;
+    tie |= (key == key_p ? 1u : 0u) << u;
+    nt += __popc(__ballot_sync(0xffffffffu, key == key_p));
   }
-  unsigned long long tie_rank = (unsigned long long)a.blk_d[blockIdx.x] + block_excl_scan(eq, sh, nullptr);
-  uint32_t selm = 0, nsel = 0;
+  uint32_t t_off = block_excl_scan(lane == 0 ? nt : 0u, sh, nullptr);
+  unsigned long long tr = (unsigned long long)a.blk_d[blockIdx.x] + __shfl_sync(0xffffffffu, t_off, 0);
+  uint32_t selm = 0, ns = 0;
 #pragma unroll
-  for (int j = 0; j < 16; ++j) {
-    bool s = keys[j] < key_p;
-    if (keys[j] == key_p) {
-      s = tie_rank < ties;
-      ++tie_rank;
-    }
-    if (s) { selm |= 1u << j; ++nsel; }
+  for (int u = 0; u < PER; ++u) {
+    const bool t = (tie >> u) & 1u;
+    const uint32_t bt = __ballot_sync(0xffffffffu, t);
+    const bool s = ((below >> u) & 1u) || (t && tr + __popc(bt & lt) < ties);
+    selm |= (s ? 1u : 0u) << u;
+    ns += __popc(__ballot_sync(0xffffffffu, s));
+    tr += __popc(bt);
   }
-  uint32_t pos = a.blk_c[blockIdx.x] + block_excl_scan(nsel, sh, nullptr);
+  const uint32_t s_off = block_excl_scan(lane == 0 ? ns : 0u, sh, nullptr);
+  uint32_t pos = a.blk_c[blockIdx.x] + __shfl_sync(0xffffffffu, s_off, 0);
 #pragma unroll
-  for (int j = 0; j < 16; ++j)
-    if (selm & (1u << j)) {
-      if (pos < k0) {
-        a.idx[0][pos] = a.idx[1][e0 + j];
-        a.lat[0][pos] = a.lat[1][e0 + j];
+  for (int u = 0; u < PER; ++u) {
+    const bool s = (selm >> u) & 1u;
+    const uint32_t bs = __ballot_sync(0xffffffffu, s);
+    if (s) {
+      const uint32_t p = pos + __popc(bs & lt), e = e0 + 32u * u;
+      if (p < k0) {
+        a.idx[0][p] = a.idx[1][e];
+        a.lat[0][p] = a.lat[1][e];
       } else {
         atomicOr(a.err, ERR_BOUNDS);  // more than k0 selected: never silent
       }
-      ++pos;
     }
+    pos += __popc(bs);
+  }
 }
 
 // off[0][p]: entries of S_0 below projection p (binary search of base[p]).
@@ -1243,19 +1321,29 @@ void mask_build(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_t s) 
 }
 
 void mask_build_fast(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_t s) {
-  kernel_launches() += 13;
+  kernel_launches() += 14;
   k_dense_sum_warp<<<(a.NBD + TPB / 32 - 1) / (TPB / 32), TPB, 0, s>>>(a, w);
   k_reduce_proj<<<a.P, TPB, 0, s>>>(a.partials, a.dpre, 1, 0, nullptr, a.base, a.S_total, a.gamma_cur, a.tau_cur,
                                     a.sw_cur);
-  k_hist_codes<<<(a.NBD + HIST_DB - 1) / HIST_DB, TPB, 0, s>>>(a, w);
-  k_select_fast<<<1, 256, 0, s>>>(a, FINE_BINS, 0, 1);
+  // The bound: with every block read, the k0-th key's bin; with a sample of
+  // one block in HIST_SAMPLE, the first bin whose sampled count reaches
+  // (k0 / HIST_SAMPLE) (1 + 1/100) plus eight binomial standard deviations.
+  const uint32_t stride = a.NBD >= HIST_SAMPLE_MIN ? HIST_SAMPLE : 1u;
+  const uint32_t ns = sampled_blocks(a.NBD, stride);
+  const double ks = (double)k0 / stride;
+  const unsigned long long target =
+      stride == 1 ? (unsigned long long)k0 : (unsigned long long)(ks * 1.01 + 8.0 * sqrt(ks) + 64.0);
+  k_hist_fine<<<(ns + HIST_DB - 1) / HIST_DB, TPB, 0, s>>>(a, w, stride);
+  k_select_fast<<<1, 256, 0, s>>>(a, FINE_BINS, 0, SEL_BOUND, target);
   k_superset<<<(a.NBD + SUP_DB - 1) / SUP_DB, TPB, 0, s>>>(a, w);
   const uint32_t nsb = (a.sup_cap + SUP_CHUNK - 1) / SUP_CHUNK;
   const uint32_t nh = nsb < 1024u ? (nsb ? nsb : 1u) : 1024u;
+  k_sup_hist_fine<<<nh < 304u ? nh : 304u, TPB, 0, s>>>(a, (uint32_t)k0);
+  k_select_fast<<<1, 256, 0, s>>>(a, FINE_BINS, 0, SEL_FIRST, 0);
   k_sup_hist<<<nh, TPB, 0, s>>>(a, 1);
-  k_select_fast<<<1, 256, 0, s>>>(a, 512, 9, 0);
+  k_select_fast<<<1, 256, 0, s>>>(a, 512, 9, SEL_RADIX, 0);
   k_sup_hist<<<nh, TPB, 0, s>>>(a, 2);
-  k_select_fast<<<1, 256, 0, s>>>(a, 512, 9, 0);
+  k_select_fast<<<1, 256, 0, s>>>(a, 512, 9, SEL_RADIX, 0);
   k_sup_count<<<nsb ? nsb : 1u, TPB, 0, s>>>(a);
   k_scan_sup<<<1, 1024, 0, s>>>(a);
   k_sup_scatter<<<nsb ? nsb : 1u, TPB, 0, s>>>(a, (uint32_t)k0);

@@ -58,11 +58,12 @@ struct MaskArgs {
 // Selects S_0 (the a.groups groups' select states must hold their k) and
 // writes the sparse store, the codes at tau_0 and xi0p.
 void mask_build(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_t s);
-// The global quantile (groups == 1, 0 < k0) in three dense passes.  hist
-// [8192], sup and scan_state must be zero and sel hold k0.  Afterwards sup[1]
-// != 0 means the superset did not fit in idx[1] / lat[1] and nothing but the
-// codes at tau_0 was written (run mask_build instead); otherwise S_0, xi0p
-// and the codes are written and mask_build_fast_offsets writes off[0].
+// The global quantile (groups == 1, 0 < k0) in two dense passes and a
+// sampled one.  hist [8192], sup and scan_state must be zero and sel hold k0.
+// Afterwards sup[1] != 0 means the superset held fewer than k0 weights or did
+// not fit in idx[1] / lat[1], and nothing but the codes at tau_0 was written
+// (run mask_build instead); otherwise S_0, xi0p and the codes are written and
+// mask_build_fast_offsets writes off[0].
 void mask_build_fast(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_t s);
 void mask_build_fast_offsets(const MaskArgs& a, uint64_t k0, cudaStream_t s);
 void mask_finish(const MaskArgs& a, cudaStream_t s);

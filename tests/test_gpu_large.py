@@ -118,6 +118,33 @@ def test_full_size_mask_requant_and_gemm(name):
         np.testing.assert_array_equal(acc.cpu().numpy()[rows], bitnet.int_matmul(q, codes))
 
 
+@pytest.mark.parametrize("planted", ["near", "far"])
+def test_mask_build_when_the_sampled_histogram_misleads(planted):
+    """A projection of 16384 x 16384 latents has 65536 dense blocks of 4096,
+    so the mask build takes its superset bound from the distance histogram
+    of one block in 16 (blocks 16 j + 8).  Those blocks are planted here:
+    with latents at about tau_0 ("near") the sample overstates the weights
+    close to the threshold 16-fold and the superset holds fewer than k0
+    weights; with latents at 10 tau_0 ("far") it understates them and the
+    superset outgrows its buffer.  Either way the build falls back to the
+    six-pass selection, and S_0, xi_0, tau_0 and every packed code are
+    bit-exact against the oracle."""
+    n, k, density = 16384, 16384, 0.01
+    w = synth.op_latents(n, k, seed=21).numpy().reshape(-1)
+    reg = otz.single_registry(n, k)
+    sampled = w.reshape(-1, 4096)[8::16]           # a view: the sampled blocks
+    rng = np.random.default_rng(5)
+    sign = np.where(rng.random(sampled.shape) < 0.5, -1.0, 1.0)
+    jitter = rng.standard_normal(sampled.shape)
+    for _ in range(2):                             # tau_0 moves a little with the planted values
+        _, tau, _ = otz.thresholds(w, reg)
+        mag = tau[0] * (1.0 + 1e-3 * jitter) if planted == "near" else 10.0 * tau[0] * (1.0 + 0.1 * np.abs(jitter))
+        sampled[...] = (sign * mag).astype(np.float32)
+    ctx = tz.Context(tz.op_cfg(n, k, 128), density)
+    ctx.termezo_load_params(torch.from_numpy(w).cuda())
+    _mask_exact(ctx, w, reg, density)
+
+
 def test_full_size_per_tensor_mask():
     """The per-tensor quantile at the full 2B shape (210 projections, 2.08 G
     latents): k0, every projection's xi_0 and the sorted index list
