@@ -811,28 +811,33 @@ __global__ void __launch_bounds__(TPB) k_dense_sum_warp(MaskArgs a, const float*
   const DenseRange r = dense_range(a, b);
   ExactAcc acc;
   ea_zero(acc);
-  uint64_t fx = 0;
-  auto add = [&](float v) {
+  uint64_t fx0 = 0, fx1 = 0;  // two chains (64 values each: < 2^62)
+  auto add = [&](float v, uint64_t& fx) {
     const uint32_t bits = __float_as_uint(v) & 0x7FFFFFFFu;
     const uint32_t sh = (bits >> 23) - 96u;
     if (sh < 32u)
       fx += (uint64_t)((bits & 0x7FFFFFu) | 0x800000u) << sh;
-    else
+    else if (bits)
       ea_add_abs(acc, v);
   };
-#pragma unroll 8
-  for (int q = 0; q < (int)(DENSE_CHUNK / 128); ++q) {
-    const uint64_t i = r.start + 4ull * (q * 32 + lane);
-    if (i < r.end) {
-      const float4 t = *reinterpret_cast<const float4*>(w + i);
-      add(t.x);
-      add(t.y);
-      add(t.z);
-      add(t.w);
+  // eight float4 loads in flight per lane before they are summed
+  for (int q0 = 0; q0 < (int)(DENSE_CHUNK / 128); q0 += 8) {
+    float4 t[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const uint64_t i = r.start + 4ull * ((q0 + u) * 32 + lane);
+      t[u] = i < r.end ? *reinterpret_cast<const float4*>(w + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      add(t[u].x, fx0);
+      add(t[u].y, fx1);
+      add(t[u].z, fx0);
+      add(t[u].w, fx1);
     }
   }
   ExactSum s = ea_result(acc);
-  s.b[1] += (u128)fx << 32;
+  s.b[1] += (u128)(fx0 + fx1) << 32;
   es_warp_reduce(s);
   if (lane == 0) a.partials[b] = s;
 }
@@ -1054,20 +1059,22 @@ __device__ __forceinline__ uint32_t superset_warp(const MaskArgs& a, const float
           byte |= ternary_code(vv[e], tau) << (2 * e);
         }
       }
-      if (stage) {
-        const int qd = lane & ~3;
-        const uint32_t c0 = __shfl_sync(0xffffffffu, byte, qd), c1 = __shfl_sync(0xffffffffu, byte, qd + 1);
-        const uint32_t c2 = __shfl_sync(0xffffffffu, byte, qd + 2), c3 = __shfl_sync(0xffffffffu, byte, qd + 3);
-        if (live && (lane & 3) == 0) a.packed[i >> 4] = c0 | (c1 << 8) | (c2 << 16) | (c3 << 24);
+      if (stage) {  // lane 4k gathers the bytes of lanes 4k .. 4k + 3
+        const uint32_t h2 = byte | (__shfl_down_sync(0xffffffffu, byte, 1) << 8);
+        const uint32_t wd = h2 | (__shfl_down_sync(0xffffffffu, h2, 2) << 16);
+        if (live && (lane & 3) == 0) a.packed[i >> 4] = wd;
         if (live && a.wbyte)
           *reinterpret_cast<uint32_t*>(a.wbyte + i) = code_e4m3(byte & 3u) | (code_e4m3((byte >> 2) & 3u) << 8) |
                                                       (code_e4m3((byte >> 4) & 3u) << 16) |
                                                       (code_e4m3((byte >> 6) & 3u) << 24);
       }
-      // lane l's four entries follow every selected entry of lanes < l
-      const uint32_t s0 = __ballot_sync(0xffffffffu, m & 1u), s1 = __ballot_sync(0xffffffffu, m & 2u);
-      const uint32_t s2 = __ballot_sync(0xffffffffu, m & 4u), s3 = __ballot_sync(0xffffffffu, m & 8u);
-      uint32_t pos = run + __popc(s0 & lt) + __popc(s1 & lt) + __popc(s2 & lt) + __popc(s3 & lt);
+      if (!__any_sync(0xffffffffu, m)) continue;
+      // lane l's entries follow every selected entry of lanes < l: the
+      // three bits of each lane's count (0 .. 4) by ballot
+      const uint32_t c = __popc(m);
+      const uint32_t s0 = __ballot_sync(0xffffffffu, c & 1u), s1 = __ballot_sync(0xffffffffu, c & 2u);
+      const uint32_t s2 = __ballot_sync(0xffffffffu, c & 4u);
+      uint32_t pos = run + __popc(s0 & lt) + 2u * __popc(s1 & lt) + 4u * __popc(s2 & lt);
 #pragma unroll
       for (int e = 0; e < 4; ++e)
         if (m & (1u << e)) {
@@ -1082,7 +1089,7 @@ __device__ __forceinline__ uint32_t superset_warp(const MaskArgs& a, const float
           }
           ++pos;
         }
-      run += __popc(s0) + __popc(s1) + __popc(s2) + __popc(s3);
+      run += __popc(s0) + 2u * __popc(s1) + 4u * __popc(s2);
     }
   }
   return run;
