@@ -705,6 +705,10 @@ int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspa
   for (float* f : {c->ma.gamma_cur, c->ma.tau_cur, c->ma.sw_cur, c->ma.gamma_plus, c->ma.tau_plus, c->ma.sw_plus,
                    c->ma.gamma_minus, c->ma.tau_minus, c->ma.sw_minus})
     cudaMemsetAsync(f, 0, (s.P + 2) * sizeof(float), st);
+  if (tmz::mask_preload() != cudaSuccess) {
+    delete c;
+    return TERMEZO_ECUDA;
+  }
   if (!s.op) {
     tmz::launch_rope_tables(s.S, s.hd, c->cosb, c->sinb, st);
     const int T = s.T, D = s.D, F = s.F, hq = s.H * s.hd, hkv = s.KV * s.hd;

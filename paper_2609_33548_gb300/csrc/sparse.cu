@@ -1328,7 +1328,7 @@ void mask_build(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_t s) 
 }
 
 void mask_build_fast(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_t s) {
-  kernel_launches() += 14;
+  kernel_launches() += 15;
   k_dense_sum_warp<<<(a.NBD + TPB / 32 - 1) / (TPB / 32), TPB, 0, s>>>(a, w);
   k_reduce_proj<<<a.P, TPB, 0, s>>>(a.partials, a.dpre, 1, 0, nullptr, a.base, a.S_total, a.gamma_cur, a.tau_cur,
                                     a.sw_cur);
@@ -1355,6 +1355,24 @@ void mask_build_fast(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_
   k_scan_sup<<<1, 1024, 0, s>>>(a);
   k_sup_scatter<<<nsb ? nsb : 1u, TPB, 0, s>>>(a, (uint32_t)k0);
   k_xi0<<<1, 256, 0, s>>>(a);
+}
+
+cudaError_t mask_preload() {
+  // CUDA loads a kernel at its first launch; the mask build runs once per
+  // context, so its kernels are loaded here instead of inside the build
+  const void* kernels[] = {(const void*)k_dense_sum_warp, (const void*)k_reduce_proj, (const void*)k_hist_fine,
+                           (const void*)k_select_fast,   (const void*)k_superset,    (const void*)k_sup_hist_fine,
+                           (const void*)k_sup_hist,      (const void*)k_sup_count,   (const void*)k_scan_sup,
+                           (const void*)k_sup_scatter,   (const void*)k_xi0,         (const void*)k_off_search,
+                           (const void*)k_sparse_abs,    (const void*)k_frozen_init, (const void*)k_dense_sum,
+                           (const void*)k_hist,          (const void*)k_select,      (const void*)k_count,
+                           (const void*)k_scan_dense,    (const void*)k_compact,     (const void*)k_dense_offsets};
+  for (const void* k : kernels) {
+    cudaFuncAttributes at;
+    const cudaError_t e = cudaFuncGetAttributes(&at, k);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 void mask_build_fast_offsets(const MaskArgs& a, uint64_t k0, cudaStream_t s) {

@@ -66,6 +66,8 @@ void mask_build(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_t s);
 // mask_build_fast_offsets writes off[0].
 void mask_build_fast(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_t s);
 void mask_build_fast_offsets(const MaskArgs& a, uint64_t k0, cudaStream_t s);
+// Loads every kernel of the mask build (done when a context is created).
+cudaError_t mask_preload();
 void mask_finish(const MaskArgs& a, cudaStream_t s);
 void sparse_pm_taus(const MaskArgs& a, int cur, uint64_t seed, float eps, cudaStream_t s);
 // use_z: read z from zbuf (filled by sparse_pm_taus for this seed and store
