@@ -395,7 +395,7 @@ __device__ __forceinline__ void perturbed(float w, float z, float eps, float* wp
   *wm = __fsub_rn(*wp, __fmul_rn(2.0f, *ee));
 }
 
-__global__ void __launch_bounds__(TPB) k_sparse_pm_sum(MaskArgs a, int cur, uint64_t seed, float eps) {
+__global__ void __launch_bounds__(TPB, 3) k_sparse_pm_sum(MaskArgs a, int cur, uint64_t seed, float eps) {
   __shared__ ExactSum red[TPB / 32];
   const SparseRange r = sparse_range(a, a.off[cur], blockIdx.x);
   ExactAcc ap, am;
@@ -918,10 +918,10 @@ __global__ void __launch_bounds__(TPB) k_hist_fine(MaskArgs a, const float* __re
 // key, and clears the histogram.  Each thread sums a chunk of bins, thread 0
 // finds the chunk and then the bin (the chunk's bins loaded at once).  Modes:
 // SEL_RADIX appends the bin's `bits` to the prefix and makes krem the rank
-// within it (rank = krem); SEL_FIRST sets the prefix to the bin, likewise;
-// SEL_BOUND sets the prefix to the first bin whose cumulative count reaches
-// `target` (the last bin if none does) and leaves krem.
-enum { SEL_RADIX = 0, SEL_FIRST = 1, SEL_BOUND = 2 };
+// within it (rank = krem); SEL_BOUND sets the prefix to the first bin whose
+// cumulative count reaches `target` (the last bin if none does) and leaves
+// krem.
+enum { SEL_RADIX = 0, SEL_BOUND = 1 };
 __global__ void __launch_bounds__(256) k_select_fast(MaskArgs a, int bins, int bits, int mode,
                                                      unsigned long long target) {
   constexpr int MAXPER = 32;
@@ -1026,6 +1026,10 @@ __device__ unsigned long long lookback_prefix(const MaskArgs& a, uint32_t b, uin
 // sup[0]; entries past the buffer are not written (the size then exceeds
 // sup_cap and the host builds the mask the other way).
 constexpr int SUP_WSTAGE = SUP_STAGE / (TPB / 32);  // staged entries per warp
+// The compaction also counts its selected weights by fine bin over the
+// SUP_WIN bins up to the bound (two octaves) and in one count below them:
+// enough to place the k0-th key unless the sample was off about 4-fold.
+constexpr int SUP_WIN = 63;
 
 // One warp's dense block b: the selected weights in index order, staged
 // (stage) or written at out0 + their rank (!stage), and with stage the codes
@@ -1033,11 +1037,12 @@ constexpr int SUP_WSTAGE = SUP_STAGE / (TPB / 32);  // staged entries per warp
 // Returns the count.
 __device__ __forceinline__ uint32_t superset_warp(const MaskArgs& a, const float* __restrict__ w, uint32_t b,
                                                   uint32_t bmax, int lane, bool stage, uint32_t* st_idx,
-                                                  float* st_lat, unsigned long long out0) {
+                                                  float* st_lat, unsigned long long out0, uint32_t* s_win) {
   const DenseRange r = dense_range(a, b);
   const float tau = a.tau_cur[r.proj];
   const uint32_t lt = (1u << lane) - 1u;
   const uint32_t klim = (bmax + 1u) << FINE_SHIFT;  // fine bin <= bmax  <=>  key < klim (bmax < 8192)
+  const uint32_t wlo = bmax >= (uint32_t)(SUP_WIN - 1) ? bmax - (SUP_WIN - 1) : 0u;  // first bin of the window
   uint32_t run = 0;
   for (int q0 = 0; q0 < (int)(DENSE_CHUNK / 128); q0 += 8) {
     float4 t[8];
@@ -1083,6 +1088,8 @@ __device__ __forceinline__ uint32_t superset_warp(const MaskArgs& a, const float
               st_idx[pos] = (uint32_t)i + e;
               st_lat[pos] = vv[e];
             }
+            const uint32_t bin = dist_key(vv[e], tau) >> FINE_SHIFT;  // <= bmax
+            atomicAdd(&s_win[bin >= wlo ? 1u + (bin - wlo) : 0u], 1u);
           } else if (out0 + pos < a.sup_cap) {
             a.idx[1][out0 + pos] = (uint32_t)i + e;
             a.lat[1][out0 + pos] = vv[e];
@@ -1101,7 +1108,9 @@ __global__ void __launch_bounds__(TPB, 4) k_superset(MaskArgs a, const float* __
   __shared__ uint32_t s_wcnt[TPB / 32];
   __shared__ uint32_t st_idx[SUP_STAGE];
   __shared__ float st_lat[SUP_STAGE];
+  __shared__ uint32_t s_win[SUP_WIN + 1];  // [0]: below the window, [1 + j]: its bin j
   if (threadIdx.x == 0) s_bid = atomicAdd(&a.sup[2], 1u);
+  if (threadIdx.x <= SUP_WIN) s_win[threadIdx.x] = 0;
   __syncthreads();
   const uint32_t c = s_bid;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -1109,9 +1118,11 @@ __global__ void __launch_bounds__(TPB, 4) k_superset(MaskArgs a, const float* __
   const uint32_t bmax = a.sel->prefix;
   uint32_t* my_idx = st_idx + warp * SUP_WSTAGE;
   float* my_lat = st_lat + warp * SUP_WSTAGE;
-  const uint32_t n = b < a.NBD ? superset_warp(a, w, b, bmax, lane, true, my_idx, my_lat, 0) : 0u;
+  const uint32_t n = b < a.NBD ? superset_warp(a, w, b, bmax, lane, true, my_idx, my_lat, 0, s_win) : 0u;
   if (lane == 0) s_wcnt[warp] = n;
   __syncthreads();
+  if (threadIdx.x <= SUP_WIN && s_win[threadIdx.x])
+    atomicAdd(&a.hist[threadIdx.x], (unsigned long long)s_win[threadIdx.x]);
   uint32_t woff = 0, total = 0;
   bool fits = true;
   for (int k = 0; k < TPB / 32; ++k) {
@@ -1135,30 +1146,43 @@ __global__ void __launch_bounds__(TPB, 4) k_superset(MaskArgs a, const float* __
         a.lat[1][base + j] = my_lat[j];
       }
   } else if (b < a.NBD) {
-    superset_warp(a, w, b, bmax, lane, false, my_idx, my_lat, base);
+    superset_warp(a, w, b, bmax, lane, false, my_idx, my_lat, base, s_win);
   }
 }
 
-// The fine histogram of the superset's keys (bins 0 .. the bound, all of
-// whose keys it holds), and sup[1] = 1 when the superset holds fewer than k0
-// weights or more than its buffer (nothing after this pass then runs).
-__global__ void __launch_bounds__(TPB) k_sup_hist_fine(MaskArgs a, uint32_t k0) {
-  __shared__ uint32_t h[FINE_BINS];
-  const uint32_t n = a.sup[0];
-  const bool ok = n >= k0 && n <= a.sup_cap;
-  if (blockIdx.x == 0 && threadIdx.x == 0) a.sup[1] = ok ? 0u : 1u;
-  if (!ok) return;  // (uniform)
-  for (int i = threadIdx.x; i < FINE_BINS; i += TPB) h[i] = 0;
+// After the compaction: sup[1] = 1 when the superset holds fewer than k0
+// weights or more than its buffer; otherwise the exact fine bin of the k0-th
+// key from the compaction's window counts (hist[0] below the window, hist[1
+// + j] in its bin j) -- the superset holds every key of those bins -- into
+// the prefix, and the rank within it into krem.  A k0-th key below the
+// window also sets sup[1].  Clears the counts.
+__global__ void k_sup_window(MaskArgs a, uint32_t k0) {
+  if (threadIdx.x == 0) {
+    SelectState* sel = a.sel;
+    const uint32_t n = a.sup[0], bmax = sel->prefix;
+    const uint32_t wlo = bmax >= (uint32_t)(SUP_WIN - 1) ? bmax - (SUP_WIN - 1) : 0u;
+    const unsigned long long krem = sel->krem;
+    bool ok = n >= k0 && n <= a.sup_cap;
+    unsigned long long cum = a.hist[0];
+    int B = -1;
+    if (cum >= krem) ok = false;
+    for (int j = 0; ok && j < SUP_WIN; ++j) {
+      const unsigned long long c = a.hist[1 + j];
+      if (cum + c >= krem) {
+        B = j;
+        break;
+      }
+      cum += c;
+    }
+    ok = ok && B >= 0;
+    if (ok) {
+      sel->krem = krem - cum;
+      sel->prefix = wlo + (uint32_t)B;
+    }
+    a.sup[1] = ok ? 0u : 1u;
+  }
   __syncthreads();
-  // grid-stride over the entries (coalesced); each thread's indices increase
-  const uint32_t e0 = blockIdx.x * TPB + threadIdx.x, step = gridDim.x * TPB;
-  ProjWalk pw;
-  if (e0 < n) pw.start(a, a.idx[1][e0]);
-  for (uint32_t e = e0; e < n; e += step)
-    atomicAdd(&h[dist_key(a.lat[1][e], a.tau_cur[pw.at(a, a.idx[1][e])]) >> FINE_SHIFT], 1u);
-  __syncthreads();
-  for (int i = threadIdx.x; i < FINE_BINS; i += TPB)
-    if (h[i]) atomicAdd(&a.hist[i], (unsigned long long)h[i]);
+  for (int i = threadIdx.x; i <= SUP_WIN; i += blockDim.x) a.hist[i] = 0;
 }
 
 // Radix passes over the superset's weights in the fine bin: pass 1 keys
@@ -1328,7 +1352,7 @@ void mask_build(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_t s) 
 }
 
 void mask_build_fast(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_t s) {
-  kernel_launches() += 15;
+  kernel_launches() += 14;
   k_dense_sum_warp<<<(a.NBD + TPB / 32 - 1) / (TPB / 32), TPB, 0, s>>>(a, w);
   k_reduce_proj<<<a.P, TPB, 0, s>>>(a.partials, a.dpre, 1, 0, nullptr, a.base, a.S_total, a.gamma_cur, a.tau_cur,
                                     a.sw_cur);
@@ -1345,8 +1369,7 @@ void mask_build_fast(const MaskArgs& a, const float* w, uint64_t k0, cudaStream_
   k_superset<<<(a.NBD + SUP_DB - 1) / SUP_DB, TPB, 0, s>>>(a, w);
   const uint32_t nsb = (a.sup_cap + SUP_CHUNK - 1) / SUP_CHUNK;
   const uint32_t nh = nsb < 1024u ? (nsb ? nsb : 1u) : 1024u;
-  k_sup_hist_fine<<<nh < 304u ? nh : 304u, TPB, 0, s>>>(a, (uint32_t)k0);
-  k_select_fast<<<1, 256, 0, s>>>(a, FINE_BINS, 0, SEL_FIRST, 0);
+  k_sup_window<<<1, 64, 0, s>>>(a, (uint32_t)k0);
   k_sup_hist<<<nh, TPB, 0, s>>>(a, 1);
   k_select_fast<<<1, 256, 0, s>>>(a, 512, 9, SEL_RADIX, 0);
   k_sup_hist<<<nh, TPB, 0, s>>>(a, 2);
@@ -1361,7 +1384,7 @@ cudaError_t mask_preload() {
   // CUDA loads a kernel at its first launch; the mask build runs once per
   // context, so its kernels are loaded here instead of inside the build
   const void* kernels[] = {(const void*)k_dense_sum_warp, (const void*)k_reduce_proj, (const void*)k_hist_fine,
-                           (const void*)k_select_fast,   (const void*)k_superset,    (const void*)k_sup_hist_fine,
+                           (const void*)k_select_fast,   (const void*)k_superset,    (const void*)k_sup_window,
                            (const void*)k_sup_hist,      (const void*)k_sup_count,   (const void*)k_scan_sup,
                            (const void*)k_sup_scatter,   (const void*)k_xi0,         (const void*)k_off_search,
                            (const void*)k_sparse_abs,    (const void*)k_frozen_init, (const void*)k_dense_sum,
