@@ -773,7 +773,7 @@ __global__ void k_normal(uint64_t seed, const uint32_t* idx, uint64_t n, float* 
   if (i < n) z[i] = normal_at(seed, idx[i]);
 }
 
-// ------------------------------------------- mask build, three dense passes --
+// -------------------------- mask build, two dense passes and a sampled one --
 // The global quantile of Eq. 4 with two reads of the dense latents and a
 // sample of a third: (1) the exact absmean sums (k_dense_sum_warp), (2) a fine
 // histogram of the distance keys (13 bits: exponent and 5 mantissa bits, 32
@@ -1108,9 +1108,10 @@ __global__ void __launch_bounds__(TPB, 4) k_superset(MaskArgs a, const float* __
   __shared__ uint32_t s_wcnt[TPB / 32];
   __shared__ uint32_t st_idx[SUP_STAGE];
   __shared__ float st_lat[SUP_STAGE];
-  __shared__ uint32_t s_win[SUP_WIN + 1];  // [0]: below the window, [1 + j]: its bin j
+  // per warp: [0] below the window, [1 + j] its bin j (only the warp's own lanes add to its row)
+  __shared__ uint32_t s_win[TPB / 32][SUP_WIN + 1];
   if (threadIdx.x == 0) s_bid = atomicAdd(&a.sup[2], 1u);
-  if (threadIdx.x <= SUP_WIN) s_win[threadIdx.x] = 0;
+  for (int j = threadIdx.x; j < (TPB / 32) * (SUP_WIN + 1); j += TPB) (&s_win[0][0])[j] = 0;
   __syncthreads();
   const uint32_t c = s_bid;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -1118,11 +1119,15 @@ __global__ void __launch_bounds__(TPB, 4) k_superset(MaskArgs a, const float* __
   const uint32_t bmax = a.sel->prefix;
   uint32_t* my_idx = st_idx + warp * SUP_WSTAGE;
   float* my_lat = st_lat + warp * SUP_WSTAGE;
-  const uint32_t n = b < a.NBD ? superset_warp(a, w, b, bmax, lane, true, my_idx, my_lat, 0, s_win) : 0u;
+  const uint32_t n = b < a.NBD ? superset_warp(a, w, b, bmax, lane, true, my_idx, my_lat, 0, s_win[warp]) : 0u;
   if (lane == 0) s_wcnt[warp] = n;
   __syncthreads();
-  if (threadIdx.x <= SUP_WIN && s_win[threadIdx.x])
-    atomicAdd(&a.hist[threadIdx.x], (unsigned long long)s_win[threadIdx.x]);
+  if (threadIdx.x <= SUP_WIN) {
+    uint32_t c = 0;
+#pragma unroll
+    for (int k = 0; k < TPB / 32; ++k) c += s_win[k][threadIdx.x];
+    if (c) atomicAdd(&a.hist[threadIdx.x], (unsigned long long)c);
+  }
   uint32_t woff = 0, total = 0;
   bool fits = true;
   for (int k = 0; k < TPB / 32; ++k) {
@@ -1146,7 +1151,7 @@ __global__ void __launch_bounds__(TPB, 4) k_superset(MaskArgs a, const float* __
         a.lat[1][base + j] = my_lat[j];
       }
   } else if (b < a.NBD) {
-    superset_warp(a, w, b, bmax, lane, false, my_idx, my_lat, base, s_win);
+    superset_warp(a, w, b, bmax, lane, false, my_idx, my_lat, base, s_win[warp]);
   }
 }
 
