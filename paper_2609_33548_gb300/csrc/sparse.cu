@@ -1018,8 +1018,9 @@ __device__ unsigned long long lookback_prefix(const MaskArgs& a, uint32_t b, uin
 // into idx[1] / lat[1], and every code at tau_0.  A CTA takes SUP_DB
 // consecutive dense blocks (in ticket order), one per warp.  A warp walks its
 // block in index order (float4 number q * 32 + lane, q-major), ranks its
-// selected weights with four ballots per float4 and stages them in its share
-// of shared memory; one barrier gives the warps their offsets, the look-back
+// selected weights with three ballots (the bits of each lane's count) per
+// float4 and stages them in its share of shared memory, counting them by bin
+// in its own row; one barrier gives the warps their offsets, the look-back
 // the CTA's global offset, and the warps copy their weights out.  A warp with
 // more than its share (a dense mask) makes the CTA read its blocks again and
 // write directly.  The CTA with the last ticket stores the superset's size in
