@@ -1,7 +1,5 @@
-// Per-token absmax int8 quantisation (with or without RMSNorm) of one row,
-// shared by the stand-alone norm / quant kernels and the GEMM epilogue that
-// quantises the residual stream it has just completed, so that both produce
-// the same codes bit for bit.
+// Per-token absmax int8 quantisation (with or without RMSNorm) of one row by
+// one warp (the norm / quant kernel for rows of up to 3072).
 #pragma once
 
 #include <cstdint>
@@ -31,9 +29,10 @@ __device__ __forceinline__ float code_hi(float q) { return __fmul_rn(floorf(__fm
 // 1e-5) (gain != null) or h_k = x_k; a = max(max|h|, 1e-5); q_k = rint(h_k *
 // (127/a)) stored as its e4m3 pair (qh, ql rows); *deq = a / 127.  Lane l
 // holds float4 number i * 32 + l of the row for i < NV (D <= 128 NV, D % 4
-// == 0); the sum of squares runs over i in order, then a butterfly over the
-// lanes (float4 past the row's end hold zeros and add nothing).  CG: x is read
-// through L2 only (rows other CTAs have just written).
+// == 0); the sum of squares runs as four fused multiply-add chains (one per
+// float4 component) over i in order, added as (x + y) + (z + w), then a
+// butterfly over the lanes (float4 past the row's end hold zeros and add
+// nothing).  CG: x is read through L2 only (rows other CTAs have just written).
 template <int NV, bool CG>
 __device__ __forceinline__ void norm_quant_row(const float* __restrict__ xr, const float* __restrict__ gain, int D,
                                                uint8_t* __restrict__ qh8, uint8_t* __restrict__ ql8,
@@ -48,14 +47,15 @@ __device__ __forceinline__ void norm_quant_row(const float* __restrict__ xr, con
     v[i] = k < D4 ? (CG ? __ldcg(x4 + k) : x4[k]) : make_float4(0.f, 0.f, 0.f, 0.f);
   }
   if (gain) {
-    float ss = 0.f;
+    float sx = 0.f, sy = 0.f, sz = 0.f, sw = 0.f;
 #pragma unroll
     for (int i = 0; i < NV; ++i) {
-      ss = __fadd_rn(ss, __fmul_rn(v[i].x, v[i].x));
-      ss = __fadd_rn(ss, __fmul_rn(v[i].y, v[i].y));
-      ss = __fadd_rn(ss, __fmul_rn(v[i].z, v[i].z));
-      ss = __fadd_rn(ss, __fmul_rn(v[i].w, v[i].w));
+      sx = __fmaf_rn(v[i].x, v[i].x, sx);
+      sy = __fmaf_rn(v[i].y, v[i].y, sy);
+      sz = __fmaf_rn(v[i].z, v[i].z, sz);
+      sw = __fmaf_rn(v[i].w, v[i].w, sw);
     }
+    float ss = __fadd_rn(__fadd_rn(sx, sy), __fadd_rn(sz, sw));
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) ss = __fadd_rn(ss, __shfl_xor_sync(0xffffffffu, ss, o));
     const float r = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(__fdiv_rn(ss, (float)D), 1e-5f)));
