@@ -782,12 +782,13 @@ __global__ void k_normal(uint64_t seed, const uint32_t* idx, uint64_t n, float* 
 // order-preserving compaction of the "superset" -- every weight whose key
 // falls in that bin or below -- into the second sparse-store buffer, with a
 // decoupled look-back scan across blocks, written together with every code
-// at tau_0.  The superset holds every key of those bins, so its own fine
-// histogram gives the exact bin of the k0-th key and the rank within it; the
-// exact xi_0 and the ties are then resolved on the superset alone (two 9-bit
-// radix passes over the weights of that bin, a count, a scan and an
-// order-preserving scatter into S_0).  When the superset holds fewer than k0
-// weights (the sample missed) or does not fit its buffer, the host runs the
+// at tau_0 and counted by fine bin over the two octaves up to the bound.  The
+// superset holds every key of those bins, so the counts give the exact bin of
+// the k0-th key and the rank within it; the exact xi_0 and the ties are then
+// resolved on the superset alone (two 9-bit radix passes over the weights of
+// that bin, a count, a scan and an order-preserving scatter into S_0).  When
+// the superset holds fewer than k0 weights (the sample missed), does not fit
+// its buffer, or the k0-th key lies below the counted bins, the host runs the
 // six-pass build instead.
 
 constexpr int FINE_SHIFT = 18;                 // fine bin = key >> 18 (bit 31 of a distance is 0)
