@@ -63,6 +63,22 @@ def test_rmsnorm_matches_torch():
     np.testing.assert_allclose(bitnet.rmsnorm(x, g), ref.float().numpy(), rtol=1e-6, atol=1e-7)
 
 
+def test_gated_hidden_is_squared_relu_times_up():
+    """relu(g)^2 u (the MLP's gate): against float64 torch within the two
+    float32 roundings, exactly 0 wherever g <= 0, and exact on values whose
+    square and product are representable."""
+    rng = np.random.default_rng(7)
+    g = rng.standard_normal((8, 688)).astype(np.float32)
+    u = rng.standard_normal((8, 688)).astype(np.float32)
+    h = bitnet.gated_hidden(g, u)
+    ref = (F.relu(torch.from_numpy(g).double()) ** 2 * torch.from_numpy(u).double()).numpy()
+    assert np.all(h[g <= 0] == 0)
+    pos = g > 0
+    assert np.all(np.abs(h[pos] - ref[pos]) <= 2.0 ** -23 * np.abs(ref[pos]))
+    exact = bitnet.gated_hidden(np.array([0.5, 3.0, -2.0], np.float32), np.array([3.0, -0.25, 5.0], np.float32))
+    np.testing.assert_array_equal(exact, np.array([0.75, -2.25, 0.0], np.float32))
+
+
 def test_rope_is_complex_rotation():
     rng = np.random.default_rng(4)
     S, nh, hd = 33, 3, 16
