@@ -117,7 +117,10 @@ int termezo_memory(const termezo_model_cfg* cfg, double density, termezo_memory_
 
 /* Creates a context over a caller-owned device workspace of `bytes` bytes
  * (>= termezo_workspace_bytes(cfg, density)); 256-byte aligned.  `stream`
- * is a cudaStream_t.  The workspace must outlive the context. */
+ * is a cudaStream_t.  The workspace must outlive the context.  The kernels
+ * of the mask build are loaded here (CUDA loads a kernel at its first launch
+ * otherwise), so termezo_build_mask's one run is not charged their loading.
+ * Returns TERMEZO_ECUDA when that loading fails. */
 int termezo_create(const termezo_model_cfg* cfg, double density, void* d_workspace,
                    size_t bytes, void* stream, termezo_ctx** out);
 
@@ -220,7 +223,10 @@ int termezo_forward_trace(termezo_ctx* ctx, const int32_t* d_tokens, const int32
  * density: the mask's rho_0 is fixed after build (xi_0 is fixed, Eq. 5); a
  * different value returns TERMEZO_WMASKFIXED and is otherwise ignored.
  * out: host report (required); per_seq_plus / per_seq_minus: host [batch]
- * per-sequence losses of the two passes (nullable).  Synchronises once. */
+ * per-sequence losses of the two passes (nullable).  Synchronises once, at
+ * the end, where it also reads back the active set's per-projection offsets
+ * and re-plans the split of the sparse store into blocks of at most 4096
+ * active weights for the next call (the results do not depend on it). */
 int termezo_step(termezo_ctx* ctx, uint64_t seed, float eps, float lr, double density,
                  const int32_t* d_tokens, const int32_t* d_targets, termezo_step_out* out,
                  double* per_seq_plus, double* per_seq_minus);
