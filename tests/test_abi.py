@@ -55,3 +55,12 @@ def test_null_context_is_rejected_without_a_device():
     assert lib.termezo_build_mask(None, 0.01, None, None) == termezo.EINVAL
     assert lib.termezo_step(None, 1, 1e-3, 1e-6, 0.01, None, None, None, None, None) == termezo.EINVAL
     assert lib.termezo_create(None, 0.01, None, 0, None, None) == termezo.EINVAL
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    """The binding has no host fallback: without the built library it raises
+    rather than computing anything."""
+    monkeypatch.setattr(termezo, "_LIB", None)
+    monkeypatch.setattr(termezo, "library_path", lambda: str(tmp_path / "libtermezo.so"))
+    with pytest.raises(OSError):
+        termezo.load(build_if_missing=False)
